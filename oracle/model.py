@@ -1,0 +1,196 @@
+"""Masked, bidirectional diffusion-LM forward pass (oracle side).
+
+Definition 3 (Sec. 3.1): a masked DLM maps a partially observed window
+S~ over Sigma u {[MASK]} to one distribution over Sigma for every masked
+position, in a single forward pass, and each masked position attends to all
+positions regardless of order (no causal mask).
+
+The paper fixes only "masked, bidirectional, LLaDA backbone" (Sec. 1,
+Sec. 4).  The block used here is a LLaDA-style pre-norm transformer:
+
+    x = E[s]                                     (E has V+1 rows, row V = [MASK])
+    per layer:
+        h = RMSNorm(x) * g_attn
+        q, k, v = h Wq^T, h Wk^T, h Wv^T          (GQA: n_kv_heads <= n_heads)
+        q, k = RoPE(q), RoPE(k)                   (rotate-half pairs (i, i+hd/2))
+        o_h = softmax(q_h k_g^T / sqrt(hd)) v_g   (every position, no mask)
+        x = x + concat(o_h) Wo^T
+        h = RMSNorm(x) * g_ffn
+        x = x + (SiLU(h Wg^T) * (h Wu^T)) Wd^T
+    logits = (RMSNorm(x) * g_final) Whead^T       (V outputs: Sigma only)
+
+Weights are stored [out x in] (row = one output feature).  Arithmetic is
+float64; a tensor that the model stores between operations is rounded to
+its storage dtype at that point:
+
+* bf16 models: weights, E, the normed activations h, q/k/v after RoPE, the
+  attention output and the SwiGLU product are bfloat16; the residual stream
+  x and the logits are float32.
+* f32 models: every stored tensor is float32.
+
+Parity: pinned by closed forms (uniform attention when Wq = Wk = 0,
+logits = head(norm(E[s])) when Wo = Wd = 0, permutation equivariance with
+RoPE frequencies set to zero, GQA == MHA with repeated KV heads, RoPE
+relative-position identity, single-position attention == V).  Against the
+paper's trained LLaDA numbers parity is unpinned (no weights exist here).
+"""
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import weights as W
+
+
+@dataclass(frozen=True)
+class ModelConfig:
+    n_layers: int
+    d: int
+    n_heads: int
+    n_kv_heads: int
+    ffn: int
+    vocab: int
+    dtype: str = "bf16"  # 'f32' | 'bf16'
+    rope_theta: float = 10000.0
+    norm_eps: float = 1e-5
+    seed: int = 0
+
+    @property
+    def head_dim(self):
+        return self.d // self.n_heads
+
+    @property
+    def mask_id(self):
+        return self.vocab
+
+
+# Tensor ids of the counter-based generator (part of the model definition).
+TID_EMBED = 0
+TID_HEAD = 1
+WQ, WK, WV, WO, WGATE, WUP, WDOWN = range(7)
+
+
+def layer_tid(layer, which):
+    return 2 + 8 * layer + which
+
+
+def tensor_shapes(cfg):
+    """Logical shapes, keyed by tensor id."""
+    hd = cfg.head_dim
+    dkv = cfg.n_kv_heads * hd
+    shapes = {TID_EMBED: (cfg.vocab + 1, cfg.d), TID_HEAD: (cfg.vocab, cfg.d)}
+    for l in range(cfg.n_layers):
+        shapes[layer_tid(l, WQ)] = (cfg.d, cfg.d)
+        shapes[layer_tid(l, WK)] = (dkv, cfg.d)
+        shapes[layer_tid(l, WV)] = (dkv, cfg.d)
+        shapes[layer_tid(l, WO)] = (cfg.d, cfg.d)
+        shapes[layer_tid(l, WGATE)] = (cfg.ffn, cfg.d)
+        shapes[layer_tid(l, WUP)] = (cfg.ffn, cfg.d)
+        shapes[layer_tid(l, WDOWN)] = (cfg.d, cfg.ffn)
+    return shapes
+
+
+class Weights:
+    """All parameters of a model as float64 arrays holding storage-dtype values."""
+
+    def __init__(self, cfg, tensors=None):
+        self.cfg = cfg
+        shapes = tensor_shapes(cfg)
+        if tensors is None:
+            tensors = {tid: W.init_tensor(cfg.seed, tid, shp, cfg.dtype) for tid, shp in shapes.items()}
+        self.t = tensors
+        self.g_attn = [np.ones(cfg.d) for _ in range(cfg.n_layers)]
+        self.g_ffn = [np.ones(cfg.d) for _ in range(cfg.n_layers)]
+        self.g_final = np.ones(cfg.d)
+
+    def layer(self, l, which):
+        return self.t[layer_tid(l, which)]
+
+    @property
+    def embed(self):
+        return self.t[TID_EMBED]
+
+    @property
+    def head(self):
+        return self.t[TID_HEAD]
+
+
+def rmsnorm(x, g, eps):
+    """x / sqrt(mean(x^2) + eps) * g, per row."""
+    ms = np.mean(x * x, axis=-1, keepdims=True)
+    return x / np.sqrt(ms + eps) * g
+
+
+def rope(u, n_heads, head_dim, theta):
+    """Rotary embedding, rotate-half pairing, position = row index in the window.
+
+    For each head, pair (i, i + hd/2), i < hd/2, rotates by angle
+    pos * theta^(-2i/hd).  ``theta = inf`` gives the identity (frequency 0).
+    """
+    L = u.shape[0]
+    half = head_dim // 2
+    i = np.arange(half, dtype=np.float64)
+    freq = np.power(float(theta), -2.0 * i / head_dim) if np.isfinite(theta) else np.zeros(half)
+    ang = np.arange(L, dtype=np.float64)[:, None] * freq[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    u = u.reshape(L, n_heads, head_dim)
+    a, b = u[..., :half], u[..., half:]
+    out = np.concatenate([a * c[:, None, :] - b * s[:, None, :], b * c[:, None, :] + a * s[:, None, :]], axis=-1)
+    return out.reshape(L, n_heads * head_dim)
+
+
+def silu(x):
+    return x / (1.0 + np.exp(-x))
+
+
+def attention(q, k, v, n_heads, n_kv_heads, head_dim):
+    """Bidirectional multi-head / grouped-query attention over one window."""
+    L = q.shape[0]
+    group = n_heads // n_kv_heads
+    out = np.empty((L, n_heads * head_dim))
+    scale = 1.0 / np.sqrt(head_dim)
+    for h in range(n_heads):
+        g = h // group
+        qh = q[:, h * head_dim:(h + 1) * head_dim]
+        kg = k[:, g * head_dim:(g + 1) * head_dim]
+        vg = v[:, g * head_dim:(g + 1) * head_dim]
+        s = (qh @ kg.T) * scale
+        s = s - s.max(axis=1, keepdims=True)
+        p = np.exp(s)
+        p /= p.sum(axis=1, keepdims=True)
+        out[:, h * head_dim:(h + 1) * head_dim] = p @ vg
+    return out
+
+
+def hidden(wts, state):
+    """Final normed hidden states [L, d] (the LM head input) for one window."""
+    cfg = wts.cfg
+    rnd = lambda a: W.storage_round(a, cfg.dtype)
+    r32 = W.round_f32
+    hd = cfg.head_dim
+    x = r32(wts.embed[np.asarray(state)])
+    for l in range(cfg.n_layers):
+        h = rnd(rmsnorm(x, wts.g_attn[l], cfg.norm_eps))
+        q = h @ wts.layer(l, WQ).T
+        k = h @ wts.layer(l, WK).T
+        v = h @ wts.layer(l, WV).T
+        q = rnd(rope(q, cfg.n_heads, hd, cfg.rope_theta))
+        k = rnd(rope(k, cfg.n_kv_heads, hd, cfg.rope_theta))
+        v = rnd(v)
+        o = rnd(attention(q, k, v, cfg.n_heads, cfg.n_kv_heads, hd))
+        x = r32(x + o @ wts.layer(l, WO).T)
+        h = rnd(rmsnorm(x, wts.g_ffn[l], cfg.norm_eps))
+        a = rnd(silu(h @ wts.layer(l, WGATE).T) * (h @ wts.layer(l, WUP).T))
+        x = r32(x + a @ wts.layer(l, WDOWN).T)
+    return rnd(rmsnorm(x, wts.g_final, cfg.norm_eps))
+
+
+def forward(wts, state, rows=None):
+    """Logits [len(rows), V] (float32 values in float64) for one window.
+
+    ``state`` holds symbol ids in [0, V] (V = [MASK]); ``rows`` selects the
+    positions whose distributions are needed (default: all).
+    """
+    h = hidden(wts, state)
+    if rows is not None:
+        h = h[np.asarray(rows, dtype=np.int64)]
+    return W.round_f32(h @ wts.head.T)

@@ -1,0 +1,162 @@
+"""Iterative DLM compression pipeline (oracle side), Sec. 3.2.
+
+Starting from the fully masked window S^(0) (no initial context, c = 0,
+Sec. 3.4), each step runs the masked DLM over the current state, turns the
+distributions of the schedule's candidate positions into integer tables,
+lets the commitment schedule (Sec. 3.3) pick positions, codes their true
+symbols in ascending position and reveals them, until the window is
+complete.  The input is cut into non-overlapping windows of ``chunk_len``
+symbols (Sec. 4), each compressed independently into its own stream.
+
+Symbols: bytes when V <= 256, otherwise little-endian uint32 token ids.
+
+``encode_window`` / ``decode_window`` take a ``logits_fn(step, state,
+rows)`` so the same schedule/coder logic runs on the DLM forward
+(``model.forward``) or on externally supplied logits.
+
+Parity: pinned by decode(encode(x)) == x on exhaustive tiny windows and on
+every workload shape, and the coverage constraint sum u_k = n.
+"""
+import numpy as np
+
+from . import container as C
+from . import model as M
+from . import quantizer as Q
+from . import selector as S
+from .coder import Decoder, Encoder
+
+
+class BadInput(ValueError):
+    pass
+
+
+def validate_policy(policy):
+    if policy.kind == S.TOPK_CONF:
+        if policy.k < 1:
+            raise BadInput("top-k policy needs k >= 1")
+    elif policy.kind == S.ENTROPY:
+        if policy.k_min < 1:
+            raise BadInput("entropy policy needs k_min >= 1")
+        if policy.k_max and policy.k_max < policy.k_min:
+            raise BadInput("k_max < k_min")
+    else:
+        raise BadInput("unknown policy kind")
+
+
+def symbols_from_bytes(data, V):
+    if V <= 256:
+        return np.frombuffer(bytes(data), dtype=np.uint8).astype(np.int64)
+    if len(data) % 4:
+        raise BadInput("token input must be a multiple of 4 bytes")
+    s = np.frombuffer(bytes(data), dtype="<u4").astype(np.int64)
+    if s.size and s.max() >= V:
+        raise BadInput("token id >= V")
+    return s
+
+
+def bytes_from_symbols(sym, V):
+    if V <= 256:
+        return np.asarray(sym, dtype=np.uint8).tobytes()
+    return np.asarray(sym, dtype="<u4").tobytes()
+
+
+def _key(qz, policy):
+    return qz["W"] if policy.kind == S.TOPK_CONF else qz["Hq"]
+
+
+def encode_window(symbols, V, logits_fn, policy, P, trace=None):
+    """Compress one window; return ((bits, bytes), steps)."""
+    symbols = np.asarray(symbols, dtype=np.int64)
+    n = symbols.size
+    state = np.full(n, V, dtype=np.int64)
+    enc = Encoder(P)
+    tq = Q.tau_q(policy.tau_bits)
+    step = 0
+    while np.any(state == V):
+        masked = state == V
+        cand = S.candidates(masked, policy)
+        qz = Q.quantize(logits_fn(step, state.copy(), cand), P)
+        key = _key(qz, policy)
+        row = {int(p): i for i, p in enumerate(cand)}
+        sel = S.select(masked, {p: key[i] for p, i in row.items()}, policy, tq)
+        assert sel, "a step must commit at least one position"
+        for p in sel:
+            i, s = row[p], int(symbols[p])
+            enc.encode(int(qz["cdf"][i, s]), int(qz["freq"][i, s]))
+        state[sel] = symbols[sel]
+        if trace is not None:
+            trace.append(list(sel))
+        step += 1
+    return enc.finish(), step
+
+
+def decode_window(stream, n, V, logits_fn, policy, P):
+    """Decompress one window of ``n`` symbols from (bits, bytes)."""
+    bits, data = stream
+    dec = Decoder(data, bits, P)
+    state = np.full(n, V, dtype=np.int64)
+    tq = Q.tau_q(policy.tau_bits)
+    step = 0
+    while np.any(state == V):
+        masked = state == V
+        cand = S.candidates(masked, policy)
+        qz = Q.quantize(logits_fn(step, state.copy(), cand), P)
+        key = _key(qz, policy)
+        row = {int(p): i for i, p in enumerate(cand)}
+        sel = S.select(masked, {p: key[i] for p, i in row.items()}, policy, tq)
+        for p in sel:
+            state[p] = dec.decode(qz["cdf"][row[p]])
+        step += 1
+    return state
+
+
+def model_logits_fn(wts):
+    return lambda step, state, rows: M.forward(wts, state, rows)
+
+
+def compress(wts, data, chunk_len, policy, batch_chunks=1):
+    """Compress ``data`` with the DLM ``wts``; return the container bytes."""
+    cfg = wts.cfg
+    V = cfg.vocab
+    validate_policy(policy)
+    if chunk_len < 1:
+        raise BadInput("chunk_len must be >= 1")
+    sym = symbols_from_bytes(data, V)
+    P = Q.precision_for_vocab(V)
+    n = sym.size
+    nchunks = (n + chunk_len - 1) // chunk_len
+    fn = model_logits_fn(wts)
+    streams = []
+    for c in range(nchunks):
+        (bits, byts), _ = encode_window(sym[c * chunk_len:(c + 1) * chunk_len], V, fn, policy, P)
+        streams.append((bits, byts))
+    h = C.Header(P=P, kind=policy.kind, fingerprint=C.fingerprint(cfg), vocab=V, chunk_len=chunk_len,
+                 batch_chunks=batch_chunks, k=policy.k, block=policy.block,
+                 tau_q=Q.tau_q(policy.tau_bits), k_min=policy.k_min, k_max=policy.k_max,
+                 n_symbols=n, n_chunks=nchunks, crc32=C.crc32(bytes(data)))
+    return C.write(h, streams)
+
+
+def policy_from_header(h):
+    return S.Policy(kind=h.kind, k=h.k, block=h.block, tau_bits=h.tau_q / 65536.0, k_min=h.k_min,
+                    k_max=h.k_max)
+
+
+def decompress(wts, blob):
+    cfg = wts.cfg
+    h, streams = C.read(blob)
+    if h.fingerprint != C.fingerprint(cfg):
+        raise C.FingerprintError("container was written with another model")
+    if h.vocab != cfg.vocab:
+        raise C.ContainerError("vocabulary mismatch")
+    policy = policy_from_header(h)
+    fn = model_logits_fn(wts)
+    out = []
+    for c, st in enumerate(streams):
+        n = min(h.chunk_len, h.n_symbols - c * h.chunk_len)
+        out.append(decode_window(st, n, cfg.vocab, fn, policy, h.P))
+    sym = np.concatenate(out) if out else np.zeros(0, dtype=np.int64)
+    data = bytes_from_symbols(sym, cfg.vocab)
+    if C.crc32(data) != h.crc32:
+        raise C.ContainerError("checksum mismatch")
+    return data
