@@ -18,7 +18,8 @@ Details") are stored so the decompressor replays every decision.  Layout
      40   4  k_min      44 4 k_max
      48   8  n_symbols
      56   4  n_chunks
-     60   4  CRC-32 (IEEE) of the original input bytes
+     60   4  checksum: CRC-32 (IEEE) of the little-endian CRC-32s of the
+             windows' input bytes, window by window
      64   -  n_chunks LEB128 varints: bit length of each chunk's stream
       -   -  streams, chunk by chunk, ceil(bits / 8) bytes each
 
@@ -151,3 +152,12 @@ def read(buf):
 
 def crc32(data):
     return zlib.crc32(data) & 0xFFFFFFFF
+
+
+def window_checksum(data, window_bytes):
+    """CRC-32 of the per-window CRC-32s (each little-endian u32)."""
+    if window_bytes == 0:
+        return crc32(b"")
+    crcs = b"".join(struct.pack("<I", crc32(data[i:i + window_bytes]))
+                    for i in range(0, len(data), window_bytes))
+    return crc32(crcs)

@@ -133,7 +133,8 @@ def compress(wts, data, chunk_len, policy, batch_chunks=1):
     h = C.Header(P=P, kind=policy.kind, fingerprint=C.fingerprint(cfg), vocab=V, chunk_len=chunk_len,
                  batch_chunks=batch_chunks, k=policy.k, block=policy.block,
                  tau_q=Q.tau_q(policy.tau_bits), k_min=policy.k_min, k_max=policy.k_max,
-                 n_symbols=n, n_chunks=nchunks, crc32=C.crc32(bytes(data)))
+                 n_symbols=n, n_chunks=nchunks,
+                 crc32=C.window_checksum(bytes(data), chunk_len * (1 if V <= 256 else 4)))
     return C.write(h, streams)
 
 
@@ -157,6 +158,6 @@ def decompress(wts, blob):
         out.append(decode_window(st, n, cfg.vocab, fn, policy, h.P))
     sym = np.concatenate(out) if out else np.zeros(0, dtype=np.int64)
     data = bytes_from_symbols(sym, cfg.vocab)
-    if C.crc32(data) != h.crc32:
+    if C.window_checksum(data, h.chunk_len * (1 if cfg.vocab <= 256 else 4)) != h.crc32:
         raise C.ContainerError("checksum mismatch")
     return data
