@@ -1,0 +1,209 @@
+/*
+ * dlmz.h -- C ABI of the GB300 (sm_103a) diffusion-LM lossless compressor.
+ *
+ * Method: "Diffuse to Compress: Leveraging Diffusion LMs for Lossless
+ * Compression".  A masked, bidirectional diffusion LM (Definition 3,
+ * Sec. 3.1) predicts a distribution for every masked position of a window
+ * in one forward pass; a commitment schedule (Sec. 3.3) picks positions;
+ * their true symbols are entropy coded under the predicted distributions
+ * and revealed as context (iterative pipeline, Sec. 3.2); the input is cut
+ * into non-overlapping windows of size w stored in the header (Sec. 4).
+ *
+ * Conventions for every entry point:
+ *  - Return 0 on success or a negative DLMZ_E* code; dlmz_strerror() names it.
+ *  - "d_" pointers are device pointers (CUDA global memory of the current
+ *    device); other pointers are host pointers.  The caller owns every
+ *    buffer it passes in; the library never frees them.
+ *  - "stream" is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Step-level calls are asynchronous on that stream; whole-file
+ *    calls synchronise it before returning.
+ *  - Device kernels never wait unboundedly: a pipeline wait that exceeds its
+ *    time limit makes the call return DLMZ_ETIMEOUT.
+ *  - A model is immutable after creation and may be shared by sequential
+ *    calls; calls on one model are not thread-safe.
+ */
+#ifndef DLMZ_H
+#define DLMZ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DLMZ_API __attribute__((visibility("default")))
+#else
+#define DLMZ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- error codes ------------------------------------------------------ */
+#define DLMZ_OK 0
+#define DLMZ_EINVAL (-1)      /* bad argument (NULL pointer, zero size, unsupported shape) */
+#define DLMZ_EBADINPUT (-2)   /* input symbols invalid (token id >= V, length not a multiple of 4) */
+#define DLMZ_ECORRUPT (-3)    /* container damaged: magic, version, lengths, stream or checksum */
+#define DLMZ_EMODEL (-4)      /* container written by a different model (fingerprint mismatch) */
+#define DLMZ_ENOMEM (-5)      /* host or device allocation failed */
+#define DLMZ_ECUDA (-6)       /* a CUDA runtime or driver call failed */
+#define DLMZ_ETIMEOUT (-7)    /* a device-side pipeline wait exceeded its limit */
+#define DLMZ_ECAPACITY (-8)   /* caller-provided output buffer too small */
+
+/* ---- model -------------------------------------------------------------- */
+#define DLMZ_FP32 0u
+#define DLMZ_BF16 1u
+
+typedef struct dlmz_model dlmz_model; /* opaque; owns the device weights */
+
+/* LLaDA-style masked DLM (Definition 3): pre-norm blocks of RMSNorm ->
+ * GQA/MHA attention with RoPE (rotate-half, applied to Q and K), no causal
+ * mask -> residual -> RMSNorm -> SwiGLU FFN -> residual; final RMSNorm and
+ * an untied LM head over V symbols.  The embedding has V+1 rows; row V is
+ * [MASK].  d must be a multiple of n_heads, n_heads of n_kv_heads, and the
+ * head dimension even. */
+typedef struct {
+  uint32_t n_layers, d, n_heads, n_kv_heads, ffn, vocab;
+  uint32_t dtype;      /* DLMZ_FP32: all storage float32; DLMZ_BF16: bf16 weights and
+                          activations between kernels, float32 residual stream and logits */
+  float rope_theta;    /* RoPE base (10000) */
+  float norm_eps;      /* RMSNorm epsilon (1e-5) */
+  uint64_t seed;       /* weights ~ N(0, 0.02) from SplitMix64 + Box-Muller of (seed, tensor, index) */
+} dlmz_model_config;
+
+/* Create a randomly initialised model on the current device (trained
+ * weights stand in: Sec. 4 uses LLaDA-8B).  *out receives the handle; on
+ * error *out is NULL.  Errors: EINVAL (shape), ENOMEM, ECUDA. */
+DLMZ_API int dlmz_model_create(const dlmz_model_config* cfg, dlmz_model** out);
+/* Release the model and its device memory.  NULL is accepted. */
+DLMZ_API void dlmz_model_destroy(dlmz_model* m);
+/* FNV-1a 64 of the packed configuration; stored in every container header. */
+DLMZ_API uint64_t dlmz_model_fingerprint(const dlmz_model* m);
+/* Copy the model configuration into *cfg. */
+DLMZ_API int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg);
+
+/* ---- commitment schedule (Sec. 3.3) ---------------------------------- */
+#define DLMZ_TOPK_CONF 0u /* k most confident masked positions of the leftmost incomplete block */
+#define DLMZ_ENTROPY 1u   /* all masked positions with entropy <= tau; at least k_min, at most k_max */
+
+typedef struct {
+  uint32_t kind;
+  uint32_t k;       /* TOPK_CONF: positions per step (>= 1) */
+  uint32_t block;   /* TOPK_CONF: block length; 0 = the whole window */
+  float tau_bits;   /* ENTROPY: threshold tau in bits (entropy base 2) */
+  uint32_t k_min;   /* ENTROPY: m, minimum positions per step (>= 1) */
+  uint32_t k_max;   /* ENTROPY: cap per step; 0 = no cap */
+} dlmz_k_policy;
+
+/* ---- whole-file API, host buffers ------------------------------------ */
+/* Compress in[0, in_bytes) with windows of chunk_len symbols (w, Sec. 4).
+ * Symbols are bytes when V <= 256, otherwise little-endian uint32 token ids
+ * (in_bytes % 4 == 0, each id < V) -- else EBADINPUT.  On success *out is a
+ * malloc'd container of *out_bytes bytes, released with dlmz_free; on error
+ * *out is NULL.  batch_chunks = 0 picks the default batch (<= 1024 windows
+ * per forward batch, bounded by device memory); the value used is stored in
+ * the header so the decoder replays the same batches. */
+DLMZ_API int dlmz_compress(const dlmz_model* m, const void* in, size_t in_bytes, uint32_t chunk_len,
+                  const dlmz_k_policy* policy, uint8_t** out, size_t* out_bytes);
+DLMZ_API int dlmz_compress_ex(const dlmz_model* m, const void* in, size_t in_bytes, uint32_t chunk_len,
+                     const dlmz_k_policy* policy, uint32_t batch_chunks, uint8_t** out,
+                     size_t* out_bytes);
+/* Decompress a container; *out is malloc'd (release with dlmz_free).
+ * Errors: ECORRUPT (header, lengths, streams or CRC-32), EMODEL (fingerprint). */
+DLMZ_API int dlmz_decompress(const dlmz_model* m, const uint8_t* stream, size_t stream_bytes,
+                    uint8_t** out, size_t* out_bytes);
+/* Free a buffer returned by the library.  NULL is accepted. */
+DLMZ_API void dlmz_free(void* p);
+/* Static description of an error code. */
+DLMZ_API const char* dlmz_strerror(int code);
+
+/* ---- whole-file API, device-resident --------------------------------- */
+/* Upper bound of the container size for in_bytes of input. */
+DLMZ_API size_t dlmz_compress_bound(const dlmz_model* m, size_t in_bytes, uint32_t chunk_len);
+/* As dlmz_compress_ex with d_in / d_out in device memory; out_cap is d_out's
+ * capacity (ECAPACITY if too small); *out_bytes is the container size. */
+DLMZ_API int dlmz_compress_device(const dlmz_model* m, const void* d_in, size_t in_bytes, uint32_t chunk_len,
+                         const dlmz_k_policy* policy, uint32_t batch_chunks, uint8_t* d_out,
+                         size_t out_cap, size_t* out_bytes, void* stream);
+/* As dlmz_decompress with d_in / d_out in device memory. */
+DLMZ_API int dlmz_decompress_device(const dlmz_model* m, const uint8_t* d_in, size_t in_bytes,
+                           uint8_t* d_out, size_t out_cap, size_t* out_bytes, void* stream);
+
+/* ---- step-level API (device pointers) ---------------------------------
+ * A batch holds n_chunks windows of equal length L.  "state" is int32
+ * [n_chunks x L] with symbol ids in [0, V] (V = [MASK]).  The LM-head rows
+ * of a step are the positions [row0, row0 + rows_per_chunk) of every window,
+ * row r belonging to window r / rows_per_chunk. */
+
+/* Masked-DLM forward (Definition 3): float32 logits [n_chunks*rows_per_chunk x V]
+ * for positions [row0, row0+rows_per_chunk) of every window of d_state. */
+DLMZ_API int dlmz_forward_logits(const dlmz_model* m, const int32_t* d_state, uint32_t n_chunks,
+                        uint32_t L, uint32_t row0, uint32_t rows_per_chunk, float* d_logits,
+                        void* stream);
+
+/* Dense contraction of the forward (Definition 3's projections and LM head):
+ * d_D [M x N] float32 = d_A [M x K] bf16 . d_B [N x K]^T bf16, all row-major
+ * and contiguous.  Runs on the tcgen05 tensor cores when N % 256 == 0 and
+ * K % 64 == 0 (16-byte aligned operands), else on CUDA cores.  Each output
+ * element's K order is fixed, so results do not depend on M. */
+DLMZ_API int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32_t M, uint32_t N, uint32_t K,
+                            void* stream);
+
+/* Integer quantiser (one rule shared by encoder and decoder): per row of
+ * float32 logits [rows x V], with P CDF bits (V < 2^P, P <= 24):
+ *   m = max, top = lowest argmax; q_v = rint(min(fl(fl(m - l_v) * C), 8191)),
+ *   C = fl32(256 log2 e); w_v = T[q_v & 255] >> (q_v >> 8), T[j] = round(2^31 2^(-j/256));
+ *   W = sum w_v; A = sum w_v q_v; f_v = 1 + floor(w_v (2^P - V) / W), remainder to top;
+ *   Hq = entropy (Sec. 3.3, bits) of w/W in units of 2^-16 bit.
+ * Outputs (any may be NULL except d_W and d_Hq): d_cdf [rows x (V+1)] uint32,
+ * d_W uint64, d_A uint64, d_Hq int32, d_top int32.  Non-finite logits give
+ * EBADINPUT (checked on the device, reported after synchronising). */
+DLMZ_API int dlmz_quantize(const float* d_logits, uint32_t rows, uint32_t V, uint32_t P, uint32_t* d_cdf,
+                  uint64_t* d_W, uint64_t* d_A, int32_t* d_Hq, int32_t* d_top, void* stream);
+
+/* Per group of group_size consecutive rows, the k rows with the smallest
+ * (key, index), written ascending as in-group indices to d_out [groups x k]
+ * (k <= group_size <= 4096).  With keys = Hq this is the entropy top-k of the
+ * isolated quantise+select workload. */
+DLMZ_API int dlmz_select_smallest(const uint64_t* d_keys, uint32_t groups, uint32_t group_size, uint32_t k,
+                         int32_t* d_out, void* stream);
+
+/* Opaque per-batch coder state (range coder, one stream per window). */
+typedef struct dlmz_coder dlmz_coder;
+/* Allocate coder state for n_chunks windows of length L with P-bit tables. */
+DLMZ_API int dlmz_coder_create(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, dlmz_coder** out);
+DLMZ_API void dlmz_coder_destroy(dlmz_coder* c);
+/* Encoder: reset every stream to the empty state.  Decoder: read stream c
+ * from d_bytes + d_offsets[c] (big-endian 16-bit units, d_bits[c] bits long;
+ * bytes past the length read as zero and are never accessed).  The device
+ * buffers must stay valid while decode steps run. */
+DLMZ_API int dlmz_coder_reset_encoder(dlmz_coder* c, void* stream);
+DLMZ_API int dlmz_coder_load_decoder(dlmz_coder* c, const uint8_t* d_bytes, const uint64_t* d_offsets,
+                            const uint32_t* d_bits, void* stream);
+/* One commitment step (Sec. 3.2 / 3.3) on logits of the step's rows:
+ * quantise, select with the policy, code the selected positions in ascending
+ * order into each window's stream (encoder: true symbols from d_symbols
+ * [n_chunks x L]; decoder: decoded) and reveal them in d_state.
+ * d_committed (may be NULL) receives the number of positions committed per
+ * window [n_chunks]. */
+DLMZ_API int dlmz_encode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits,
+                     uint32_t row0, uint32_t rows_per_chunk, const int32_t* d_symbols,
+                     int32_t* d_state, int32_t* d_committed, void* stream);
+DLMZ_API int dlmz_decode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits,
+                     uint32_t row0, uint32_t rows_per_chunk, int32_t* d_state,
+                     int32_t* d_committed, void* stream);
+/* Terminate every stream (call once per encoded batch): bit lengths to
+ * d_bits [n_chunks]; if d_bytes is not NULL each stream's ceil(bits/8) bytes
+ * are copied to d_bytes + d_offsets[c], or to d_bytes + c * 2 *
+ * dlmz_coder_capacity_units() when d_offsets is NULL. */
+DLMZ_API int dlmz_coder_finish(dlmz_coder* c, uint32_t* d_bits, uint8_t* d_bytes, const uint64_t* d_offsets,
+                      void* stream);
+/* Maximum stream size in units per window for this coder. */
+DLMZ_API uint32_t dlmz_coder_capacity_units(const dlmz_coder* c);
+/* Synchronise and report any device-side error flag (ECORRUPT for a stream
+ * that cannot come from the encoder, ETIMEOUT, EBADINPUT). */
+DLMZ_API int dlmz_check(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DLMZ_H */

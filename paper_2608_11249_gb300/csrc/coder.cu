@@ -1,0 +1,377 @@
+// Commitment schedule (Sec. 3.3) and per-window range coding of the
+// committed symbols (statistical coding, Sec. 2.1 / Sec. 4), one
+// independent stream per window.
+//
+// Selection: every schedule here commits the n smallest candidates under
+// (key, position): top-k confidence (key W, n = min(k, #candidates) of the
+// leftmost incomplete block) and the entropy threshold (key H_q, n = #{H_q <=
+// tau} or m if fewer, capped by k_max).  A CTA per window ranks its
+// candidates, so the result does not depend on thread order.
+//
+// Range coder: 64-bit low/range, 16-bit output units stored big-endian,
+// renormalisation below 2^48, carries propagated into the emitted units,
+// minimal termination.  The decoder keeps val = code - low and reads units
+// beyond the stream's length as zero (never past its buffer).
+#include "kernels.cuh"
+#include "coder.cuh"
+#include "exp_table.inc"
+
+namespace dlmz {
+
+static __constant__ uint32_t c_exp_table[256] = DLMZ_EXP_TABLE_INIT;
+
+// ---- selection ----------------------------------------------------------------------
+template <typename K>
+__global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask_id, int row0, int rpc,
+                              const K* __restrict__ keys, int n_rule, int k, int64_t tau_q, int k_min, int k_max,
+                              int kcap, int32_t* __restrict__ sel_count, int32_t* __restrict__ sel_pos) {
+  extern __shared__ uint64_t skey[];  // rpc keys, then rpc flags (as bytes)
+  uint8_t* valid = reinterpret_cast<uint8_t*>(skey + rpc);
+  __shared__ int red[32];
+  __shared__ int s_nsel;
+  const int c = blockIdx.x;
+  int nv = 0, nb = 0;
+  for (int i = threadIdx.x; i < rpc; i += blockDim.x) {
+    const bool ok = state ? state[(size_t)c * L + row0 + i] == mask_id : true;
+    const uint64_t key = (uint64_t)(int64_t)keys[(size_t)c * rpc + i];
+    skey[i] = key;
+    valid[i] = ok;
+    nv += ok;
+    nb += ok && (int64_t)key <= tau_q;
+  }
+  // block sums of nv, nb
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    nv += __shfl_xor_sync(0xffffffffu, nv, o);
+    nb += __shfl_xor_sync(0xffffffffu, nb, o);
+  }
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = nv | (nb << 16);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int tv = 0, tb = 0;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) {
+      tv += red[i] & 0xffff;
+      tb += red[i] >> 16;
+    }
+    int n;
+    if (n_rule == 0) {
+      n = min(k, tv);
+    } else {
+      n = tb < k_min ? min(k_min, tv) : tb;
+      if (k_max > 0 && n > k_max) n = k_max;
+    }
+    s_nsel = min(n, kcap);
+  }
+  __syncthreads();
+  const int nsel = s_nsel;
+  // rank every candidate; selected iff rank < nsel; write ascending positions
+  __shared__ int wcount[32];
+  int base = 0;
+  for (int i0 = 0; i0 < rpc; i0 += blockDim.x) {
+    const int i = i0 + threadIdx.x;
+    bool sel = false;
+    if (i < rpc && valid[i]) {
+      const uint64_t ki = skey[i];
+      int rank = 0;
+      for (int j = 0; j < rpc; ++j)
+        rank += valid[j] && (skey[j] < ki || (skey[j] == ki && j < i));
+      sel = rank < nsel;
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, sel);
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    if (lane == 0) wcount[w] = __popc(bal);
+    __syncthreads();
+    int off = base;
+    for (int j = 0; j < w; ++j) off += wcount[j];
+    if (sel) sel_pos[(size_t)c * kcap + off + __popc(bal & ((1u << lane) - 1))] = row0 + i;
+    int tot = 0;
+    for (int j = 0; j < (int)(blockDim.x >> 5); ++j) tot += wcount[j];
+    base += tot;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) sel_count[c] = nsel;
+}
+
+template <typename K>
+int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0, int rpc, const K* keys, int n_rule,
+                int k, int64_t tau_q, int k_min, int k_max, int kcap, int32_t* sel_count, int32_t* sel_pos,
+                cudaStream_t s) {
+  if (n_chunks == 0) return DLMZ_OK;
+  const size_t smem = (size_t)rpc * 9 + 16;
+  if (smem > 200 * 1024) return DLMZ_EINVAL;
+  static bool attr = false;
+  if (!attr) {
+    DLMZ_CUDA_TRY(cudaFuncSetAttribute(select_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024));
+    attr = true;
+  }
+  select_kernel<K><<<n_chunks, 256, smem, s>>>(state, L, mask_id, row0, rpc, keys, n_rule, k, tau_q, k_min, k_max,
+                                               kcap, sel_count, sel_pos);
+  return launch_status();
+}
+template int select_rows<uint64_t>(const int32_t*, int, int, int, int, int, const uint64_t*, int, int, int64_t, int,
+                                   int, int, int32_t*, int32_t*, cudaStream_t);
+template int select_rows<int32_t>(const int32_t*, int, int, int, int, int, const int32_t*, int, int, int64_t, int,
+                                  int, int, int32_t*, int32_t*, cudaStream_t);
+
+// ---- range coder -----------------------------------------------------------------------
+constexpr uint64_t RENORM = 1ull << 48;
+constexpr int CT = 256;  // threads per window in the coding kernel
+
+__device__ __forceinline__ uint32_t unit_at(const uint8_t* b, uint64_t nbytes, uint32_t i) {
+  const uint64_t o = 2ull * i;
+  uint32_t hi = o < nbytes ? b[o] : 0u;
+  uint32_t lo = o + 1 < nbytes ? b[o + 1] : 0u;
+  return (hi << 8) | lo;
+}
+
+__device__ __forceinline__ void put_unit(uint8_t* b, uint32_t i, uint32_t u) {
+  b[2 * i] = (uint8_t)(u >> 8);
+  b[2 * i + 1] = (uint8_t)u;
+}
+
+__device__ void enc_symbol(CoderState& st, uint8_t* buf, uint32_t cap_units, int P, uint64_t cs, uint64_t fs,
+                           int* err) {
+  const uint64_t r = st.rng >> P;
+  const uint64_t nl = st.low + r * cs;
+  if (nl < st.low) {  // carry into the emitted units
+    int i = (int)st.n_units - 1;
+    for (; i >= 0; --i) {
+      const uint32_t u = ((unit_at(buf, 2ull * cap_units, i) + 1) & 0xFFFFu);
+      put_unit(buf, i, u);
+      if (u) break;
+    }
+    if (i < 0) atomicOr(err, ERR_CORRUPT);
+  }
+  st.low = nl;
+  st.rng = r * fs;
+  while (st.rng < RENORM) {
+    if (st.n_units < cap_units) put_unit(buf, st.n_units, (uint32_t)(st.low >> 48));
+    else atomicOr(err, ERR_CAPACITY);
+    st.n_units++;
+    st.low <<= 16;
+    st.rng <<= 16;
+  }
+}
+
+__device__ __forceinline__ uint64_t block_excl_scan(uint64_t v, uint64_t* wsum, uint64_t* total) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  uint64_t inc = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint64_t t = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += t;
+  }
+  __syncthreads();
+  if (lane == 31) wsum[w] = inc;
+  __syncthreads();
+  uint64_t pre = 0, tot = 0;
+  for (int i = 0; i < nw; ++i) {
+    if (i < w) pre += wsum[i];
+    tot += wsum[i];
+  }
+  *total = tot;
+  return pre + inc - v;
+}
+
+template <bool DECODE>
+__global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
+  __shared__ uint32_t T[256];
+  __shared__ uint64_t wsum[CT / 32];
+  __shared__ uint64_t s_slot, s_cs, s_fs;
+  __shared__ int s_sym;
+  __shared__ CoderState st;
+  for (int i = threadIdx.x; i < 256; i += CT) T[i] = c_exp_table[i];
+  const int c = blockIdx.x;
+  const int n = a.sel_count[c];
+  if (threadIdx.x == 0) st = a.state_c[c];
+  __syncthreads();
+  const int V = a.V, P = a.P;
+  const uint64_t R = (1ull << P) - (uint64_t)V;
+  const int segl = (V + CT - 1) / CT;
+  const int v0 = threadIdx.x * segl, v1 = min(V, v0 + segl);
+  uint8_t* ebuf = a.bytes + (size_t)c * a.cap_bytes;  // encoder stream
+  const uint8_t* dbuf = DECODE ? a.in_bytes + (a.in_offsets ? a.in_offsets[c] : 0) : nullptr;
+  const uint64_t dn = DECODE ? (a.in_bits[c] + 7) / 8 : 0;
+  for (int j = 0; j < n; ++j) {
+    const int pos = a.sel_pos[(size_t)c * a.kcap + j];
+    const size_t row = (size_t)c * a.rpc + (pos - a.row0);
+    const float* lr = a.logits + row * V;
+    const float m = a.mx[row];
+    const uint64_t Wr = a.W[row];
+    const int top = a.top[row];
+    uint64_t sseg = 0;
+    for (int v = v0; v < v1; ++v) {
+      const float x = lr[v];
+      const int q = isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f)) : 8191;
+      sseg += 1 + (uint64_t)(T[q & 255] >> (q >> 8)) * R / Wr;
+    }
+    uint64_t total;
+    const uint64_t pre = block_excl_scan(sseg, wsum, &total);
+    const uint64_t D = (1ull << P) - total;
+    const uint64_t lo = pre + (v0 > top ? D : 0);
+    const uint64_t hi = lo + sseg + (top >= v0 && top < v1 ? D : 0);
+    if (!DECODE) {
+      const int sym = a.symbols[(size_t)c * a.L + pos];
+      if (sym >= v0 && sym < v1) {
+        uint64_t cum = lo;
+        for (int v = v0; v < v1; ++v) {
+          const float x = lr[v];
+          const int q = isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f)) : 8191;
+          const uint64_t f = 1 + (uint64_t)(T[q & 255] >> (q >> 8)) * R / Wr + (v == top ? D : 0);
+          if (v == sym) {
+            s_cs = cum;
+            s_fs = f;
+            break;
+          }
+          cum += f;
+        }
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        CoderState t = st;
+        enc_symbol(t, ebuf, a.cap_bytes / 2, P, s_cs, s_fs, a.err);
+        st = t;
+        a.state[(size_t)c * a.L + pos] = sym;
+      }
+      __syncthreads();
+    } else {
+      if (threadIdx.x == 0) {
+        const uint64_t r = st.rng >> P;
+        uint64_t slot = st.low / r;  // decoder keeps val in .low
+        if (slot >= (1ull << P)) {
+          atomicOr(a.err, ERR_CORRUPT);
+          slot = (1ull << P) - 1;
+        }
+        s_slot = slot;
+      }
+      __syncthreads();
+      const uint64_t slot = s_slot;
+      if (slot >= lo && slot < hi) {
+        uint64_t cum = lo;
+        for (int v = v0; v < v1; ++v) {
+          const float x = lr[v];
+          const int q = isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f)) : 8191;
+          const uint64_t f = 1 + (uint64_t)(T[q & 255] >> (q >> 8)) * R / Wr + (v == top ? D : 0);
+          if (slot < cum + f) {
+            s_sym = v;
+            s_cs = cum;
+            s_fs = f;
+            break;
+          }
+          cum += f;
+        }
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        CoderState t = st;
+        const uint64_t r = t.rng >> P;
+        t.low -= r * s_cs;
+        t.rng = r * s_fs;
+        while (t.rng < RENORM) {
+          t.low = (t.low << 16) | unit_at(dbuf, dn, t.n_units++);
+          t.rng <<= 16;
+        }
+        st = t;
+        a.state[(size_t)c * a.L + pos] = s_sym;
+      }
+      __syncthreads();
+    }
+  }
+  if (threadIdx.x == 0) {
+    a.state_c[c] = st;
+    if (a.committed) a.committed[c] = n;
+  }
+}
+
+int code_step(const CodeArgs& a, bool decode, int n_chunks, cudaStream_t s) {
+  if (n_chunks == 0) return DLMZ_OK;
+  if (decode) code_kernel<true><<<n_chunks, CT, 0, s>>>(a);
+  else code_kernel<false><<<n_chunks, CT, 0, s>>>(a);
+  return launch_status();
+}
+
+__global__ void coder_reset_kernel(CoderState* st, int n) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c < n) {
+    st[c].low = 0;
+    st[c].rng = ~0ull;
+    st[c].n_units = 0;
+  }
+}
+
+__global__ void coder_load_kernel(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets,
+                                  const uint32_t* bits) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n) return;
+  const uint8_t* b = bytes + (offsets ? offsets[c] : 0);
+  const uint64_t nb = (bits[c] + 7) / 8;
+  uint64_t v = 0;
+  for (int i = 0; i < 4; ++i) v = (v << 16) | unit_at(b, nb, i);
+  st[c].low = v;
+  st[c].rng = ~0ull;
+  st[c].n_units = 4;
+}
+
+// Minimal termination: shortest t with a multiple of 2^(64-t) in [low, low+rng).
+__global__ void coder_finish_kernel(CoderState* st, int n, uint8_t* bytes, uint64_t cap_bytes, uint32_t* bits_out,
+                                    uint8_t* out, const uint64_t* offsets, int* err) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n) return;
+  CoderState t = st[c];
+  uint8_t* buf = bytes + (size_t)c * cap_bytes;
+  const unsigned __int128 low = t.low;
+  const unsigned __int128 hi = low + t.rng - 1;
+  unsigned __int128 v = 0;
+  int tb = 0;
+  for (tb = 0; tb <= 64; ++tb) {
+    const unsigned __int128 g = (unsigned __int128)1 << (64 - tb);
+    v = (low + g - 1) / g * g;
+    if (v <= hi) break;
+  }
+  if (v >> 64) {  // carry into the emitted units
+    int i = (int)t.n_units - 1;
+    for (; i >= 0; --i) {
+      const uint32_t u = (unit_at(buf, cap_bytes, i) + 1) & 0xFFFFu;
+      put_unit(buf, i, u);
+      if (u) break;
+    }
+    if (i < 0) atomicOr(err, ERR_CORRUPT);
+  }
+  const uint64_t v64 = (uint64_t)v;
+  const uint32_t nb = (tb + 7) / 8;
+  const uint64_t tail = tb ? (v64 >> (64 - tb)) << (8 * nb - tb) : 0;
+  const uint64_t base = 2ull * t.n_units;
+  if (base + nb > cap_bytes) {
+    atomicOr(err, ERR_CAPACITY);
+  } else {
+    for (uint32_t i = 0; i < nb; ++i) buf[base + i] = (uint8_t)(tail >> (8 * (nb - 1 - i)));
+  }
+  const uint64_t total_bits = 16ull * t.n_units + tb;
+  bits_out[c] = (uint32_t)total_bits;
+  if (out && base + nb <= cap_bytes) {  // copy out: at offsets[c], or at c * cap_bytes
+    const uint64_t nbytes = (total_bits + 7) / 8;
+    uint8_t* dst = out + (offsets ? offsets[c] : (uint64_t)c * cap_bytes);
+    for (uint64_t i = 0; i < nbytes; ++i) dst[i] = buf[i];
+  }
+}
+
+int coder_reset(CoderState* st, int n, cudaStream_t s) {
+  if (!n) return DLMZ_OK;
+  coder_reset_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n);
+  return launch_status();
+}
+int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits,
+               cudaStream_t s) {
+  if (!n) return DLMZ_OK;
+  coder_load_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n, bytes, offsets, bits);
+  return launch_status();
+}
+int coder_finish(CoderState* st, int n, uint8_t* bytes, uint64_t cap_bytes, uint32_t* bits, uint8_t* out,
+                 const uint64_t* offsets, cudaStream_t s) {
+  if (!n) return DLMZ_OK;
+  coder_finish_kernel<<<(n + 127) / 128, 128, 0, s>>>(st, n, bytes, cap_bytes, bits, out, offsets,
+                                                      device_error_word());
+  return launch_status();
+}
+
+}  // namespace dlmz

@@ -1,0 +1,49 @@
+// Coder state and launch helpers of the selection / range-coding step.
+#pragma once
+
+#include "kernels.cuh"
+
+namespace dlmz {
+
+// Per-window range-coder state.  Encoder: low/rng and the count of emitted
+// 16-bit units.  Decoder: `low` holds val = code - low, `n_units` the next
+// unit to read.
+struct CoderState {
+  uint64_t low;
+  uint64_t rng;
+  uint32_t n_units;
+  uint32_t pad;
+};
+
+struct CodeArgs {
+  const float* logits;       // [n_chunks * rpc x V]
+  const float* mx;           // per row: max logit
+  const uint64_t* W;         // per row: W
+  const int32_t* top;        // per row: lowest argmax
+  const int32_t* sel_count;  // [n_chunks]
+  const int32_t* sel_pos;    // [n_chunks x kcap], ascending
+  const int32_t* symbols;    // encoder: true symbols [n_chunks x L]
+  int32_t* state;            // [n_chunks x L]
+  CoderState* state_c;       // [n_chunks]
+  uint8_t* bytes;            // encoder streams [n_chunks x cap_bytes]
+  uint64_t cap_bytes;
+  const uint8_t* in_bytes;   // decoder streams
+  const uint64_t* in_offsets;
+  const uint32_t* in_bits;
+  int32_t* committed;        // optional [n_chunks]
+  int* err;
+  int V, P, L, row0, rpc, kcap;
+};
+
+template <typename K>
+int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0, int rpc, const K* keys, int n_rule,
+                int k, int64_t tau_q, int k_min, int k_max, int kcap, int32_t* sel_count, int32_t* sel_pos,
+                cudaStream_t s);
+int code_step(const CodeArgs& a, bool decode, int n_chunks, cudaStream_t s);
+int coder_reset(CoderState* st, int n, cudaStream_t s);
+int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits,
+               cudaStream_t s);
+int coder_finish(CoderState* st, int n, uint8_t* bytes, uint64_t cap_bytes, uint32_t* bits, uint8_t* out,
+                 const uint64_t* offsets, cudaStream_t s);
+
+}  // namespace dlmz

@@ -1,0 +1,415 @@
+// Dense bf16 GEMM on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+//
+//   D[m, n] = sum_k A[m, k] * B[n, k]      A: [M x K] bf16, B: [N x K] bf16 (both K-major)
+//
+// This is every dense contraction of the masked-DLM forward (Definition 3):
+// the fused QKV projection (with RoPE in the epilogue), the attention output
+// projection and the FFN down projection (residual add into the float32
+// stream), the gate/up projection (SwiGLU in the epilogue) and the LM head
+// (float32 logits).
+//
+// Design (one CTA per SM, persistent over output tiles of 128 x 256):
+//   warp 0      TMA producer: 128B-swizzled A/B K-slices (64 elements) into a
+//               4-stage shared-memory ring, completion on mbarriers.
+//   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
+//               issues tcgen05.mma (M=128, N=256, K=16) from one thread;
+//               tcgen05.commit frees a ring slot / publishes an accumulator.
+//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns per warp (each
+//               thread owns one output row), fused op, vectorised stores.
+// Two accumulators let the epilogue of tile i overlap the MMAs of tile i+1.
+// Every mbarrier wait is bounded; on timeout the CTA sets the error word,
+// waits (bounded) for its own outstanding copies and MMAs, frees TMEM and
+// returns.  Output values depend only on (m, n) and K (fixed K order, no
+// split-K), so results are independent of M and of the batch composition.
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace dlmz {
+namespace tc {
+
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;  // bf16 elements = 128 bytes = one swizzle row
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int THREADS = 192;
+constexpr int TMEM_COLS = 512;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+
+// Instruction descriptor (kind::f16): D f32, A/B bf16, both K-major, M=128, N=256.
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                           ((uint32_t)(BM >> 4) << 24);
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (SBO), descriptor version 1.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFF) >> 4);
+  d |= (uint64_t)1 << 16;             // LBO (unused for swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;   // SBO
+  d |= (uint64_t)1 << 46;             // version
+  d |= (uint64_t)2 << 61;             // SWIZZLE_128B
+  return d;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(IDESC), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%"
+      "15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v) {
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    uint32_t w[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      __nv_bfloat162 p = __floats2bfloat162_rn(v[8 * j + 2 * t], v[8 * j + 2 * t + 1]);
+      w[t] = *reinterpret_cast<uint32_t*>(&p);
+    }
+    d4[j] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void epilogue_tile(uint32_t tacc, int lane_base, int m, int M, int n0,
+                                              const GemmEpilogue& ep) {
+  const bool live = m < M;
+  if constexpr (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID_F32) {
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      float v[32];
+      tmem_ld32(tacc + ((uint32_t)lane_base << 16) + c * 32, v);
+      if (!live) continue;
+      const size_t off = (size_t)m * ep.ldo + n0 + c * 32;
+      if constexpr (EPI == EPI_BF16) {
+        store_bf16x32(reinterpret_cast<__nv_bfloat16*>(ep.out) + off, v);
+      } else if constexpr (EPI == EPI_F32) {
+        float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + off);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) d[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+      } else {
+        float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + off);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 r = d[j];
+          r.x += v[4 * j];
+          r.y += v[4 * j + 1];
+          r.z += v[4 * j + 2];
+          r.w += v[4 * j + 3];
+          d[j] = r;
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU_BF16) {
+    // tile columns [0,128) = gate, [128,256) = up of the same 128 features
+#pragma unroll 1
+    for (int c = 0; c < BN / 64; ++c) {
+      float g[32], u[32];
+      tmem_ld32(tacc + ((uint32_t)lane_base << 16) + c * 32, g);
+      tmem_ld32(tacc + ((uint32_t)lane_base << 16) + BN / 2 + c * 32, u);
+      if (!live) continue;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) g[i] = g[i] / (1.0f + __expf(-g[i])) * u[i];
+      const size_t off = (size_t)m * ep.ldo + (n0 / 2) + c * 32;
+      store_bf16x32(reinterpret_cast<__nv_bfloat16*>(ep.out) + off, g);
+    }
+  } else {  // EPI_ROPE*_BF16: rotate-half RoPE on columns < rope_cols, then bf16
+    constexpr int HD = EPI == EPI_ROPE32_BF16 ? 32 : (EPI == EPI_ROPE64_BF16 ? 64 : 128);
+    constexpr int HALF = HD / 2;
+    const int pos = live ? (m % ep.L) : 0;
+#pragma unroll 1
+    for (int h0 = 0; h0 < BN; h0 += HD) {
+      float v[HD];
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) tmem_ld32(tacc + ((uint32_t)lane_base << 16) + h0 + c * 32, v + 32 * c);
+      if (!live) continue;
+      if (n0 + h0 < ep.rope_cols) {
+        const float2* cs = ep.rope_cs + (size_t)pos * HALF;
+#pragma unroll
+        for (int i = 0; i < HALF; ++i) {
+          float2 t = cs[i];
+          float a = v[i], b = v[i + HALF];
+          v[i] = a * t.x - b * t.y;
+          v[i + HALF] = b * t.x + a * t.y;
+        }
+      }
+      __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)m * ep.ldo + n0 + h0;
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) store_bf16x32(dst + 32 * c, v + 32 * c);
+    }
+  }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(THREADS, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                int M, int N, int K, GemmEpilogue ep, int* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2], drain
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t tfull0 = empty0 + 8 * STAGES;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain = tempty0 + 16;
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 4 * 32);
+    }
+    mbar_init(drain, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  const int num_k = K / BK;
+  const int n_tiles = N / BN;
+  const int m_tiles = (M + BM - 1) / BM;
+  const int total = m_tiles * n_tiles;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / its last phase
+      for (int tile = blockIdx.x; tile < total && !abort_flag; tile += gridDim.x) {
+        const int m0 = (tile / n_tiles) * BM;
+        const int n0 = (tile % n_tiles) * BN;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, &abort_flag, err)) break;
+          mbar_arrive_expect_tx(full0 + 8 * stage, STAGE_BYTES);
+          tma_load_2d(smem_u32(sA + stage * A_BYTES), &tmA, kb * BK, m0, full0 + 8 * stage);
+          tma_load_2d(smem_u32(sB + stage * B_BYTES), &tmB, kb * BK, n0, full0 + 8 * stage);
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (abort_flag) {  // drain our own copies before the CTA may exit
+        volatile int never = 0;
+        for (int s = 0; s < STAGES; ++s)
+          if (issued_mask & (1u << s))
+            mbar_wait_bounded(full0 + 8 * s, (issued_phase >> s) & 1, &never, err, 100000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool issued_any = false;
+      for (int tile = blockIdx.x; tile < total && !abort_flag; tile += gridDim.x) {
+        if (!mbar_wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1, &abort_flag, err)) break;
+        fence_after();
+        const uint32_t d_tmem = tmem + acc * BN;
+        bool ok = true;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait_bounded(full0 + 8 * stage, phase, &abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16(d_tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (kb | k) != 0);
+          issued_any = true;
+          mma_commit(empty0 + 8 * stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        mma_commit(tfull0 + 8 * acc);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1;
+        }
+      }
+      if (abort_flag && issued_any) {  // wait for our MMAs before TMEM is freed
+        volatile int never = 0;
+        mma_commit(drain);
+        mbar_wait_bounded(drain, 0, &never, err, 100000000ull);
+      }
+    }
+  } else {
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int lane_base = q * 32;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      if (!mbar_wait_bounded(tfull0 + 8 * acc, acc_phase, &abort_flag, err)) break;
+      fence_after();
+      const int m0 = (tile / n_tiles) * BM;
+      const int n0 = (tile % n_tiles) * BN;
+      epilogue_tile<EPI>(tmem + acc * BN, lane_base, m0 + lane_base + lane, M, n0, ep);
+      fence_before();
+      mbar_arrive(tempty0 + 8 * acc);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+  }
+}
+
+// ---- host side ------------------------------------------------------------
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor [rows x cols] row-major (ld elements per row), box
+// [box_rows x 64], 128-byte swizzle, out-of-range rows read as zero.
+static int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                    uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return DLMZ_ECUDA;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    fprintf(stderr, "dlmz: cuTensorMapEncodeTiled failed (%d)\n", (int)r);
+    return DLMZ_ECUDA;
+  }
+  return DLMZ_OK;
+}
+
+template <int EPI>
+static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const GemmEpilogue& ep,
+                  cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    DLMZ_CUDA_TRY(cudaFuncSetAttribute(gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
+    attr = true;
+  }
+  const int tiles = ((M + BM - 1) / BM) * (N / BN);
+  const int grid = tiles < num_sms() ? tiles : num_sms();
+  gemm_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(a, b, M, N, K, ep, device_error_word());
+  return launch_status();
+}
+
+}  // namespace tc
+
+bool gemm_tc_supported(int M, int N, int K) { return M > 0 && N % tc::BN == 0 && K % tc::BK == 0 && K > 0; }
+
+int gemm_bf16_tc(const __nv_bfloat16* A, int lda, const __nv_bfloat16* B, int ldb, int M, int N, int K,
+                 int epi, const GemmEpilogue& ep, cudaStream_t s) {
+  if (!gemm_tc_supported(M, N, K)) return DLMZ_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) return DLMZ_EINVAL;
+  if ((lda | ldb) & 7) return DLMZ_EINVAL;
+  CUtensorMap ma, mb;
+  DLMZ_TRY(tc::make_map(&ma, A, M, K, lda, tc::BM));
+  DLMZ_TRY(tc::make_map(&mb, B, N, K, ldb, tc::BN));
+  switch (epi) {
+    case EPI_BF16: return tc::launch<EPI_BF16>(ma, mb, M, N, K, ep, s);
+    case EPI_F32: return tc::launch<EPI_F32>(ma, mb, M, N, K, ep, s);
+    case EPI_RESID_F32: return tc::launch<EPI_RESID_F32>(ma, mb, M, N, K, ep, s);
+    case EPI_SWIGLU_BF16: return tc::launch<EPI_SWIGLU_BF16>(ma, mb, M, N, K, ep, s);
+    case EPI_ROPE_BF16:
+      if (ep.head_dim == 32) return tc::launch<EPI_ROPE32_BF16>(ma, mb, M, N, K, ep, s);
+      if (ep.head_dim == 64) return tc::launch<EPI_ROPE64_BF16>(ma, mb, M, N, K, ep, s);
+      if (ep.head_dim == 128) return tc::launch<EPI_ROPE128_BF16>(ma, mb, M, N, K, ep, s);
+      return DLMZ_EINVAL;
+  }
+  return DLMZ_EINVAL;
+}
+
+}  // namespace dlmz

@@ -1,0 +1,65 @@
+// Launch helpers shared between the translation units of libdlmz.
+#pragma once
+
+#include "common.cuh"
+
+namespace dlmz {
+
+typedef __nv_bfloat16 bf16;
+
+// ---- GEMM epilogues --------------------------------------------------------
+enum {
+  EPI_BF16 = 0,        // out = bf16(acc)
+  EPI_F32 = 1,         // out = acc (float32)
+  EPI_RESID_F32 = 2,   // out += acc (float32 residual stream, in place)
+  EPI_SWIGLU_BF16 = 3, // out[:, f] = bf16(silu(g_f) * u_f), gate/up interleaved in blocks
+  EPI_ROPE_BF16 = 4,   // out = bf16(RoPE(acc)) on columns < rope_cols, bf16(acc) beyond
+  // internal instantiations of EPI_ROPE_BF16 per head dimension
+  EPI_ROPE32_BF16 = 5,
+  EPI_ROPE64_BF16 = 6,
+  EPI_ROPE128_BF16 = 7,
+};
+
+struct GemmEpilogue {
+  void* out;
+  int ldo;               // output leading dimension (elements)
+  const float2* rope_cs; // [L x head_dim/2] (cos, sin) for EPI_ROPE_BF16
+  int L;                 // window length (position = row % L)
+  int head_dim;
+  int rope_cols;         // columns [0, rope_cols) get RoPE (Q and K heads)
+  int gu_block;          // SwiGLU: gate/up interleave block (columns)
+};
+
+// tcgen05 path: N % 256 == 0, K % 64 == 0, 16-byte aligned operands.
+bool gemm_tc_supported(int M, int N, int K);
+int gemm_bf16_tc(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, int epi,
+                 const GemmEpilogue& ep, cudaStream_t s);
+// CUDA-core path (any shape; float32 or bf16 inputs, float32 accumulation).
+template <typename T>
+int gemm_simt(const T* A, int lda, const T* B, int ldb, int M, int N, int K, int epi,
+              const GemmEpilogue& ep, cudaStream_t s);
+
+// ---- layers -------------------------------------------------------------------
+template <typename T>
+int embed(const int32_t* state, int T_tokens, const T* E, int d, float* x, cudaStream_t s);
+// h[r] = OutT(x[row(r)] * g / sqrt(mean(x^2) + eps)); row(r) = (r / rpc) * L + row0 + r % rpc
+// when rpc > 0, else r.
+template <typename OutT>
+int rmsnorm(const float* x, int rows, int d, const float* g, float eps, OutT* h, int L, int row0,
+            int rpc, cudaStream_t s);
+template <typename T>
+int rope_inplace(T* qkv, int T_tokens, int ld, int n_heads_rot, int head_dim, int L,
+                 const float2* cs, cudaStream_t s);
+template <typename T>
+int swiglu(const float* gu, int T_tokens, int F, int gu_block, T* out, cudaStream_t s);
+template <typename T>
+int attention_simt(const T* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
+                   int head_dim, int d, T* out, cudaStream_t s);
+int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
+                       int head_dim, int d, bf16* out, cudaStream_t s);
+
+// ---- quantiser / selector / coder --------------------------------------------------
+int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, uint64_t* W,
+                  uint64_t* A, int32_t* Hq, int32_t* top, float* mx, cudaStream_t s);
+
+}  // namespace dlmz

@@ -1,0 +1,68 @@
+// Model object: device weights of the masked DLM and its forward workspace.
+#pragma once
+
+#include <vector>
+
+#include "kernels.cuh"
+
+namespace dlmz {
+
+// Grow-only device buffer.
+struct DevBuf {
+  void* p = nullptr;
+  size_t bytes = 0;
+  int ensure(size_t n) {
+    if (n <= bytes) return DLMZ_OK;
+    if (p) cudaFree(p);
+    p = nullptr;
+    bytes = 0;
+    if (n == 0) return DLMZ_OK;
+    if (cudaMalloc(&p, n) != cudaSuccess) {
+      cudaGetLastError();
+      return DLMZ_ENOMEM;
+    }
+    bytes = n;
+    return DLMZ_OK;
+  }
+  void release() {
+    if (p) cudaFree(p);
+    p = nullptr;
+    bytes = 0;
+  }
+  template <typename T>
+  T* as() const { return reinterpret_cast<T*>(p); }
+};
+
+struct ForwardWorkspace {
+  DevBuf x, h, qkv, attn, act, gu, hc, rope;
+  int rope_L = 0;
+};
+
+}  // namespace dlmz
+
+struct dlmz_model {
+  dlmz_model_config cfg;
+  int hd, dkv, nqkv, gu_block;
+  bool bf16;
+  bool tc;  // tensor-core GEMM path usable for every projection
+  size_t esz;
+  void* weights = nullptr;  // one allocation
+  void* E = nullptr;
+  std::vector<void*> wqkv, wo, wgu, wdown;
+  void* head = nullptr;
+  float* gains = nullptr;  // ones [d]
+  uint64_t fingerprint = 0;
+  dlmz::ForwardWorkspace ws;
+  void* pipe = nullptr;  // pipeline workspace (owned, see pipeline.cu)
+};
+
+namespace dlmz {
+// Forward of a batch (Definition 3): logits [n_chunks*rpc x V] for positions
+// [row0, row0+rpc) of every window.
+int model_forward(dlmz_model* m, const int32_t* state, int n_chunks, int L, int row0, int rpc, float* logits,
+                  cudaStream_t s);
+// Frees the pipeline workspace attached to the model (pipeline.cu).
+void pipeline_release(dlmz_model* m);
+// Bytes of forward workspace per token (for batch sizing).
+size_t model_workspace_per_token(const dlmz_model* m);
+}  // namespace dlmz

@@ -1,0 +1,783 @@
+// Iterative DLM compression pipeline (Sec. 3.2) and the C ABI.
+//
+// compress: the input is cut into non-overlapping windows of chunk_len
+// symbols (w, Sec. 4); windows of equal length run as a batch.  Each batch
+// starts fully masked (c = 0) and repeats forward -> quantise -> select ->
+// code -> reveal until every position is committed (coverage sum u_k = n,
+// Sec. 3.3).  Each window owns one range-coder stream.  decompress replays
+// the same batches and schedule from the header alone (Sec. 3.3, last
+// paragraph): the selection of a step never depends on the symbols that
+// step codes, so the decoder sees the same logits at every step.
+//
+// Container (little-endian): 64-byte header (magic "DLMZ", version, P,
+// policy kind, model fingerprint, V, chunk_len, batch_chunks, k, block,
+// tau_q, k_min, k_max, n_symbols, n_chunks, checksum), one LEB128 varint per
+// window with its stream's bit length, then the streams (ceil(bits/8) bytes
+// each).  The checksum is the CRC-32 (IEEE) of the windows' CRC-32s.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <vector>
+
+#include "coder.cuh"
+#include "model.cuh"
+
+namespace dlmz {
+
+// ---- error word -------------------------------------------------------------------------
+static int* g_err = nullptr;
+int* device_error_word() {
+  if (!g_err) {
+    if (cudaMalloc(&g_err, sizeof(int)) != cudaSuccess) return nullptr;
+    cudaMemset(g_err, 0, sizeof(int));
+  }
+  return g_err;
+}
+
+static int clear_device_error(cudaStream_t s) {
+  DLMZ_CUDA_TRY(cudaMemsetAsync(device_error_word(), 0, sizeof(int), s));
+  return DLMZ_OK;
+}
+
+static int check_device(cudaStream_t s) {
+  DLMZ_CUDA_TRY(cudaStreamSynchronize(s));
+  int* e = device_error_word();
+  int h = 0;
+  DLMZ_CUDA_TRY(cudaMemcpy(&h, e, sizeof(int), cudaMemcpyDeviceToHost));
+  if (h) DLMZ_CUDA_TRY(cudaMemset(e, 0, sizeof(int)));
+  if (h & ERR_TIMEOUT) return DLMZ_ETIMEOUT;
+  if (h & ERR_NONFINITE) return DLMZ_EBADINPUT;
+  if (h & (ERR_CORRUPT | ERR_CAPACITY)) return DLMZ_ECORRUPT;
+  return DLMZ_OK;
+}
+
+// ---- small kernels ---------------------------------------------------------------------
+__global__ void fill_i32(int32_t* p, int64_t n, int32_t v) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) p[i] = v;
+}
+
+// input symbols of windows [c0, c0+nc) (each Lb long) -> int32
+__global__ void symbols_in_kernel(const uint8_t* in, int64_t sym0, int64_t n, int tok, int V, int32_t* out, int* err) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    int64_t v;
+    if (tok) {
+      const uint8_t* p = in + 4 * (sym0 + i);
+      v = (int64_t)p[0] | ((int64_t)p[1] << 8) | ((int64_t)p[2] << 16) | ((int64_t)p[3] << 24);
+      if (v >= V) {
+        atomicOr(err, ERR_NONFINITE);  // reported as EBADINPUT
+        v = 0;
+      }
+    } else {
+      v = in[sym0 + i];
+    }
+    out[i] = (int32_t)v;
+  }
+}
+
+__global__ void symbols_out_kernel(const int32_t* sym, int64_t sym0, int64_t n, int tok, uint8_t* out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t v = (uint32_t)sym[i];
+    if (tok) {
+      uint8_t* p = out + 4 * (sym0 + i);
+      p[0] = (uint8_t)v;
+      p[1] = (uint8_t)(v >> 8);
+      p[2] = (uint8_t)(v >> 16);
+      p[3] = (uint8_t)(v >> 24);
+    } else {
+      out[sym0 + i] = (uint8_t)v;
+    }
+  }
+}
+
+// CRC-32 (IEEE, reflected polynomial 0xEDB88320) of each window, one thread per window.
+__global__ void window_crc_kernel(const uint8_t* data, uint64_t nbytes, uint64_t wbytes, int nwin, uint32_t* out) {
+  __shared__ uint32_t T[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+    uint32_t c = (uint32_t)i;
+    for (int k = 0; k < 8; ++k) c = (c >> 1) ^ (0xEDB88320u & (0u - (c & 1u)));
+    T[i] = c;
+  }
+  __syncthreads();
+  const int w = blockIdx.x * blockDim.x + threadIdx.x;
+  if (w >= nwin) return;
+  const uint64_t b0 = (uint64_t)w * wbytes;
+  const uint64_t b1 = b0 + wbytes < nbytes ? b0 + wbytes : nbytes;
+  uint32_t crc = 0xFFFFFFFFu;
+  for (uint64_t i = b0; i < b1; ++i) crc = T[(crc ^ data[i]) & 0xFF] ^ (crc >> 8);
+  out[w] = ~crc;
+}
+
+__global__ void gather_streams_kernel(const uint8_t* staging, uint64_t cap, const uint32_t* bits,
+                                      const uint64_t* offsets, int n, uint8_t* out) {
+  const int c = blockIdx.x;
+  if (c >= n) return;
+  const uint64_t nb = (bits[c] + 7) / 8;
+  const uint8_t* src = staging + (size_t)c * cap;
+  uint8_t* dst = out + offsets[c];
+  for (uint64_t i = threadIdx.x; i < nb; i += blockDim.x) dst[i] = src[i];
+}
+
+__global__ void sum_i32_kernel(const int32_t* v, int n, unsigned long long* out) {
+  unsigned long long s = 0;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) s += (unsigned long long)v[i];
+  for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  __shared__ unsigned long long red[32];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long t = 0;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t += red[i];
+    *out = t;
+  }
+}
+
+static unsigned grid_for(int64_t n, int threads = 256) {
+  int64_t b = (n + threads - 1) / threads;
+  if (b < 1) b = 1;
+  if (b > 65535) b = 65535;
+  return (unsigned)b;
+}
+
+static uint32_t crc32_host(const uint8_t* p, size_t n) {
+  uint32_t crc = 0xFFFFFFFFu;
+  for (size_t i = 0; i < n; ++i) {
+    crc ^= p[i];
+    for (int k = 0; k < 8; ++k) crc = (crc >> 1) ^ (0xEDB88320u & (0u - (crc & 1u)));
+  }
+  return ~crc;
+}
+
+// ---- per-batch step state ---------------------------------------------------------
+struct StepBufs {
+  DevBuf logits, W, Hq, top, mx, sel_count, sel_pos, committed, sum;
+  int ensure(size_t rows, int V, int nc, int kcap) {
+    DLMZ_TRY(logits.ensure(rows * (size_t)V * 4));
+    DLMZ_TRY(W.ensure(rows * 8));
+    DLMZ_TRY(Hq.ensure(rows * 4));
+    DLMZ_TRY(top.ensure(rows * 4));
+    DLMZ_TRY(mx.ensure(rows * 4));
+    DLMZ_TRY(sel_count.ensure((size_t)nc * 4));
+    DLMZ_TRY(sel_pos.ensure((size_t)nc * kcap * 4));
+    DLMZ_TRY(committed.ensure((size_t)nc * 4));
+    DLMZ_TRY(sum.ensure(8));
+    return DLMZ_OK;
+  }
+  void release() {
+    logits.release(); W.release(); Hq.release(); top.release(); mx.release();
+    sel_count.release(); sel_pos.release(); committed.release(); sum.release();
+  }
+};
+
+static int kcap_for(const dlmz_k_policy& p, int rpc) {
+  int k = p.kind == DLMZ_TOPK_CONF ? (int)p.k : (p.k_max ? (int)p.k_max : rpc);
+  if (p.kind == DLMZ_ENTROPY && (int)p.k_min > k) k = (int)p.k_min;
+  return k < rpc ? k : rpc;
+}
+
+static int64_t tau_q_of(float tau) { return (int64_t)floor((double)tau * 65536.0); }
+
+// quantise + select + code one step on logits of rows [row0, row0+rpc) of each window
+static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int P, const dlmz_k_policy& pol,
+                    int row0, int rpc, const int32_t* symbols, int32_t* state, CoderState* cst, uint8_t* ebytes,
+                    uint64_t cap_bytes, const uint8_t* in_bytes, const uint64_t* in_off, const uint32_t* in_bits,
+                    bool decode, int32_t* committed, cudaStream_t s) {
+  const int rows = nc * rpc;
+  const int kcap = kcap_for(pol, rpc);
+  DLMZ_TRY(sb.ensure(rows, 1, nc, kcap));
+  DLMZ_TRY(quantize_rows(logits, rows, V, P, nullptr, sb.W.as<uint64_t>(), nullptr, sb.Hq.as<int32_t>(),
+                         sb.top.as<int32_t>(), sb.mx.as<float>(), s));
+  if (pol.kind == DLMZ_TOPK_CONF)
+    DLMZ_TRY(select_rows<uint64_t>(state, nc, L, V, row0, rpc, sb.W.as<uint64_t>(), 0, (int)pol.k, 0, 0, 0, kcap,
+                                   sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), s));
+  else
+    DLMZ_TRY(select_rows<int32_t>(state, nc, L, V, row0, rpc, sb.Hq.as<int32_t>(), 1, 0, tau_q_of(pol.tau_bits),
+                                  (int)pol.k_min, (int)pol.k_max, kcap, sb.sel_count.as<int32_t>(),
+                                  sb.sel_pos.as<int32_t>(), s));
+  CodeArgs a{};
+  a.logits = logits;
+  a.mx = sb.mx.as<float>();
+  a.W = sb.W.as<uint64_t>();
+  a.top = sb.top.as<int32_t>();
+  a.sel_count = sb.sel_count.as<int32_t>();
+  a.sel_pos = sb.sel_pos.as<int32_t>();
+  a.symbols = symbols;
+  a.state = state;
+  a.state_c = cst;
+  a.bytes = ebytes;
+  a.cap_bytes = cap_bytes;
+  a.in_bytes = in_bytes;
+  a.in_offsets = in_off;
+  a.in_bits = in_bits;
+  a.committed = committed;
+  a.err = device_error_word();
+  a.V = V;
+  a.P = P;
+  a.L = L;
+  a.row0 = row0;
+  a.rpc = rpc;
+  a.kcap = kcap;
+  return code_step(a, decode, nc, s);
+}
+
+static int validate_policy(const dlmz_k_policy* p) {
+  if (!p) return DLMZ_EINVAL;
+  if (p->kind == DLMZ_TOPK_CONF) return p->k >= 1 ? DLMZ_OK : DLMZ_EINVAL;
+  if (p->kind == DLMZ_ENTROPY) {
+    if (p->k_min < 1) return DLMZ_EINVAL;
+    if (p->k_max && p->k_max < p->k_min) return DLMZ_EINVAL;
+    if (!(p->tau_bits >= 0.0f) || p->tau_bits > 30000.0f) return DLMZ_EINVAL;
+    return DLMZ_OK;
+  }
+  return DLMZ_EINVAL;
+}
+
+static int precision_for(uint32_t V) { return V <= 4096 ? 16 : 24; }
+
+static uint64_t cap_bytes_for(uint32_t L, int P) {
+  const uint64_t units = ((uint64_t)L * P + 80) / 16 + 4;
+  return 2 * units;
+}
+
+// One batch of nc windows of length Lb through all steps.
+static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int nc, int Lb, const int32_t* symbols,
+                     int32_t* state, CoderState* cst, uint8_t* ebytes, uint64_t cap_bytes, const uint8_t* in_bytes,
+                     const uint64_t* in_off, const uint32_t* in_bits, bool decode, cudaStream_t s) {
+  const int V = (int)m->cfg.vocab, P = precision_for(m->cfg.vocab);
+  fill_i32<<<grid_for((int64_t)nc * Lb), 256, 0, s>>>(state, (int64_t)nc * Lb, V);
+  DLMZ_TRY(launch_status());
+  if (decode) DLMZ_TRY(coder_load(cst, nc, in_bytes, in_off, in_bits, s));
+  else DLMZ_TRY(coder_reset(cst, nc, s));
+  if (pol.kind == DLMZ_TOPK_CONF) {
+    const int B = pol.block ? (int)pol.block : Lb;
+    for (int b0 = 0; b0 < Lb; b0 += B) {
+      const int Bl = B < Lb - b0 ? B : Lb - b0;
+      DLMZ_TRY(sb.ensure((size_t)nc * Bl, V, nc, kcap_for(pol, Bl)));
+      for (int rem = Bl; rem > 0; rem -= ((int)pol.k < rem ? (int)pol.k : rem)) {
+        DLMZ_TRY(model_forward(m, state, nc, Lb, b0, Bl, sb.logits.as<float>(), s));
+        DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, pol, b0, Bl, symbols, state, cst, ebytes,
+                          cap_bytes, in_bytes, in_off, in_bits, decode, nullptr, s));
+      }
+    }
+  } else {
+    DLMZ_TRY(sb.ensure((size_t)nc * Lb, V, nc, kcap_for(pol, Lb)));
+    int64_t remaining = (int64_t)nc * Lb;
+    for (int64_t step = 0; remaining > 0; ++step) {
+      if (step > (int64_t)Lb) return DLMZ_ECORRUPT;  // every step commits >= 1 per live window
+      DLMZ_TRY(model_forward(m, state, nc, Lb, 0, Lb, sb.logits.as<float>(), s));
+      DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, pol, 0, Lb, symbols, state, cst, ebytes, cap_bytes,
+                        in_bytes, in_off, in_bits, decode, sb.committed.as<int32_t>(), s));
+      sum_i32_kernel<<<1, 256, 0, s>>>(sb.committed.as<int32_t>(), nc, sb.sum.as<unsigned long long>());
+      DLMZ_TRY(launch_status());
+      unsigned long long done = 0;
+      DLMZ_CUDA_TRY(cudaMemcpyAsync(&done, sb.sum.p, 8, cudaMemcpyDeviceToHost, s));
+      DLMZ_CUDA_TRY(cudaStreamSynchronize(s));
+      if (done == 0) return DLMZ_ECORRUPT;
+      remaining -= (int64_t)done;
+    }
+  }
+  return DLMZ_OK;
+}
+
+struct PipeWs {
+  StepBufs sb;
+  DevBuf symbols, state, cst, staging, bits, crcs, offsets, hin, hout;
+  void release() {
+    sb.release(); symbols.release(); state.release(); cst.release(); staging.release(); bits.release();
+    crcs.release(); offsets.release(); hin.release(); hout.release();
+  }
+};
+
+static PipeWs& pipe_of(dlmz_model* m) {
+  if (!m->pipe) m->pipe = new PipeWs();
+  return *reinterpret_cast<PipeWs*>(m->pipe);
+}
+
+static int default_batch(const dlmz_model* m, uint32_t L, uint32_t n_chunks) {
+  size_t freeb = 0, total = 0;
+  cudaMemGetInfo(&freeb, &total);
+  size_t budget = freeb / 2;
+  const size_t cap = (size_t)48 << 30;
+  if (budget > cap) budget = cap;
+  const size_t per_chunk = (size_t)L * (model_workspace_per_token(m) + 8 + 4ull * m->cfg.vocab + 64);
+  size_t b = per_chunk ? budget / per_chunk : 1;
+  if (b > 1024) b = 1024;
+  if (b < 1) b = 1;
+  if (b > n_chunks) b = n_chunks ? n_chunks : 1;
+  return (int)b;
+}
+
+struct Header {
+  uint32_t P, kind, vocab, chunk_len, batch_chunks, k, block, tau_q, k_min, k_max, n_chunks, crc;
+  uint64_t fingerprint, n_symbols;
+};
+
+static void put32(uint8_t* p, uint32_t v) { for (int i = 0; i < 4; ++i) p[i] = (uint8_t)(v >> (8 * i)); }
+static void put64(uint8_t* p, uint64_t v) { for (int i = 0; i < 8; ++i) p[i] = (uint8_t)(v >> (8 * i)); }
+static uint32_t get32(const uint8_t* p) { uint32_t v = 0; for (int i = 0; i < 4; ++i) v |= (uint32_t)p[i] << (8 * i); return v; }
+static uint64_t get64(const uint8_t* p) { uint64_t v = 0; for (int i = 0; i < 8; ++i) v |= (uint64_t)p[i] << (8 * i); return v; }
+
+static void write_header(uint8_t* o, const Header& h) {
+  memcpy(o, "DLMZ", 4);
+  o[4] = 1;
+  o[5] = 0;
+  o[6] = (uint8_t)h.P;
+  o[7] = (uint8_t)h.kind;
+  put64(o + 8, h.fingerprint);
+  put32(o + 16, h.vocab);
+  put32(o + 20, h.chunk_len);
+  put32(o + 24, h.batch_chunks);
+  put32(o + 28, h.k);
+  put32(o + 32, h.block);
+  put32(o + 36, h.tau_q);
+  put32(o + 40, h.k_min);
+  put32(o + 44, h.k_max);
+  put64(o + 48, h.n_symbols);
+  put32(o + 56, h.n_chunks);
+  put32(o + 60, h.crc);
+}
+
+static int read_header(const uint8_t* o, size_t n, Header& h) {
+  if (n < 64) return DLMZ_ECORRUPT;
+  if (memcmp(o, "DLMZ", 4) || o[4] != 1 || o[5] != 0) return DLMZ_ECORRUPT;
+  h.P = o[6];
+  h.kind = o[7];
+  h.fingerprint = get64(o + 8);
+  h.vocab = get32(o + 16);
+  h.chunk_len = get32(o + 20);
+  h.batch_chunks = get32(o + 24);
+  h.k = get32(o + 28);
+  h.block = get32(o + 32);
+  h.tau_q = get32(o + 36);
+  h.k_min = get32(o + 40);
+  h.k_max = get32(o + 44);
+  h.n_symbols = get64(o + 48);
+  h.n_chunks = get32(o + 56);
+  h.crc = get32(o + 60);
+  if (h.chunk_len == 0 && h.n_symbols) return DLMZ_ECORRUPT;
+  const uint64_t exp = h.chunk_len ? (h.n_symbols + h.chunk_len - 1) / h.chunk_len : 0;
+  if (exp != h.n_chunks) return DLMZ_ECORRUPT;
+  return DLMZ_OK;
+}
+
+static void put_varint(std::vector<uint8_t>& o, uint64_t v) {
+  do {
+    uint8_t b = v & 0x7F;
+    v >>= 7;
+    o.push_back(v ? (b | 0x80) : b);
+  } while (v);
+}
+
+// Batches: full windows in groups of bc, then the ragged tail window alone.
+struct BatchPlan {
+  int c0, nc, L;
+};
+static std::vector<BatchPlan> plan_batches(uint64_t n_sym, uint32_t L, int bc) {
+  std::vector<BatchPlan> v;
+  const uint64_t nfull = n_sym / L;
+  for (uint64_t c = 0; c < nfull; c += bc) v.push_back({(int)c, (int)(nfull - c < (uint64_t)bc ? nfull - c : bc), (int)L});
+  if (n_sym % L) v.push_back({(int)nfull, 1, (int)(n_sym % L)});
+  return v;
+}
+
+static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, uint32_t L, const dlmz_k_policy* pol,
+                           uint32_t batch_chunks, uint8_t* d_out, size_t out_cap, size_t* out_bytes, cudaStream_t s) {
+  if (!m || !pol || !out_bytes || L == 0) return DLMZ_EINVAL;
+  if (in_bytes && !d_in) return DLMZ_EINVAL;
+  DLMZ_TRY(validate_policy(pol));
+  const uint32_t V = m->cfg.vocab;
+  const int tok = V > 256;
+  if (tok && in_bytes % 4) return DLMZ_EBADINPUT;
+  const uint64_t n_sym = tok ? in_bytes / 4 : in_bytes;
+  const uint64_t n_chunks64 = (n_sym + L - 1) / L;
+  if (n_chunks64 > 0x7fffffff) return DLMZ_EINVAL;
+  const int n_chunks = (int)n_chunks64;
+  const int P = precision_for(V);
+  const uint64_t cap = cap_bytes_for(L, P);
+  const int bc = batch_chunks ? (int)batch_chunks : default_batch(m, L, (uint32_t)n_chunks);
+  PipeWs& w = pipe_of(m);
+  DLMZ_TRY(device_error_word() ? DLMZ_OK : DLMZ_ENOMEM);
+  DLMZ_TRY(clear_device_error(s));
+  DLMZ_TRY(w.staging.ensure((size_t)n_chunks * cap + 16));
+  DLMZ_TRY(w.bits.ensure((size_t)n_chunks * 4 + 4));
+  DLMZ_TRY(w.crcs.ensure((size_t)n_chunks * 4 + 4));
+  DLMZ_TRY(w.offsets.ensure((size_t)n_chunks * 8 + 8));
+  const size_t bl = (size_t)bc * L;
+  DLMZ_TRY(w.symbols.ensure(bl * 4));
+  DLMZ_TRY(w.state.ensure(bl * 4));
+  DLMZ_TRY(w.cst.ensure((size_t)bc * sizeof(CoderState)));
+  const uint64_t wbytes = (uint64_t)L * (tok ? 4 : 1);
+  if (n_chunks) {
+    window_crc_kernel<<<(n_chunks + 127) / 128, 128, 0, s>>>(d_in, in_bytes, wbytes, n_chunks, w.crcs.as<uint32_t>());
+    DLMZ_TRY(launch_status());
+  }
+  for (const BatchPlan& b : plan_batches(n_sym, L, bc)) {
+    const int64_t nsym_b = (int64_t)b.nc * b.L;
+    symbols_in_kernel<<<grid_for(nsym_b), 256, 0, s>>>(d_in, (int64_t)b.c0 * L, nsym_b, tok, (int)V,
+                                                       w.symbols.as<int32_t>(), device_error_word());
+    DLMZ_TRY(launch_status());
+    uint8_t* eb = w.staging.as<uint8_t>() + (size_t)b.c0 * cap;
+    DLMZ_TRY(run_batch(m, w.sb, *pol, b.nc, b.L, w.symbols.as<int32_t>(), w.state.as<int32_t>(),
+                       w.cst.as<CoderState>(), eb, cap, nullptr, nullptr, nullptr, false, s));
+    DLMZ_TRY(coder_finish(w.cst.as<CoderState>(), b.nc, eb, cap, w.bits.as<uint32_t>() + b.c0, nullptr, nullptr, s));
+  }
+  DLMZ_TRY(check_device(s));
+  std::vector<uint32_t> bits(n_chunks), crcs(n_chunks);
+  if (n_chunks) {
+    DLMZ_CUDA_TRY(cudaMemcpy(bits.data(), w.bits.p, (size_t)n_chunks * 4, cudaMemcpyDeviceToHost));
+    DLMZ_CUDA_TRY(cudaMemcpy(crcs.data(), w.crcs.p, (size_t)n_chunks * 4, cudaMemcpyDeviceToHost));
+  }
+  std::vector<uint8_t> crcb((size_t)n_chunks * 4);
+  for (int c = 0; c < n_chunks; ++c) put32(crcb.data() + 4 * c, crcs[c]);
+  Header h{};
+  h.P = P;
+  h.kind = pol->kind;
+  h.vocab = V;
+  h.chunk_len = L;
+  h.batch_chunks = bc;
+  h.k = pol->k;
+  h.block = pol->block;
+  h.tau_q = (uint32_t)tau_q_of(pol->tau_bits);
+  h.k_min = pol->k_min;
+  h.k_max = pol->k_max;
+  h.n_chunks = n_chunks;
+  h.crc = crc32_host(crcb.data(), crcb.size());
+  h.fingerprint = m->fingerprint;
+  h.n_symbols = n_sym;
+  std::vector<uint8_t> head(64);
+  write_header(head.data(), h);
+  for (int c = 0; c < n_chunks; ++c) put_varint(head, bits[c]);
+  std::vector<uint64_t> offs(n_chunks);
+  uint64_t pos = head.size();
+  for (int c = 0; c < n_chunks; ++c) {
+    offs[c] = pos;
+    pos += (bits[c] + 7) / 8;
+  }
+  *out_bytes = pos;
+  if (pos > out_cap) return DLMZ_ECAPACITY;
+  if (!d_out) return DLMZ_EINVAL;
+  DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out, head.data(), head.size(), cudaMemcpyHostToDevice, s));
+  if (n_chunks) {
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(w.offsets.p, offs.data(), (size_t)n_chunks * 8, cudaMemcpyHostToDevice, s));
+    gather_streams_kernel<<<n_chunks, 128, 0, s>>>(w.staging.as<uint8_t>(), cap, w.bits.as<uint32_t>(),
+                                                   w.offsets.as<uint64_t>(), n_chunks, d_out);
+    DLMZ_TRY(launch_status());
+  }
+  return check_device(s);
+}
+
+static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, uint8_t* d_out, size_t out_cap,
+                             size_t* out_bytes, cudaStream_t s) {
+  if (!m || !d_in || !out_bytes) return DLMZ_EINVAL;
+  DLMZ_TRY(device_error_word() ? DLMZ_OK : DLMZ_ENOMEM);
+  DLMZ_TRY(clear_device_error(s));
+  uint8_t hb[64];
+  if (in_bytes < 64) return DLMZ_ECORRUPT;
+  DLMZ_CUDA_TRY(cudaMemcpy(hb, d_in, 64, cudaMemcpyDeviceToHost));
+  Header h{};
+  DLMZ_TRY(read_header(hb, in_bytes, h));
+  if (h.fingerprint != m->fingerprint) return DLMZ_EMODEL;
+  if (h.vocab != m->cfg.vocab || (int)h.P != precision_for(h.vocab)) return DLMZ_ECORRUPT;
+  dlmz_k_policy pol{h.kind, h.k, h.block, (float)(h.tau_q / 65536.0), h.k_min, h.k_max};
+  if (validate_policy(&pol) != DLMZ_OK) return DLMZ_ECORRUPT;
+  if (h.n_symbols && h.batch_chunks == 0) return DLMZ_ECORRUPT;
+  const int tok = h.vocab > 256;
+  const uint64_t out_need = h.n_symbols * (tok ? 4 : 1);
+  *out_bytes = out_need;
+  if (out_need > out_cap) return DLMZ_ECAPACITY;
+  if (out_need && !d_out) return DLMZ_EINVAL;
+  const int n_chunks = (int)h.n_chunks;
+  const size_t vmax = (size_t)n_chunks * 5 < in_bytes - 64 ? (size_t)n_chunks * 5 : in_bytes - 64;
+  std::vector<uint8_t> vb(vmax);
+  if (vmax) DLMZ_CUDA_TRY(cudaMemcpy(vb.data(), d_in + 64, vmax, cudaMemcpyDeviceToHost));
+  std::vector<uint32_t> bits(n_chunks);
+  size_t p = 0;
+  for (int c = 0; c < n_chunks; ++c) {
+    uint64_t v = 0;
+    int sh = 0;
+    for (;;) {
+      if (p >= vmax || sh > 35) return DLMZ_ECORRUPT;
+      const uint8_t b = vb[p++];
+      v |= (uint64_t)(b & 0x7F) << sh;
+      sh += 7;
+      if (!(b & 0x80)) break;
+    }
+    if (v > 0xFFFFFFFFull) return DLMZ_ECORRUPT;
+    bits[c] = (uint32_t)v;
+  }
+  std::vector<uint64_t> offs(n_chunks);
+  uint64_t pos = 64 + p;
+  for (int c = 0; c < n_chunks; ++c) {
+    offs[c] = pos;
+    pos += (bits[c] + 7) / 8;
+  }
+  if (pos != in_bytes) return DLMZ_ECORRUPT;
+  const uint32_t L = h.chunk_len;
+  const int bc = (int)h.batch_chunks;
+  PipeWs& w = pipe_of(m);
+  DLMZ_TRY(w.bits.ensure((size_t)n_chunks * 4 + 4));
+  DLMZ_TRY(w.offsets.ensure((size_t)n_chunks * 8 + 8));
+  DLMZ_TRY(w.crcs.ensure((size_t)n_chunks * 4 + 4));
+  if (n_chunks) {
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(w.bits.p, bits.data(), (size_t)n_chunks * 4, cudaMemcpyHostToDevice, s));
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(w.offsets.p, offs.data(), (size_t)n_chunks * 8, cudaMemcpyHostToDevice, s));
+  }
+  const size_t bl = (size_t)(bc < n_chunks ? bc : (n_chunks ? n_chunks : 1)) * L;
+  DLMZ_TRY(w.state.ensure(bl * 4));
+  DLMZ_TRY(w.cst.ensure((size_t)bc * sizeof(CoderState)));
+  for (const BatchPlan& b : plan_batches(h.n_symbols, L, bc)) {
+    DLMZ_TRY(run_batch(m, w.sb, pol, b.nc, b.L, nullptr, w.state.as<int32_t>(), w.cst.as<CoderState>(), nullptr, 0,
+                       d_in, w.offsets.as<uint64_t>() + b.c0, w.bits.as<uint32_t>() + b.c0, true, s));
+    const int64_t nsym_b = (int64_t)b.nc * b.L;
+    symbols_out_kernel<<<grid_for(nsym_b), 256, 0, s>>>(w.state.as<int32_t>(), (int64_t)b.c0 * L, nsym_b, tok, d_out);
+    DLMZ_TRY(launch_status());
+  }
+  int rc = check_device(s);
+  if (rc != DLMZ_OK) return rc;
+  std::vector<uint32_t> crcs(n_chunks);
+  if (n_chunks) {
+    window_crc_kernel<<<(n_chunks + 127) / 128, 128, 0, s>>>(d_out, out_need, (uint64_t)L * (tok ? 4 : 1), n_chunks,
+                                                             w.crcs.as<uint32_t>());
+    DLMZ_TRY(launch_status());
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(crcs.data(), w.crcs.p, (size_t)n_chunks * 4, cudaMemcpyDeviceToHost, s));
+    DLMZ_CUDA_TRY(cudaStreamSynchronize(s));
+  }
+  std::vector<uint8_t> crcb((size_t)n_chunks * 4);
+  for (int c = 0; c < n_chunks; ++c) put32(crcb.data() + 4 * c, crcs[c]);
+  if (crc32_host(crcb.data(), crcb.size()) != h.crc) return DLMZ_ECORRUPT;
+  return DLMZ_OK;
+}
+
+void pipeline_release(dlmz_model* m) {
+  if (m && m->pipe) {
+    PipeWs* w = reinterpret_cast<PipeWs*>(m->pipe);
+    w->release();
+    delete w;
+    m->pipe = nullptr;
+  }
+}
+
+}  // namespace dlmz
+
+using namespace dlmz;
+
+extern "C" {
+
+const char* dlmz_strerror(int code) {
+  switch (code) {
+    case DLMZ_OK: return "ok";
+    case DLMZ_EINVAL: return "invalid argument";
+    case DLMZ_EBADINPUT: return "invalid input symbols";
+    case DLMZ_ECORRUPT: return "corrupt container";
+    case DLMZ_EMODEL: return "container written by another model";
+    case DLMZ_ENOMEM: return "out of memory";
+    case DLMZ_ECUDA: return "CUDA error";
+    case DLMZ_ETIMEOUT: return "device wait timed out";
+    case DLMZ_ECAPACITY: return "output buffer too small";
+  }
+  return "unknown error";
+}
+
+void dlmz_free(void* p) { free(p); }
+
+size_t dlmz_compress_bound(const dlmz_model* m, size_t in_bytes, uint32_t chunk_len) {
+  if (!m || !chunk_len) return 0;
+  const uint64_t n_sym = m->cfg.vocab > 256 ? in_bytes / 4 : in_bytes;
+  const uint64_t nc = (n_sym + chunk_len - 1) / chunk_len;
+  return 64 + nc * 5 + nc * cap_bytes_for(chunk_len, precision_for(m->cfg.vocab));
+}
+
+int dlmz_compress_device(const dlmz_model* m, const void* d_in, size_t in_bytes, uint32_t chunk_len,
+                         const dlmz_k_policy* policy, uint32_t batch_chunks, uint8_t* d_out, size_t out_cap,
+                         size_t* out_bytes, void* stream) {
+  return compress_device(const_cast<dlmz_model*>(m), reinterpret_cast<const uint8_t*>(d_in), in_bytes, chunk_len,
+                         policy, batch_chunks, d_out, out_cap, out_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_decompress_device(const dlmz_model* m, const uint8_t* d_in, size_t in_bytes, uint8_t* d_out, size_t out_cap,
+                           size_t* out_bytes, void* stream) {
+  return decompress_device(const_cast<dlmz_model*>(m), d_in, in_bytes, d_out, out_cap, out_bytes,
+                           reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_compress_ex(const dlmz_model* mc, const void* in, size_t in_bytes, uint32_t chunk_len,
+                     const dlmz_k_policy* policy, uint32_t batch_chunks, uint8_t** out, size_t* out_bytes) {
+  if (out) *out = nullptr;
+  if (!mc || !out || !out_bytes || (in_bytes && !in)) return DLMZ_EINVAL;
+  dlmz_model* m = const_cast<dlmz_model*>(mc);
+  PipeWs& w = pipe_of(m);
+  const size_t bound = dlmz_compress_bound(m, in_bytes, chunk_len);
+  if (!bound) return DLMZ_EINVAL;
+  DLMZ_TRY(w.hin.ensure(in_bytes + 16));
+  DLMZ_TRY(w.hout.ensure(bound));
+  if (in_bytes) DLMZ_CUDA_TRY(cudaMemcpy(w.hin.p, in, in_bytes, cudaMemcpyHostToDevice));
+  size_t n = 0;
+  DLMZ_TRY(compress_device(m, w.hin.as<uint8_t>(), in_bytes, chunk_len, policy, batch_chunks, w.hout.as<uint8_t>(),
+                           bound, &n, 0));
+  uint8_t* o = (uint8_t*)malloc(n ? n : 1);
+  if (!o) return DLMZ_ENOMEM;
+  if (cudaMemcpy(o, w.hout.p, n, cudaMemcpyDeviceToHost) != cudaSuccess) {
+    free(o);
+    return DLMZ_ECUDA;
+  }
+  *out = o;
+  *out_bytes = n;
+  return DLMZ_OK;
+}
+
+int dlmz_compress(const dlmz_model* m, const void* in, size_t in_bytes, uint32_t chunk_len, const dlmz_k_policy* policy,
+                  uint8_t** out, size_t* out_bytes) {
+  return dlmz_compress_ex(m, in, in_bytes, chunk_len, policy, 0, out, out_bytes);
+}
+
+int dlmz_decompress(const dlmz_model* mc, const uint8_t* stream, size_t stream_bytes, uint8_t** out, size_t* out_bytes) {
+  if (out) *out = nullptr;
+  if (!mc || !stream || !out || !out_bytes) return DLMZ_EINVAL;
+  if (stream_bytes < 64) return DLMZ_ECORRUPT;
+  dlmz_model* m = const_cast<dlmz_model*>(mc);
+  Header h{};
+  DLMZ_TRY(read_header(stream, stream_bytes, h));
+  const uint64_t need = h.n_symbols * (h.vocab > 256 ? 4 : 1);
+  if (need > ((uint64_t)1 << 40)) return DLMZ_ECORRUPT;
+  PipeWs& w = pipe_of(m);
+  DLMZ_TRY(w.hin.ensure(stream_bytes + 16));
+  DLMZ_TRY(w.hout.ensure(need + 16));
+  DLMZ_CUDA_TRY(cudaMemcpy(w.hin.p, stream, stream_bytes, cudaMemcpyHostToDevice));
+  size_t n = 0;
+  DLMZ_TRY(decompress_device(m, w.hin.as<uint8_t>(), stream_bytes, w.hout.as<uint8_t>(), need, &n, 0));
+  uint8_t* o = (uint8_t*)malloc(n ? n : 1);
+  if (!o) return DLMZ_ENOMEM;
+  if (n && cudaMemcpy(o, w.hout.p, n, cudaMemcpyDeviceToHost) != cudaSuccess) {
+    free(o);
+    return DLMZ_ECUDA;
+  }
+  *out = o;
+  *out_bytes = n;
+  return DLMZ_OK;
+}
+
+int dlmz_check(void* stream) { return check_device(reinterpret_cast<cudaStream_t>(stream)); }
+
+// ---- step-level API ---------------------------------------------------------------------
+
+int dlmz_forward_logits(const dlmz_model* m, const int32_t* d_state, uint32_t n_chunks, uint32_t L, uint32_t row0,
+                        uint32_t rows_per_chunk, float* d_logits, void* stream) {
+  if (!m || !d_state || !d_logits) return DLMZ_EINVAL;
+  if (!device_error_word()) return DLMZ_ENOMEM;
+  return model_forward(const_cast<dlmz_model*>(m), d_state, (int)n_chunks, (int)L, (int)row0, (int)rows_per_chunk,
+                       d_logits, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32_t M, uint32_t N, uint32_t K, void* stream) {
+  if (!d_A || !d_B || !d_D || !M || !N || !K) return DLMZ_EINVAL;
+  if (!device_error_word()) return DLMZ_ENOMEM;
+  GemmEpilogue ep{};
+  ep.out = d_D;
+  ep.ldo = (int)N;
+  const bf16* A = reinterpret_cast<const bf16*>(d_A);
+  const bf16* B = reinterpret_cast<const bf16*>(d_B);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (gemm_tc_supported((int)M, (int)N, (int)K) && !((reinterpret_cast<uintptr_t>(d_A) | reinterpret_cast<uintptr_t>(d_B)) & 15))
+    return gemm_bf16_tc(A, (int)K, B, (int)K, (int)M, (int)N, (int)K, EPI_F32, ep, s);
+  return gemm_simt<bf16>(A, (int)K, B, (int)K, (int)M, (int)N, (int)K, EPI_F32, ep, s);
+}
+
+int dlmz_quantize(const float* d_logits, uint32_t rows, uint32_t V, uint32_t P, uint32_t* d_cdf, uint64_t* d_W,
+                  uint64_t* d_A, int32_t* d_Hq, int32_t* d_top, void* stream) {
+  if (!d_logits || !d_W || !d_Hq || V < 2 || P > 24 || (1ull << P) <= V) return DLMZ_EINVAL;
+  if (!device_error_word()) return DLMZ_ENOMEM;
+  return quantize_rows(d_logits, (int)rows, (int)V, (int)P, d_cdf, d_W, d_A, d_Hq, d_top, nullptr,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_select_smallest(const uint64_t* d_keys, uint32_t groups, uint32_t group_size, uint32_t k, int32_t* d_out,
+                         void* stream) {
+  if (!d_keys || !d_out || k == 0 || k > group_size || group_size > 4096) return DLMZ_EINVAL;
+  static DevBuf counts;
+  DLMZ_TRY(counts.ensure((size_t)groups * 4 + 4));
+  return select_rows<uint64_t>(nullptr, (int)groups, (int)group_size, -1, 0, (int)group_size, d_keys, 0, (int)k, 0, 0,
+                               0, (int)k, counts.as<int32_t>(), d_out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+struct dlmz_coder {
+  int nc, L, V, P;
+  uint64_t cap;
+  DevBuf cst, bytes;
+  StepBufs sb;
+  const uint8_t* in_bytes = nullptr;
+  const uint64_t* in_off = nullptr;
+  const uint32_t* in_bits = nullptr;
+};
+
+int dlmz_coder_create(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, dlmz_coder** out) {
+  if (!out) return DLMZ_EINVAL;
+  *out = nullptr;
+  if (!n_chunks || !L || V < 2 || P > 24 || (1ull << P) <= V) return DLMZ_EINVAL;
+  if (!device_error_word()) return DLMZ_ENOMEM;
+  dlmz_coder* c = new dlmz_coder();
+  c->nc = (int)n_chunks;
+  c->L = (int)L;
+  c->V = (int)V;
+  c->P = (int)P;
+  c->cap = cap_bytes_for(L, (int)P);
+  if (c->cst.ensure((size_t)n_chunks * sizeof(CoderState)) || c->bytes.ensure((size_t)n_chunks * c->cap)) {
+    dlmz_coder_destroy(c);
+    return DLMZ_ENOMEM;
+  }
+  *out = c;
+  return DLMZ_OK;
+}
+
+void dlmz_coder_destroy(dlmz_coder* c) {
+  if (!c) return;
+  c->cst.release();
+  c->bytes.release();
+  c->sb.release();
+  delete c;
+}
+
+uint32_t dlmz_coder_capacity_units(const dlmz_coder* c) { return c ? (uint32_t)(c->cap / 2) : 0; }
+
+int dlmz_coder_reset_encoder(dlmz_coder* c, void* stream) {
+  if (!c) return DLMZ_EINVAL;
+  return coder_reset(c->cst.as<CoderState>(), c->nc, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_coder_load_decoder(dlmz_coder* c, const uint8_t* d_bytes, const uint64_t* d_offsets, const uint32_t* d_bits,
+                            void* stream) {
+  if (!c || !d_bytes || !d_offsets || !d_bits) return DLMZ_EINVAL;
+  c->in_bytes = d_bytes;
+  c->in_off = d_offsets;
+  c->in_bits = d_bits;
+  return coder_load(c->cst.as<CoderState>(), c->nc, d_bytes, d_offsets, d_bits, reinterpret_cast<cudaStream_t>(stream));
+}
+
+static int step_common(dlmz_coder* c, const dlmz_k_policy* pol, const float* d_logits, uint32_t row0, uint32_t rpc,
+                       const int32_t* d_symbols, int32_t* d_state, int32_t* d_committed, bool decode, void* stream) {
+  if (!c || !d_logits || !d_state || validate_policy(pol) != DLMZ_OK) return DLMZ_EINVAL;
+  if (rpc == 0 || row0 + rpc > (uint32_t)c->L) return DLMZ_EINVAL;
+  if (!decode && !d_symbols) return DLMZ_EINVAL;
+  if (decode && !c->in_bytes) return DLMZ_EINVAL;
+  return run_step(c->sb, d_logits, c->nc, c->L, c->V, c->P, *pol, (int)row0, (int)rpc, d_symbols, d_state,
+                  c->cst.as<CoderState>(), c->bytes.as<uint8_t>(), c->cap, c->in_bytes, c->in_off, c->in_bits, decode,
+                  d_committed, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_encode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits, uint32_t row0,
+                     uint32_t rows_per_chunk, const int32_t* d_symbols, int32_t* d_state, int32_t* d_committed,
+                     void* stream) {
+  return step_common(c, policy, d_logits, row0, rows_per_chunk, d_symbols, d_state, d_committed, false, stream);
+}
+
+int dlmz_decode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits, uint32_t row0,
+                     uint32_t rows_per_chunk, int32_t* d_state, int32_t* d_committed, void* stream) {
+  return step_common(c, policy, d_logits, row0, rows_per_chunk, nullptr, d_state, d_committed, true, stream);
+}
+
+int dlmz_coder_finish(dlmz_coder* c, uint32_t* d_bits, uint8_t* d_bytes, const uint64_t* d_offsets, void* stream) {
+  if (!c || !d_bits) return DLMZ_EINVAL;
+  return coder_finish(c->cst.as<CoderState>(), c->nc, c->bytes.as<uint8_t>(), c->cap, d_bits, d_bytes, d_offsets,
+                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,283 @@
+// Logits -> integer frequency tables, CDFs and scores.
+//
+// The statistical coder (Sec. 2.1; Sec. 4 "Implementation Details") needs
+// integer tables that encoder and decoder rebuild bit-identically from the
+// same logits.  Per row l[0..V):
+//   m = max l, top = lowest v with l_v = m
+//   q_v = rint_even(min(fl32(fl32(m - l_v) * C), 8191)),  C = fl32(256 log2 e)
+//   w_v = T[q_v & 255] >> (q_v >> 8),   T[j] = round(2^31 2^(-j/256))
+//   W = sum w_v, A = sum w_v q_v (exact 64-bit integer sums: order-free)
+//   R = 2^P - V, f_v = 1 + floor(w_v R / W), f_top += R - sum floor(w_v R / W)
+//   H_q = log2q16(W) - 31*2^16 + floor(2^8 A / W)      (entropy, Sec. 3.3, 2^-16 bit)
+// Only __fsub_rn / __fmul_rn / __float2int_rn touch floating point, so the
+// result is independent of thread layout and reduction order.
+#include "kernels.cuh"
+#include "exp_table.inc"
+
+namespace dlmz {
+
+__constant__ uint32_t c_exp_table[256] = DLMZ_EXP_TABLE_INIT;
+
+__device__ __forceinline__ int quant_q(float m, float l) {
+  const float t = __fmul_rn(__fsub_rn(m, l), __uint_as_float(DLMZ_QSCALE_BITS));
+  return __float2int_rn(fminf(t, 8191.0f));
+}
+
+__device__ __forceinline__ uint32_t quant_w(const uint32_t* T, int q) { return T[q & 255] >> (q >> 8); }
+
+// Digit-by-digit binary logarithm: ~floor(2^16 log2 W) for W >= 2^31.
+__device__ __forceinline__ uint32_t log2q16(uint64_t W) {
+  const int n = 63 - __clzll((long long)W);
+  uint64_t y = W >> (n - 31);
+  uint32_t frac = 0;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    y = (y * y) >> 31;
+    frac <<= 1;
+    if (y >= (1ull << 32)) {
+      frac |= 1;
+      y >>= 1;
+    }
+  }
+  return ((uint32_t)n << 16) + frac;
+}
+
+__device__ __forceinline__ int32_t entropy_q(uint64_t W, uint64_t A) {
+  const uint64_t qt = A / W, rm = A % W;
+  return (int32_t)((int64_t)log2q16(W) - (31ll << 16) + (int64_t)((qt << 8) + ((rm << 8) / W)));
+}
+
+__device__ __forceinline__ void argmax_merge(float& m, int& i, float m2, int i2) {
+  if (m2 > m || (m2 == m && i2 < i)) {
+    m = m2;
+    i = i2;
+  }
+}
+
+// ---- warp per row, V <= 32 * NPL, values in registers ------------------------------
+template <int NPL>
+__global__ void __launch_bounds__(256) quantize_warp_kernel(const float* __restrict__ logits, int rows, int V, int P,
+                                                            uint32_t* __restrict__ cdf, uint64_t* __restrict__ Wout,
+                                                            uint64_t* __restrict__ Aout, int32_t* __restrict__ Hq,
+                                                            int32_t* __restrict__ topout, float* __restrict__ mxout,
+                                                            int* err) {
+  __shared__ uint32_t T[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) T[i] = c_exp_table[i];
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  if (r >= rows) return;
+  const float* lr = logits + (size_t)r * V;
+  float x[NPL];
+  float m = -INFINITY;
+  int mi = 0x7fffffff;
+  bool finite = true;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int v = lane + 32 * i;
+    x[i] = v < V ? lr[v] : -INFINITY;
+    if (v < V) {
+      finite &= isfinite(x[i]);
+      argmax_merge(m, mi, x[i], v);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const int i2 = __shfl_xor_sync(0xffffffffu, mi, o);
+    argmax_merge(m, mi, m2, i2);
+  }
+  if (!__all_sync(0xffffffffu, finite)) {
+    if (lane == 0) atomicOr(err, ERR_NONFINITE);
+    m = 0.f;  // keep going with defined values; the call reports EBADINPUT
+  }
+  uint32_t w[NPL];
+  uint64_t Ws = 0, As = 0;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int v = lane + 32 * i;
+    if (v < V) {
+      const int q = isfinite(x[i]) ? quant_q(m, x[i]) : 8191;
+      w[i] = quant_w(T, q);
+      Ws += w[i];
+      As += (uint64_t)w[i] * (uint64_t)q;
+    } else {
+      w[i] = 0;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    Ws += __shfl_xor_sync(0xffffffffu, Ws, o);
+    As += __shfl_xor_sync(0xffffffffu, As, o);
+  }
+  if (lane == 0) {
+    Wout[r] = Ws;
+    if (Aout) Aout[r] = As;
+    Hq[r] = entropy_q(Ws, As);
+    if (topout) topout[r] = mi;
+    if (mxout) mxout[r] = m;
+  }
+  if (!cdf) return;
+  const uint64_t R = (1ull << P) - (uint64_t)V;
+  uint64_t fl[NPL];
+  uint64_t fsum = 0;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    fl[i] = (uint64_t)w[i] * R / Ws;
+    fsum += fl[i];
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) fsum += __shfl_xor_sync(0xffffffffu, fsum, o);
+  const uint32_t D = (uint32_t)(R - fsum);
+  uint32_t* cr = cdf + (size_t)r * (V + 1);
+  uint32_t carry = 0;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int v = lane + 32 * i;
+    uint32_t f = v < V ? 1u + (uint32_t)fl[i] + (v == mi ? D : 0u) : 0u;
+    uint32_t inc = f;  // inclusive scan across the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += t;
+    }
+    if (v < V) cr[v + 1] = carry + inc;
+    carry += __shfl_sync(0xffffffffu, inc, 31);
+  }
+  if (lane == 0) cr[0] = 0;
+}
+
+// ---- CTA per row, any V: passes over the row through L1/L2 ---------------------------
+template <typename U>
+__device__ __forceinline__ U block_sum(U v, U* red) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  U t = 0;
+  for (int i = 0; i < nw; ++i) t += red[i];
+  return t;
+}
+
+constexpr int QT = 512;  // threads per row in the CTA kernel
+
+__global__ void __launch_bounds__(QT) quantize_cta_kernel(const float* __restrict__ logits, int rows, int V, int P,
+                                                         uint32_t* __restrict__ cdf, uint64_t* __restrict__ Wout,
+                                                         uint64_t* __restrict__ Aout, int32_t* __restrict__ Hq,
+                                                         int32_t* __restrict__ topout, float* __restrict__ mxout,
+                                                         int* err) {
+  __shared__ uint32_t T[256];
+  __shared__ float redf[QT / 32];
+  __shared__ int redi[QT / 32];
+  __shared__ uint64_t redu[QT / 32];
+  __shared__ uint64_t seg[QT];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) T[i] = c_exp_table[i];
+  const int r = blockIdx.x;
+  const float* lr = logits + (size_t)r * V;
+  // pass 1: max / lowest argmax / finiteness
+  float m = -INFINITY;
+  int mi = 0x7fffffff;
+  int bad = 0;
+  for (int v = threadIdx.x; v < V; v += QT) {
+    const float x = lr[v];
+    bad |= !isfinite(x);
+    argmax_merge(m, mi, x, v);
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    argmax_merge(m, mi, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, mi, o));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, o);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    redf[threadIdx.x >> 5] = m;
+    redi[threadIdx.x >> 5] = mi | (bad ? 0x80000000 : 0);
+  }
+  __syncthreads();
+  m = -INFINITY;
+  mi = 0x7fffffff;
+  bad = 0;
+  for (int i = 0; i < QT / 32; ++i) {
+    bad |= redi[i] < 0;
+    argmax_merge(m, mi, redf[i], redi[i] & 0x7fffffff);
+  }
+  if (bad) {
+    if (threadIdx.x == 0) atomicOr(err, ERR_NONFINITE);
+    m = 0.f;
+  }
+  // pass 2: W, A
+  uint64_t Ws = 0, As = 0;
+  for (int v = threadIdx.x; v < V; v += QT) {
+    const float x = lr[v];
+    const int q = isfinite(x) ? quant_q(m, x) : 8191;
+    const uint32_t w = quant_w(T, q);
+    Ws += w;
+    As += (uint64_t)w * (uint64_t)q;
+  }
+  Ws = block_sum(Ws, redu);
+  As = block_sum(As, redu);
+  if (threadIdx.x == 0) {
+    Wout[r] = Ws;
+    if (Aout) Aout[r] = As;
+    Hq[r] = entropy_q(Ws, As);
+    if (topout) topout[r] = mi;
+    if (mxout) mxout[r] = m;
+  }
+  if (!cdf) return;
+  // pass 3: per-thread contiguous segment sums of f (without the remainder)
+  const uint64_t R = (1ull << P) - (uint64_t)V;
+  const int segl = (V + QT - 1) / QT;
+  const int v0 = threadIdx.x * segl, v1 = min(V, v0 + segl);
+  uint64_t s = 0;
+  for (int v = v0; v < v1; ++v) {
+    const float x = lr[v];
+    const int q = isfinite(x) ? quant_q(m, x) : 8191;
+    s += 1 + (uint64_t)quant_w(T, q) * R / Ws;
+  }
+  seg[threadIdx.x] = s;
+  __syncthreads();
+  // exclusive scan of the segment sums (QT entries, one warp)
+  if (threadIdx.x < 32) {
+    uint64_t run = 0;
+    for (int base = 0; base < QT; base += 32) {
+      uint64_t val = seg[base + threadIdx.x], inc = val;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint64_t t = __shfl_up_sync(0xffffffffu, inc, o);
+        if (threadIdx.x >= o) inc += t;
+      }
+      seg[base + threadIdx.x] = run + inc - val;
+      run += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    if (threadIdx.x == 0) redu[0] = run;
+  }
+  __syncthreads();
+  const uint32_t D = (uint32_t)((1ull << P) - redu[0]);
+  // pass 4: write the CDF (remainder D added from top + 1 on)
+  uint32_t* cr = cdf + (size_t)r * (V + 1);
+  uint64_t c = seg[threadIdx.x] + (v0 > mi ? D : 0);
+  for (int v = v0; v < v1; ++v) {
+    const float x = lr[v];
+    const int q = isfinite(x) ? quant_q(m, x) : 8191;
+    c += 1 + (uint64_t)quant_w(T, q) * R / Ws + (v == mi ? D : 0);
+    cr[v + 1] = (uint32_t)c;
+  }
+  if (threadIdx.x == 0) cr[0] = 0;
+}
+
+int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, uint64_t* W, uint64_t* A, int32_t* Hq,
+                  int32_t* top, float* mx, cudaStream_t s) {
+  if (rows == 0) return DLMZ_OK;
+  int* err = device_error_word();
+  const int grid = (rows + 7) / 8;
+  if (V <= 32) quantize_warp_kernel<1><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  else if (V <= 64) quantize_warp_kernel<2><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  else if (V <= 128) quantize_warp_kernel<4><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  else if (V <= 256) quantize_warp_kernel<8><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  else if (V <= 512) quantize_warp_kernel<16><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  else quantize_cta_kernel<<<rows, QT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  return launch_status();
+}
+
+}  // namespace dlmz

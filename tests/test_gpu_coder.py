@@ -1,0 +1,102 @@
+"""GPU quantise + select + range-code steps vs the oracle on identical logits.
+
+Logits come from the seeded ``sources.synthetic_logits`` for (window, step),
+so both sides code with the same tables: the streams must agree bit for bit,
+and the GPU decoder must recover the symbols from the GPU streams.
+"""
+import numpy as np
+import pytest
+
+from oracle import pipeline as OP
+from oracle import quantizer as Q
+from oracle import selector as S
+from paper_2608_11249_gb300 import sources
+from tests.gpu_helpers import dlmz, ptr, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu_run(d, symbols, V, pol, opol, seed, L):
+    """Encode all windows on the GPU, then decode; return (bits, streams, decoded)."""
+    import torch
+    nc = symbols.shape[0]
+    P = Q.precision_for_vocab(V)
+    coder = d.Coder(nc, L, V, P)
+    coder.reset_encoder()
+    sym = to_dev(symbols.astype(np.int32))
+    state = torch.full((nc, L), V, dtype=torch.int32, device="cuda")
+    committed = torch.zeros(nc, dtype=torch.int32, device="cuda")
+
+    def steps(fn):
+        step = 0
+        if opol.kind == S.TOPK_CONF:
+            B = opol.block or L
+            for b0 in range(0, L, B):
+                Bl = min(B, L - b0)
+                rem = Bl
+                while rem > 0:
+                    lg = np.concatenate([sources.synthetic_logits(seed, c, step, L, V)[b0:b0 + Bl] for c in range(nc)])
+                    fn(to_dev(lg), b0, Bl)
+                    rem -= min(opol.k, rem)
+                    step += 1
+        else:
+            while True:
+                lg = np.concatenate([sources.synthetic_logits(seed, c, step, L, V) for c in range(nc)])
+                fn(to_dev(lg), 0, L)
+                step += 1
+                if int((state == V).sum().item()) == 0:
+                    break
+                assert step <= L
+
+    steps(lambda lg, r0, rpc: coder.encode_step(pol, ptr(lg), r0, rpc, ptr(sym), ptr(state), ptr(committed)))
+    d.check()
+    assert np.array_equal(state.cpu().numpy(), symbols)
+    bits = torch.empty(nc, dtype=torch.int32, device="cuda")
+    cap = coder.capacity_units * 2
+    raw = torch.zeros(nc * cap, dtype=torch.uint8, device="cuda")
+    coder.finish(ptr(bits), ptr(raw))
+    d.check()
+    bits_h = bits.cpu().numpy().astype(np.int64)
+    raw_h = raw.cpu().numpy()
+    streams = [bytes(raw_h[c * cap:c * cap + (bits_h[c] + 7) // 8]) for c in range(nc)]
+    # decode from a packed copy of the streams
+    offs = np.concatenate([[0], np.cumsum([(b + 7) // 8 for b in bits_h])[:-1]]).astype(np.uint64)
+    packed = np.frombuffer(b"".join(streams) + b"\0" * 8, dtype=np.uint8)
+    dcoder = d.Coder(nc, L, V, P)
+    d_packed, d_offs, d_bits = to_dev(packed), to_dev(offs.view(np.int64)), to_dev(bits_h.astype(np.int32))
+    dcoder.load_decoder(ptr(d_packed), ptr(d_offs), ptr(d_bits))
+    state.fill_(V)
+    steps(lambda lg, r0, rpc: dcoder.decode_step(pol, ptr(lg), r0, rpc, ptr(state), ptr(committed)))
+    d.check()
+    return bits_h, streams, state.cpu().numpy()
+
+
+CASES = [
+    # V, L, nc, policy
+    (4, 6, 5, S.Policy(kind=S.TOPK_CONF, k=2, block=4)),
+    (256, 100, 3, S.Policy(kind=S.TOPK_CONF, k=4, block=64)),
+    (256, 512, 2, S.Policy(kind=S.TOPK_CONF, k=8, block=128)),
+    (37, 50, 4, S.Policy(kind=S.TOPK_CONF, k=3, block=0)),
+    (256, 64, 3, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=0)),
+    (256, 80, 2, S.Policy(kind=S.ENTROPY, tau_bits=2.0, k_min=2, k_max=5)),
+    (5000, 40, 2, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=64)),
+    (5000, 33, 2, S.Policy(kind=S.TOPK_CONF, k=16, block=0)),
+]
+
+
+@pytest.mark.parametrize("ci", range(len(CASES)))
+def test_steps_bit_exact_and_decode(dev, ci):
+    d = dlmz()
+    V, L, nc, opol = CASES[ci]
+    seed = 100 + ci
+    rng = np.random.default_rng(seed)
+    symbols = rng.integers(0, V, (nc, L))
+    pol = d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max)
+    bits, streams, decoded = _gpu_run(d, symbols, V, pol, opol, seed, L)
+    P = Q.precision_for_vocab(V)
+    for c in range(nc):
+        fn = lambda step, state, rows, c=c: sources.synthetic_logits(seed, c, step, L, V)[rows]
+        (obits, obytes), _ = OP.encode_window(symbols[c], V, fn, opol, P)
+        assert int(bits[c]) == obits, (c, int(bits[c]), obits)
+        assert streams[c] == obytes, c
+    assert np.array_equal(decoded, symbols)

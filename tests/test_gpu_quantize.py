@@ -1,0 +1,72 @@
+"""GPU quantiser vs the oracle, bit-exact on identical float32 logits."""
+import numpy as np
+import pytest
+
+from oracle import quantizer as Q
+from paper_2608_11249_gb300 import sources
+from tests.gpu_helpers import dlmz, ptr, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _rows(V, n, seed):
+    l = sources.synthetic_logits(seed, 0, 0, n, V)
+    extra = [np.zeros(V), np.full(V, -1e30), np.linspace(-100, 100, V)]
+    x = np.zeros(V); x[V // 3] = 1e6; extra.append(x)
+    x = np.full(V, -3e38); x[-1] = 3e38; extra.append(x)
+    x = np.zeros(V); x[[1, V - 1]] = 7.0; extra.append(x)  # tie for the maximum
+    return np.concatenate([l, np.array(extra, dtype=np.float32)]).astype(np.float32)
+
+
+@pytest.mark.parametrize("V,n", [(2, 9), (4, 33), (37, 70), (256, 300), (300, 50), (512, 40), (1000, 20),
+                                 (5000, 17), (126464, 5), (152064, 3)])
+def test_quantize_bit_exact(dev, V, n):
+    import torch
+    d = dlmz()
+    l = _rows(V, n, V)
+    rows = l.shape[0]
+    P = Q.precision_for_vocab(V)
+    ref = Q.quantize(l, P)
+    dl = to_dev(l)
+    cdf = torch.empty(rows, V + 1, dtype=torch.int32, device="cuda")
+    W = torch.empty(rows, dtype=torch.int64, device="cuda")
+    A = torch.empty(rows, dtype=torch.int64, device="cuda")
+    Hq = torch.empty(rows, dtype=torch.int32, device="cuda")
+    top = torch.empty(rows, dtype=torch.int32, device="cuda")
+    d.quantize(ptr(dl), rows, V, P, ptr(cdf), ptr(W), ptr(A), ptr(Hq), ptr(top))
+    d.check()
+    assert np.array_equal(cdf.cpu().numpy().view(np.uint32), ref["cdf"])
+    assert np.array_equal(W.cpu().numpy().view(np.uint64), ref["W"])
+    assert np.array_equal(A.cpu().numpy().view(np.uint64), ref["A"])
+    assert np.array_equal(Hq.cpu().numpy(), ref["Hq"].astype(np.int32))
+    assert np.array_equal(top.cpu().numpy(), ref["top"].astype(np.int32))
+
+
+def test_quantize_isolated_workload_rows(dev):
+    """Rows of the isolated quantise+select workload (N(0,3) + spike U(5,15), V = 126464)."""
+    import torch
+    d = dlmz()
+    V, rows = 126464, 24
+    l = sources.spiked_rows(0, 1000, rows, V)
+    ref = Q.quantize(l, 24)
+    cdf = torch.empty(rows, V + 1, dtype=torch.int32, device="cuda")
+    W = torch.empty(rows, dtype=torch.int64, device="cuda")
+    Hq = torch.empty(rows, dtype=torch.int32, device="cuda")
+    d.quantize(ptr(to_dev(l)), rows, V, 24, ptr(cdf), ptr(W), 0, ptr(Hq), 0)
+    d.check()
+    assert np.array_equal(cdf.cpu().numpy().view(np.uint32), ref["cdf"])
+    assert np.array_equal(Hq.cpu().numpy(), ref["Hq"].astype(np.int32))
+
+
+def test_quantize_rejects_non_finite(dev):
+    import torch
+    d = dlmz()
+    l = np.zeros((3, 64), dtype=np.float32)
+    l[1, 5] = np.nan
+    W = torch.empty(3, dtype=torch.int64, device="cuda")
+    Hq = torch.empty(3, dtype=torch.int32, device="cuda")
+    d.quantize(ptr(to_dev(l)), 3, 64, 16, 0, ptr(W), 0, ptr(Hq), 0)
+    with pytest.raises(d.DlmzError) as e:
+        d.check()
+    assert e.value.code == d.EBADINPUT
+    d.check()  # flag cleared

@@ -1,0 +1,120 @@
+"""End-to-end GPU compress / decompress through the C ABI.
+
+Round trips must be bit-exact; the GPU container's size must be within
+0.5% of the oracle's own end-to-end compression of the same input with the
+same model (the two forwards differ by rounding, so the streams differ).
+"""
+import numpy as np
+import pytest
+
+from oracle import container as OC
+from oracle import model as OM
+from oracle import pipeline as OP
+from oracle import selector as S
+from paper_2608_11249_gb300 import sources
+from tests.gpu_helpers import dlmz, ptr, to_dev
+
+pytestmark = pytest.mark.gpu
+
+CASES = [
+    # model (nl, d, h, kv, F, V, dtype), data kind, n, chunk_len, policy, batch_chunks
+    ((1, 32, 2, 2, 64, 256, "f32"), "bytes", 1500, 512, S.Policy(kind=S.TOPK_CONF, k=4, block=64), 0),
+    ((2, 256, 4, 4, 256, 256, "bf16"), "bytes", 1100, 256, S.Policy(kind=S.TOPK_CONF, k=8, block=128), 3),
+    ((1, 64, 4, 2, 128, 5000, "f32"), "tokens", 300, 100, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=8), 0),
+    ((2, 256, 4, 4, 256, 256, "bf16"), "bytes", 600, 200, S.Policy(kind=S.ENTROPY, tau_bits=6.0, k_min=2, k_max=16), 2),
+]
+
+
+def _data(kind, n, V):
+    if kind == "bytes":
+        return sources.markov_bytes(n, seed=2)
+    return sources.tokens_to_bytes(sources.zipf_bigram_tokens(n, V, seed=2))
+
+
+def _model(d, spec, seed):
+    nl, dm, h, kv, F, V, dt = spec
+    return d.Model(nl, dm, h, kv, F, V, d.BF16 if dt == "bf16" else d.FP32, seed=seed)
+
+
+@pytest.mark.parametrize("ci", range(len(CASES)))
+def test_roundtrip_and_size_vs_oracle(dev, ci):
+    d = dlmz()
+    spec, kind, n, L, opol, bc = CASES[ci]
+    m = _model(d, spec, 40 + ci)
+    data = _data(kind, n, spec[5])
+    pol = d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max)
+    blob = m.compress(data, L, pol, bc)
+    assert m.decompress(blob) == data
+    h, streams = OC.read(blob)  # the oracle's container reader parses the GPU file
+    assert h.fingerprint == m.fingerprint and h.chunk_len == L and h.n_symbols * (4 if kind == "tokens" else 1) == len(data)
+    w = OM.Weights(OM.ModelConfig(*spec, seed=40 + ci))
+    oblob = OP.compress(w, data, L, opol)
+    assert abs(len(blob) - len(oblob)) <= 0.005 * len(oblob) + 8, (len(blob), len(oblob))
+
+
+def test_edge_inputs(dev):
+    d = dlmz()
+    m = _model(d, (1, 32, 2, 2, 64, 256, "f32"), 1)
+    pol = d.policy(d.TOPK_CONF, 3, 8)
+    for data in (b"", b"\x07", bytes(range(256)), b"\xff" * 33):
+        blob = m.compress(data, 16, pol)
+        assert m.decompress(blob) == data
+    tm = _model(d, (1, 32, 2, 2, 64, 300, "f32"), 1)
+    with pytest.raises(d.DlmzError) as e:
+        tm.compress(b"\x01\x02\x03", 16, pol)
+    assert e.value.code == d.EBADINPUT
+    with pytest.raises(d.DlmzError) as e:
+        tm.compress(np.array([300], dtype="<u4").tobytes(), 16, pol)
+    assert e.value.code == d.EBADINPUT
+    with pytest.raises(d.DlmzError):
+        m.compress(b"abc", 0, pol)
+    with pytest.raises(d.DlmzError):
+        m.compress(b"abc", 4, d.policy(d.TOPK_CONF, 0))
+
+
+def test_device_api_matches_host_api_and_batches_agree(dev):
+    import torch
+    d = dlmz()
+    m = _model(d, (2, 256, 4, 4, 256, 256, "bf16"), 7)
+    data = sources.markov_bytes(2000, seed=5)
+    pol = d.policy(d.TOPK_CONF, 8, 64)
+    a = m.compress(data, 256, pol, 1)
+    b = m.compress(data, 256, pol, 4)
+    # batch composition changes no stream (batch-invariant forward): only the header's batch field differs
+    assert a[:24] == b[:24] and a[28:] == b[28:]
+    din = to_dev(np.frombuffer(data, dtype=np.uint8))
+    cap = m.compress_bound(len(data), 256)
+    dout = torch.empty(cap, dtype=torch.uint8, device="cuda")
+    n = m.compress_device(ptr(din), len(data), 256, pol, ptr(dout), cap, batch_chunks=4)
+    assert bytes(dout[:n].cpu().numpy()) == b
+    back = torch.empty(len(data), dtype=torch.uint8, device="cuda")
+    k = m.decompress_device(ptr(dout), n, ptr(back), len(data))
+    assert k == len(data) and bytes(back.cpu().numpy()) == data
+
+
+def test_corrupt_containers_are_rejected(dev):
+    d = dlmz()
+    m = _model(d, (1, 32, 2, 2, 64, 256, "f32"), 9)
+    data = sources.markov_bytes(400, seed=9)
+    blob = m.compress(data, 128, d.policy(d.TOPK_CONF, 4, 32))
+    bad = [b"XXXX" + blob[4:], blob[:4] + b"\x09" + blob[5:], blob[:-1], blob[:30], blob + b"\0"]
+    for x in bad:
+        with pytest.raises(d.DlmzError) as e:
+            m.decompress(x)
+        assert e.value.code == d.ECORRUPT
+    other = _model(d, (1, 32, 2, 2, 64, 256, "f32"), 10)
+    with pytest.raises(d.DlmzError) as e:
+        other.decompress(blob)
+    assert e.value.code == d.EMODEL
+    rng = np.random.default_rng(0)
+    for _ in range(20):  # flipped bits: rejected by the checksum or the coder, never a crash;
+        x = bytearray(blob)  # a flip inside a stream's final zero padding may still decode correctly
+        i = int(rng.integers(70, len(x)))
+        x[i] ^= 1 << int(rng.integers(0, 8))
+        try:
+            out = m.decompress(bytes(x))
+        except d.DlmzError as e:
+            assert e.code == d.ECORRUPT
+        else:
+            assert out == data
+    d.check()
