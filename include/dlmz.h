@@ -203,6 +203,24 @@ DLMZ_API uint32_t dlmz_coder_capacity_units(const dlmz_coder* c);
  * that cannot come from the encoder, ETIMEOUT, EBADINPUT). */
 DLMZ_API int dlmz_check(void* stream);
 
+/* ---- live profiling (not part of the method) ------------------------------
+ * Between dlmz_profile_begin and dlmz_profile_end the library records CUDA
+ * events on each launch's stream around every kernel and counts launches.
+ * Classes: 0 tensor-core GEMM, 1 CUDA-core GEMM, 2 attention, 3 quantiser,
+ * 4 selector, 5 coder, 6 embedding/norm/RoPE/SwiGLU, 7 other.  flops and
+ * bytes are the algorithmic work of the timed launches (2MNK for a GEMM,
+ * 4 L^2 hd per window-head for attention, logits read for the quantiser). */
+typedef struct {
+  uint64_t launches;     /* every kernel launched by the library */
+  uint64_t n[8];         /* timed launches per class */
+  double ms[8];          /* summed launch durations per class (ms) */
+  double flops[8];
+  double bytes[8];
+} dlmz_profile;
+DLMZ_API int dlmz_profile_begin(void);
+/* Synchronises the device and fills *out. */
+DLMZ_API int dlmz_profile_end(dlmz_profile* out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -216,6 +216,7 @@ int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int nh, int
   if ((ld % 8) || (d % 8) || (reinterpret_cast<uintptr_t>(qkv) & 15)) return DLMZ_EINVAL;
   dim3 grid((L + fa::BMQ - 1) / fa::BMQ, nh, n_chunks);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
+  ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
   if (hd == 64) {
     constexpr int SM = 5 * 64 * 64 * 2;
     fa::flash_kernel<64><<<grid, 128, SM, s>>>(qkv, ld, L, nh, nkv, d, out, scale_log2);

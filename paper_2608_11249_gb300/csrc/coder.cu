@@ -104,6 +104,7 @@ int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0
     DLMZ_CUDA_TRY(cudaFuncSetAttribute(select_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024));
     attr = true;
   }
+  ProfScope prof(PROF_SELECT, s, 0, (double)n_chunks * rpc * (sizeof(K) + 4));
   select_kernel<K><<<n_chunks, 256, smem, s>>>(state, L, mask_id, row0, rpc, keys, n_rule, k, tau_q, k_min, k_max,
                                                kcap, sel_count, sel_pos);
   return launch_status();
@@ -285,6 +286,7 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
 
 int code_step(const CodeArgs& a, bool decode, int n_chunks, cudaStream_t s) {
   if (n_chunks == 0) return DLMZ_OK;
+  ProfScope prof(PROF_CODE, s, 0, 0);
   if (decode) code_kernel<true><<<n_chunks, CT, 0, s>>>(a);
   else code_kernel<false><<<n_chunks, CT, 0, s>>>(a);
   return launch_status();

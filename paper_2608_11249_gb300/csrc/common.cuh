@@ -34,7 +34,29 @@ int* device_error_word();  // lazily allocated device int
     if (r_ != DLMZ_OK) return r_; \
   } while (0)
 
+// ---- live per-kernel-class profiler (CUDA events on the launch stream) ----------
+enum ProfClass { PROF_GEMM_TC = 0, PROF_GEMM_SIMT, PROF_ATTN, PROF_QUANT, PROF_SELECT, PROF_CODE, PROF_LAYER,
+                 PROF_OTHER, PROF_NCLASS };
+bool prof_on();
+void prof_count_launch();
+void prof_record(int cls, cudaStream_t s, bool start, double flops, double bytes);
+
+// Records CUDA events around the launches of one kernel class while
+// profiling is enabled (dlmz_profile_begin / dlmz_profile_end).
+struct ProfScope {
+  int cls;
+  cudaStream_t s;
+  double flops, bytes;
+  ProfScope(int c, cudaStream_t st, double f, double b) : cls(c), s(st), flops(f), bytes(b) {
+    if (prof_on()) prof_record(cls, s, true, 0, 0);
+  }
+  ~ProfScope() {
+    if (prof_on()) prof_record(cls, s, false, flops, bytes);
+  }
+};
+
 inline int launch_status() {
+  prof_count_launch();
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     fprintf(stderr, "dlmz: kernel launch failed: %s\n", cudaGetErrorString(e));

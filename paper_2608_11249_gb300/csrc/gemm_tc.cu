@@ -382,6 +382,9 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   }
   const int tiles = ((M + BM - 1) / BM) * (N / BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
+  const double out_b = EPI == EPI_F32 ? 4.0 * M * N : EPI == EPI_RESID_F32 ? 8.0 * M * N
+                     : EPI == EPI_SWIGLU_BF16 ? 1.0 * M * N : 2.0 * M * N;
+  ProfScope prof(PROF_GEMM_TC, s, 2.0 * M * N * K, 2.0 * M * K + 2.0 * N * K + out_b);
   gemm_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(a, b, M, N, K, ep, device_error_word());
   return launch_status();
 }

@@ -22,6 +22,7 @@ __global__ void embed_kernel(const int32_t* __restrict__ state, int n, const T* 
 template <typename T>
 int embed(const int32_t* state, int n, const T* E, int d, float* x, cudaStream_t s) {
   if (n == 0) return DLMZ_OK;
+  ProfScope prof(PROF_LAYER, s, 0, (double)n * d * (sizeof(T) + 4));
   embed_kernel<T><<<n, 128, 0, s>>>(state, n, E, d, x);
   return launch_status();
 }
@@ -50,6 +51,7 @@ template <typename OutT>
 int rmsnorm(const float* x, int rows, int d, const float* g, float eps, OutT* h, int L, int row0, int rpc,
             cudaStream_t s) {
   if (rows == 0) return DLMZ_OK;
+  ProfScope prof(PROF_LAYER, s, 0, (double)rows * d * (4 + sizeof(OutT)));
   rmsnorm_kernel<OutT><<<(rows + 7) / 8, 256, 0, s>>>(x, rows, d, g, eps, h, L, row0, rpc);
   return launch_status();
 }
@@ -77,6 +79,7 @@ __global__ void rope_kernel(T* __restrict__ qkv, int n, int ld, int nh, int hd, 
 template <typename T>
 int rope_inplace(T* qkv, int n, int ld, int nh, int hd, int L, const float2* cs, cudaStream_t s) {
   if (n == 0) return DLMZ_OK;
+  ProfScope prof(PROF_LAYER, s, 0, 2.0 * n * nh * hd * sizeof(T));
   rope_kernel<T><<<n, 128, 0, s>>>(qkv, n, ld, nh, hd, L, cs);
   return launch_status();
 }
@@ -99,6 +102,7 @@ __global__ void swiglu_kernel(const float* __restrict__ gu, int n, int F, int gb
 template <typename T>
 int swiglu(const float* gu, int n, int F, int gb, T* out, cudaStream_t s) {
   if (n == 0) return DLMZ_OK;
+  ProfScope prof(PROF_LAYER, s, 0, (double)n * F * (8 + sizeof(T)));
   swiglu_kernel<T><<<n, 256, 0, s>>>(gu, n, F, gb, out);
   return launch_status();
 }
@@ -163,6 +167,7 @@ int gemm_simt(const T* A, int lda, const T* B, int ldb, int M, int N, int K, int
   if (epi != EPI_F32 && epi != EPI_RESID_F32 && epi != EPI_BF16) return DLMZ_EINVAL;
   if (M == 0 || N == 0) return DLMZ_OK;
   dim3 grid((N + 63) / 64, (M + 63) / 64);
+  ProfScope prof(PROF_GEMM_SIMT, s, 2.0 * M * N * K, (double)sizeof(T) * ((double)M * K + (double)N * K) + 4.0 * M * N);
   gemm_simt_kernel<T><<<grid, 256, 0, s>>>(A, lda, B, ldb, M, N, K, epi, ep);
   return launch_status();
 }
@@ -229,6 +234,8 @@ int attention_simt(const T* qkv, int ld, int n_chunks, int L, int nh, int nkv, i
                    cudaStream_t s) {
   if (n_chunks == 0 || L == 0) return DLMZ_OK;
   dim3 grid((L + 63) / 64, nh, n_chunks);
+  ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd,
+                 (double)sizeof(T) * n_chunks * L * (ld + d));
   switch (hd) {
     case 8: attention_simt_kernel<T, 8><<<grid, 64, 0, s>>>(qkv, ld, L, nh, nkv, d, out); break;
     case 16: attention_simt_kernel<T, 16><<<grid, 64, 0, s>>>(qkv, ld, L, nh, nkv, d, out); break;

@@ -271,6 +271,7 @@ int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, ui
   if (rows == 0) return DLMZ_OK;
   int* err = device_error_word();
   const int grid = (rows + 7) / 8;
+  ProfScope prof(PROF_QUANT, s, 0, (double)rows * V * 4 + (cdf ? (double)rows * (V + 1) * 4 : 0.0));
   if (V <= 32) quantize_warp_kernel<1><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V <= 64) quantize_warp_kernel<2><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V <= 128) quantize_warp_kernel<4><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);

@@ -10,7 +10,8 @@ torch CUDA tensor) and streams as integer handles (``torch.cuda.Stream
 """
 import ctypes
 import os
-from ctypes import POINTER, Structure, byref, c_char_p, c_float, c_int, c_size_t, c_uint8, c_uint32, c_uint64, c_void_p
+from ctypes import (POINTER, Structure, byref, c_char_p, c_double, c_float, c_int, c_size_t, c_uint8, c_uint32,
+                    c_uint64, c_void_p)
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdlmz.so")
 if not os.path.exists(_LIB_PATH):
@@ -37,6 +38,11 @@ class ModelConfig(Structure):
 class KPolicy(Structure):
     _fields_ = [("kind", c_uint32), ("k", c_uint32), ("block", c_uint32), ("tau_bits", c_float),
                 ("k_min", c_uint32), ("k_max", c_uint32)]
+
+
+class Profile(Structure):
+    _fields_ = [("launches", c_uint64), ("n", c_uint64 * 8), ("ms", c_double * 8), ("flops", c_double * 8),
+                ("bytes", c_double * 8)]
 
 
 def _sig(name, restype, *args):
@@ -74,6 +80,8 @@ _sig("dlmz_decode_step", c_int, _P, POINTER(KPolicy), _P, c_uint32, c_uint32, _P
 _sig("dlmz_coder_finish", c_int, _P, _P, _P, _P, _P)
 _sig("dlmz_coder_capacity_units", c_uint32, _P)
 _sig("dlmz_check", c_int, _P)
+_sig("dlmz_profile_begin", c_int)
+_sig("dlmz_profile_end", c_int, POINTER(Profile))
 
 
 def _ok(rc, where):
@@ -165,6 +173,14 @@ def quantize(d_logits, rows, V, P, d_cdf, d_W, d_A, d_Hq, d_top, stream=0):
 
 def select_smallest(d_keys, groups, group_size, k, d_out, stream=0):
     _ok(lib.dlmz_select_smallest(d_keys, groups, group_size, k, d_out, stream), "dlmz_select_smallest")
+
+
+def profile_begin():
+    _ok(lib.dlmz_profile_begin(), "dlmz_profile_begin")
+
+
+def profile_end(prof):
+    _ok(lib.dlmz_profile_end(byref(prof)), "dlmz_profile_end")
 
 
 def check(stream=0):

@@ -11,7 +11,7 @@ def dlmz():
 
 def to_dev(a):
     import torch
-    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    return torch.from_numpy(np.array(a, copy=True, order="C")).cuda()
 
 
 def ptr(t):
