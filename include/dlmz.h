@@ -167,6 +167,21 @@ DLMZ_API int dlmz_quantize(const float* d_logits, uint32_t rows, uint32_t V, uin
 DLMZ_API int dlmz_select_smallest(const uint64_t* d_keys, uint32_t groups, uint32_t group_size, uint32_t k,
                          int32_t* d_out, void* stream);
 
+/* Allocation-free dlmz_select_smallest (the paper has no counterpart: this is
+ * a deployment entry point).  For callers that cannot call cudaMalloc -- code
+ * whose device memory belongs to another allocator, latency-critical paths
+ * that cannot take cudaMalloc's implicit device synchronisation, hosts with a
+ * fixed device-memory budget.  Same arguments and results as
+ * dlmz_select_smallest; the kernel's scratch (one count per group) is a
+ * static device array of 65536 int32 (256 KiB, held by every GPU that loads
+ * the library until exit), so groups > 65536 returns DLMZ_EINVAL.  The first
+ * call on a device looks up the array's device address (cudaGetSymbolAddress)
+ * and must come before any stream capture.  Calls share the array: calls that
+ * overlap on the GPU race; sequential calls need no clearing between them.
+ * It calls no cudaMalloc or cudaFree. */
+DLMZ_API int dlmz_select_smallest_noalloc(const uint64_t* d_keys, uint32_t groups, uint32_t group_size, uint32_t k,
+                                          int32_t* d_out, void* stream);
+
 /* Opaque per-batch coder state (range coder, one stream per window). */
 typedef struct dlmz_coder dlmz_coder;
 /* Allocate coder state for n_chunks windows of length L with P-bit tables. */

@@ -71,6 +71,7 @@ _sig("dlmz_forward_logits", c_int, _P, _P, c_uint32, c_uint32, c_uint32, c_uint3
 _sig("dlmz_gemm_bf16", c_int, _P, _P, _P, c_uint32, c_uint32, c_uint32, _P)
 _sig("dlmz_quantize", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P, _P, _P, _P, _P)
 _sig("dlmz_select_smallest", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
+_sig("dlmz_select_smallest_noalloc", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_coder_create", c_int, c_uint32, c_uint32, c_uint32, c_uint32, POINTER(c_void_p))
 _sig("dlmz_coder_destroy", None, _P)
 _sig("dlmz_coder_reset_encoder", c_int, _P, _P)
@@ -173,6 +174,12 @@ def quantize(d_logits, rows, V, P, d_cdf, d_W, d_A, d_Hq, d_top, stream=0):
 
 def select_smallest(d_keys, groups, group_size, k, d_out, stream=0):
     _ok(lib.dlmz_select_smallest(d_keys, groups, group_size, k, d_out, stream), "dlmz_select_smallest")
+
+
+def select_smallest_noalloc(d_keys, groups, group_size, k, d_out, stream=0):
+    """dlmz_select_smallest without any device allocation (static scratch, <= 65536 groups)."""
+    _ok(lib.dlmz_select_smallest_noalloc(d_keys, groups, group_size, k, d_out, stream),
+        "dlmz_select_smallest_noalloc")
 
 
 def profile_begin():
