@@ -187,7 +187,7 @@ def run(args):
         torch.cuda.set_device(0)
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2608_11249_gb300 import dlmz, sources
+    from paper_2608_11249_gb300 import dlmz, shard, sources
 
     dev = torch.device("cuda", torch.cuda.current_device())
     stream = torch.cuda.current_stream().cuda_stream
@@ -204,7 +204,7 @@ def run(args):
     pol = dlmz.policy(dlmz.TOPK_CONF, K, BLOCK)
 
     def step(i, check=False):
-        b = (i * ws + rank) % nb
+        b = shard.rank_batch(i, rank, ws, nb)
         src = d_in[b * per:(b + 1) * per]
         n = m.compress_device(src.data_ptr(), per, CHUNK, pol, d_c.data_ptr(), cap, BATCH, stream)
         k = m.decompress_device(d_c.data_ptr(), n, d_out.data_ptr(), per, stream)
@@ -240,10 +240,8 @@ def run(args):
     dlmz.profile_end(prof)
     clk = clocks.stop()
     step(0, check=True)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
     if ws > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    total_ms = float(t.item())
+        total_ms = shard.max_over_ranks(total_ms, device=dev)
     value = ws * per * args.steps / (total_ms / 1000.0)
 
     # end to end through the host-buffer C ABI (H2D/D2H inside the timed region)
@@ -252,7 +250,7 @@ def run(args):
     h2d = d2h = 0
     e2e_steps = max(1, min(args.steps, 3))
     for i in range(e2e_steps):
-        b = (i * ws + rank) % nb
+        b = shard.rank_batch(i, rank, ws, nb)
         chunk = host_in[b * per:(b + 1) * per].numpy().tobytes()
         torch.cuda.synchronize()
         t0 = time.perf_counter()

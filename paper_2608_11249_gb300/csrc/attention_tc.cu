@@ -1,0 +1,287 @@
+// Bidirectional attention on the 5th-generation tensor cores (Definition 3:
+// every position attends to every position of its window, no mask).
+//
+// CTA = (128 queries, head, window), 6 warps:
+//   warp 0      TMA: Q once; per key tile of 128: K (into a single buffer)
+//               and V^T (keys contiguous, written so by the QKV epilogue).
+//   warp 1      allocates 256 TMEM columns (S: 128, O: head_dim) and issues
+//               S_j = Q K_j^T and O += P_j V_j with tcgen05.mma from one thread.
+//   warps 2-5   softmax, one thread per query row (its TMEM lane): row max of
+//               S_j, P_j = 2^(S_j - m) written to shared memory as bf16 (the A
+//               operand of P V), running sum; the running max is raised (and O
+//               rescaled in TMEM) only when it grows by more than 8 (log2
+//               units), so P <= 2^8; finally O / l -> bf16.
+// GQA: query head h reads KV head h / (n_heads / n_kv_heads).  Requires the
+// window length to be a multiple of 128.  All waits are bounded.
+#include "kernels.cuh"
+#include "tcgen05.cuh"
+
+namespace dlmz {
+namespace fat {
+
+constexpr int BQ = 128, BK = 128;
+constexpr int THREADS = 192;
+constexpr int TMEM_COLS = 256;
+constexpr float RESCALE_THRESHOLD = 8.0f;
+
+template <int HD>
+struct Smem {
+  static constexpr int Q = 0;                        // HD/64 blocks of [128 x 64] bf16
+  static constexpr int K = Q + BQ * HD * 2;          // HD/64 blocks of [128 x 64]
+  static constexpr int VT = K + BK * HD * 2;         // 2 blocks of [HD x 64] (keys 0-63, 64-127)
+  static constexpr int P = VT + HD * BK * 2;         // 2 blocks of [128 x 64]
+  static constexpr int BARS = P + BQ * BK * 2;
+  static constexpr int TOTAL = BARS + 128 + 1024;    // + barriers + alignment slack
+};
+
+template <int HD>
+__global__ void __launch_bounds__(THREADS, 1)
+    fa_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt, int L, int nh,
+                 int nkv, int d, bf16* __restrict__ out, float scale_log2, int* err) {
+  using S = Smem<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+  const uint32_t base = smem_u32(sm);
+  const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT, sP = base + S::P;
+  const uint32_t bar = base + S::BARS;
+  const uint32_t q_full = bar, k_full = bar + 8, k_empty = bar + 16, v_full = bar + 24, v_empty = bar + 32,
+                 s_full = bar + 40, p_ready = bar + 48, o_done = bar + 56;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int w = blockIdx.z, h = blockIdx.y, q0 = blockIdx.x * BQ;
+  const int g = h / (nh / nkv);
+  const int nt = L / BK;
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(q_full, 1);
+    mbar_init(k_full, 1);
+    mbar_init(k_empty, 1);
+    mbar_init(v_full, 1);
+    mbar_init(v_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(p_ready, 4 * 32);
+    mbar_init(o_done, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) t5::tmem_alloc(smem_u32(&tmem_slot), TMEM_COLS);
+  t5::fence_before();
+  __syncthreads();
+  t5::fence_after();
+  const uint32_t tmem = tmem_slot;
+  const uint32_t tS = tmem, tO = tmem + BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const int row0 = w * L;
+      mbar_arrive_expect_tx(q_full, BQ * HD * 2);
+      for (int kb = 0; kb < HD / 64; ++kb) t5::tma_load_2d(sQ + kb * BQ * 128, &tmQK, h * HD + kb * 64, row0 + q0, q_full);
+      bool k_pend = false, v_pend = false;
+      uint32_t kp = 0, vp = 0;
+      for (int j = 0; j < nt && !abort_flag; ++j) {
+        if (!mbar_wait_bounded(k_empty, (j & 1) ^ 1, &abort_flag, err)) break;
+        mbar_arrive_expect_tx(k_full, BK * HD * 2);
+        for (int kb = 0; kb < HD / 64; ++kb)
+          t5::tma_load_2d(sK + kb * BK * 128, &tmQK, d + g * HD + kb * 64, row0 + j * BK, k_full);
+        k_pend = true;
+        kp = j & 1;
+        if (!mbar_wait_bounded(v_empty, (j & 1) ^ 1, &abort_flag, err)) break;
+        mbar_arrive_expect_tx(v_full, BK * HD * 2);
+        for (int kk = 0; kk < 2; ++kk)
+          t5::tma_load_2d(sVt + kk * HD * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HD, v_full);
+        v_pend = true;
+        vp = j & 1;
+      }
+      if (abort_flag) {  // let our own copies land before the CTA can exit
+        volatile int never = 0;
+        mbar_wait_bounded(q_full, 0, &never, err, 100000000ull);
+        if (k_pend) mbar_wait_bounded(k_full, kp, &never, err, 100000000ull);
+        if (v_pend) mbar_wait_bounded(v_full, vp, &never, err, 100000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
+      constexpr uint32_t ID_O = t5::idesc_bf16(BQ, HD);
+      bool issued = false;
+      auto issue_s = [&]() {
+        for (int kb = 0; kb < HD / 64; ++kb)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            t5::mma_bf16(tS, t5::sw128_desc(sQ + kb * BQ * 128 + 32 * k), t5::sw128_desc(sK + kb * BK * 128 + 32 * k),
+                         ID_S, (kb | k) != 0);
+        t5::commit(s_full);
+        t5::commit(k_empty);
+        issued = true;
+      };
+      bool ok = mbar_wait_bounded(q_full, 0, &abort_flag, err) && mbar_wait_bounded(k_full, 0, &abort_flag, err);
+      if (ok) {
+        t5::fence_after();
+        issue_s();
+      }
+      for (int j = 0; ok && j < nt; ++j) {
+        if (!mbar_wait_bounded(p_ready, j & 1, &abort_flag, err)) break;
+        t5::fence_after();
+        if (j + 1 < nt) {
+          if (!mbar_wait_bounded(k_full, (j + 1) & 1, &abort_flag, err)) break;
+          t5::fence_after();
+          issue_s();
+        }
+        if (!mbar_wait_bounded(v_full, j & 1, &abort_flag, err)) break;
+        t5::fence_after();
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            t5::mma_bf16(tO, t5::sw128_desc(sP + kk * BQ * 128 + 32 * k), t5::sw128_desc(sVt + kk * HD * 128 + 32 * k),
+                         ID_O, (j | kk | k) != 0);
+        t5::commit(v_empty);
+        t5::commit(o_done);
+      }
+      if (abort_flag && issued) {
+        volatile int never = 0;
+        const uint32_t drain = bar + 64;
+        mbar_init(drain, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        t5::commit(drain);
+        mbar_wait_bounded(drain, 0, &never, err, 100000000ull);
+      }
+    }
+  } else {
+    const int q = warp & 3;
+    const int r = q * 32 + lane;  // query row within the tile (= TMEM lane)
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nt; ++j) {
+      // waits are made warp-uniform: tcgen05.ld/st below are warp-collective
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(s_full, j & 1, &abort_flag, err))) {
+        ok = false;
+        break;
+      }
+      t5::fence_after();
+      float mx = -INFINITY;
+#pragma unroll 1
+      for (int c = 0; c < BK / 32; ++c) {
+        float v[32];
+        t5::tmem_ld32(tS + lane_off + c * 32, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) mx = fmaxf(mx, v[i]);
+      }
+      mx *= scale_log2;
+      if (j > 0) {  // PV_{j-1} done: P buffer free, O stable
+        if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (j - 1) & 1, &abort_flag, err))) {
+          ok = false;
+          break;
+        }
+        t5::fence_after();
+      }
+      if (j == 0) {
+        m = mx;
+      } else {
+        const bool need = mx > m + RESCALE_THRESHOLD;
+        float f = 1.0f;
+        if (need) {
+          f = t5::ex2(m - mx);
+          l *= f;
+          m = mx;
+        }
+        if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            float o[32];
+            t5::tmem_ld32(tO + lane_off + c * 32, o);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= f;
+            t5::tmem_st32(tO + lane_off + c * 32, o);
+          }
+        }
+      }
+      float sum = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < BK / 32; ++c) {
+        float v[32];
+        t5::tmem_ld32(tS + lane_off + c * 32, v);
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float a = t5::ex2(fmaf(v[2 * i], scale_log2, -m));
+          const float b = t5::ex2(fmaf(v[2 * i + 1], scale_log2, -m));
+          sum += a + b;
+          __nv_bfloat162 p2 = __floats2bfloat162_rn(a, b);
+          pk[i] = *reinterpret_cast<uint32_t*>(&p2);
+        }
+        const int kk = c >> 1;  // 64-key block
+        const uint32_t rowaddr = sP + kk * BQ * 128 + r * 128;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int cc = (c & 1) * 4 + t;  // 16-byte chunk of 8 keys within the 128-byte row
+          const uint32_t a = rowaddr + ((cc ^ (r & 7)) << 4);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(pk[4 * t]), "r"(pk[4 * t + 1]),
+                       "r"(pk[4 * t + 2]), "r"(pk[4 * t + 3])
+                       : "memory");
+        }
+      }
+      l += sum;
+      t5::fence_proxy_async();
+      t5::fence_before();
+      mbar_arrive(p_ready);
+    }
+    if (__all_sync(0xffffffffu, ok && mbar_wait_bounded(o_done, (nt - 1) & 1, &abort_flag, err))) {
+      t5::fence_after();
+      const float inv = 1.0f / l;
+      bf16* dst = out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        float o[32];
+        t5::tmem_ld32(tO + lane_off + c * 32, o);
+        uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          uint32_t u[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 p2 = __floats2bfloat162_rn(o[8 * t + 2 * e] * inv, o[8 * t + 2 * e + 1] * inv);
+            u[e] = *reinterpret_cast<uint32_t*>(&p2);
+          }
+          d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
+        }
+      }
+    }
+  }
+  t5::fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    t5::fence_after();
+    t5::tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+}  // namespace fat
+
+bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 && hd == 64; }
+
+int attention_bf16_tc(const bf16* qkv, int ld, const bf16* vt, int n_chunks, int L, int nh, int nkv, int hd, int d,
+                      bf16* out, cudaStream_t s) {
+  if (n_chunks == 0) return DLMZ_OK;
+  if (!attention_tc_supported(L, hd) || (ld % 8) || (reinterpret_cast<uintptr_t>(qkv) & 15) ||
+      (reinterpret_cast<uintptr_t>(vt) & 15))
+    return DLMZ_EINVAL;
+  CUtensorMap mqk, mvt;
+  DLMZ_TRY(t5::make_map_bf16(&mqk, qkv, (uint64_t)n_chunks * L, ld, ld, 128, 64));
+  DLMZ_TRY(t5::make_map_bf16(&mvt, vt, (uint64_t)n_chunks * nkv * hd, L, L, hd, 64));
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
+  constexpr int SM = fat::Smem<64>::TOTAL;
+  static bool attr = false;
+  if (!attr) {
+    DLMZ_CUDA_TRY(cudaFuncSetAttribute(fat::fa_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM));
+    attr = true;
+  }
+  dim3 grid(L / fat::BQ, nh, n_chunks);
+  ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
+  fat::fa_tc_kernel<64><<<grid, fat::THREADS, SM, s>>>(mqk, mvt, L, nh, nkv, d, out, scale_log2, device_error_word());
+  return launch_status();
+}
+
+}  // namespace dlmz

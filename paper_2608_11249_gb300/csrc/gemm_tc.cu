@@ -23,6 +23,7 @@
 // split-K), so results are independent of M and of the batch composition.
 #include "common.cuh"
 #include "kernels.cuh"
+#include "tcgen05.cuh"
 
 namespace dlmz {
 namespace tc {
@@ -34,9 +35,11 @@ constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int THREADS = 192;
+constexpr int BM_ALIGN_VT = 128;  // transposed V needs whole windows per 128-row tile
+constexpr int THREADS = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr int STG_BYTES = 8 * 32 * 128;  // epilogue staging, 8 warps x 32 x 32 float32
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256 + STG_BYTES;
 
 // Instruction descriptor (kind::f16): D f32, A/B bf16, both K-major, M=128, N=256.
 constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
@@ -99,87 +102,150 @@ __device__ __forceinline__ void fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v) {
-  uint4* d4 = reinterpret_cast<uint4*>(dst);
+// Epilogue staging: each epilogue warp owns a 32 x 32 float32 buffer; 16-byte
+// chunks are XOR-swizzled by row so both the row-per-thread writes and the
+// row-contiguous read-out are free of bank conflicts.
+__device__ __forceinline__ uint32_t stg_off(int row, int chunk) {
+  return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
+  __nv_bfloat162 p = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&p);
+}
+
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Global data an epilogue chunk needs besides the accumulator (residual
+// values or RoPE (cos, sin) pairs), loaded one chunk ahead to hide latency.
+struct EpiAux {
+  float4 x[8];
+};
+
+template <int EPI>
+__device__ __forceinline__ void epi_load_aux(EpiAux& a, int c, int lane, int row0, int M, int n0,
+                                             const GemmEpilogue& ep) {
+  if constexpr (EPI == EPI_RESID_F32) {
+    const int col0 = n0 + c * 32;
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    uint32_t w[4];
-#pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      __nv_bfloat162 p = __floats2bfloat162_rn(v[8 * j + 2 * t], v[8 * j + 2 * t + 1]);
-      w[t] = *reinterpret_cast<uint32_t*>(&p);
+    for (int it = 0; it < 8; ++it) {
+      const int r = it * 4 + (lane >> 3), m = row0 + r;
+      a.x[it] = m < M ? *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(ep.out) + (size_t)m * ep.ldo +
+                                                         col0 + (lane & 7) * 4)
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    d4[j] = make_uint4(w[0], w[1], w[2], w[3]);
+  } else if constexpr (EPI == EPI_ROPE_BF16) {
+    const int col = n0 + c * 32 + 8 * (lane & 3);
+    if (col < ep.rope_cols) {
+      const int half = ep.head_dim >> 1;
+      const int t0 = (col % ep.head_dim) >> 1;
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const int m = row0 + it * 8 + (lane >> 2);
+        const float4* cs = reinterpret_cast<const float4*>(ep.rope_cs + (size_t)((m < M ? m : 0) % ep.L) * half + t0);
+        a.x[2 * it] = cs[0];
+        a.x[2 * it + 1] = cs[1];
+      }
+    }
   }
 }
 
+// Drain one accumulator tile.  Epilogue warp e (0..7) reads TMEM lane quadrant
+// q = warp % 4 (tile rows [32q, 32q+32)) and the column half e / 4.  Per
+// 32-column chunk: tcgen05.ld (thread = row), optional SwiGLU, stage, then
+// row-contiguous global accesses (8 lanes x 16 B per float32 row segment, 4
+// lanes x 16 B per bf16 row segment) with the residual add, RoPE rotation or
+// bf16 conversion.
 template <int EPI>
-__device__ __forceinline__ void epilogue_tile(uint32_t tacc, int lane_base, int m, int M, int n0,
-                                              const GemmEpilogue& ep) {
-  const bool live = m < M;
-  if constexpr (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID_F32) {
+__device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, int lane, int m0, int M, int n0,
+                                              const GemmEpilogue& ep, uint8_t* stg) {
+  const uint32_t tbase = tacc + ((uint32_t)(q * 32) << 16);
+  const int row0 = m0 + q * 32;
+  constexpr int NCH = (EPI == EPI_SWIGLU_BF16 ? BN / 64 : BN / 32) / 2;  // chunks per column half
+  const int c0 = half * NCH;
+  EpiAux cur, nxt;
+  epi_load_aux<EPI>(cur, c0, lane, row0, M, n0, ep);
 #pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
-      float v[32];
-      tmem_ld32(tacc + ((uint32_t)lane_base << 16) + c * 32, v);
-      if (!live) continue;
-      const size_t off = (size_t)m * ep.ldo + n0 + c * 32;
-      if constexpr (EPI == EPI_BF16) {
-        store_bf16x32(reinterpret_cast<__nv_bfloat16*>(ep.out) + off, v);
-      } else if constexpr (EPI == EPI_F32) {
-        float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + off);
+  for (int c = c0; c < c0 + NCH; ++c) {
+    if (c + 1 < c0 + NCH) epi_load_aux<EPI>(nxt, c + 1, lane, row0, M, n0, ep);
+    float v[32];
+    tmem_ld32(tbase + c * 32, v);
+    if constexpr (EPI == EPI_SWIGLU_BF16) {  // columns [0,128) gate, [128,256) up of the same features
+      float u[32];
+      tmem_ld32(tbase + BN / 2 + c * 32, u);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) d[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-      } else {
-        float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + off);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          float4 r = d[j];
-          r.x += v[4 * j];
-          r.y += v[4 * j + 1];
-          r.z += v[4 * j + 2];
-          r.w += v[4 * j + 3];
-          d[j] = r;
-        }
+      for (int i = 0; i < 32; ++i) {
+        const float hg = 0.5f * v[i];
+        v[i] = fmaf(hg, tanh_approx(hg), hg) * u[i];  // silu(g) = g/2 (1 + tanh(g/2))
       }
     }
-  } else if constexpr (EPI == EPI_SWIGLU_BF16) {
-    // tile columns [0,128) = gate, [128,256) = up of the same 128 features
-#pragma unroll 1
-    for (int c = 0; c < BN / 64; ++c) {
-      float g[32], u[32];
-      tmem_ld32(tacc + ((uint32_t)lane_base << 16) + c * 32, g);
-      tmem_ld32(tacc + ((uint32_t)lane_base << 16) + BN / 2 + c * 32, u);
-      if (!live) continue;
 #pragma unroll
-      for (int i = 0; i < 32; ++i) g[i] = g[i] / (1.0f + __expf(-g[i])) * u[i];
-      const size_t off = (size_t)m * ep.ldo + (n0 / 2) + c * 32;
-      store_bf16x32(reinterpret_cast<__nv_bfloat16*>(ep.out) + off, g);
-    }
-  } else {  // EPI_ROPE*_BF16: rotate-half RoPE on columns < rope_cols, then bf16
-    constexpr int HD = EPI == EPI_ROPE32_BF16 ? 32 : (EPI == EPI_ROPE64_BF16 ? 64 : 128);
-    constexpr int HALF = HD / 2;
-    const int pos = live ? (m % ep.L) : 0;
-#pragma unroll 1
-    for (int h0 = 0; h0 < BN; h0 += HD) {
-      float v[HD];
+    for (int j = 0; j < 8; ++j)
+      *reinterpret_cast<float4*>(stg + stg_off(lane, j)) = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+    __syncwarp();
+    const int col0 = (EPI == EPI_SWIGLU_BF16 ? n0 / 2 : n0) + c * 32;
+    if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_F32) {
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) tmem_ld32(tacc + ((uint32_t)lane_base << 16) + h0 + c * 32, v + 32 * c);
-      if (!live) continue;
-      if (n0 + h0 < ep.rope_cols) {
-        const float2* cs = ep.rope_cs + (size_t)pos * HALF;
-#pragma unroll
-        for (int i = 0; i < HALF; ++i) {
-          float2 t = cs[i];
-          float a = v[i], b = v[i + HALF];
-          v[i] = a * t.x - b * t.y;
-          v[i + HALF] = b * t.x + a * t.y;
+      for (int it = 0; it < 8; ++it) {
+        const int r = it * 4 + (lane >> 3), ch = lane & 7;
+        const int m = row0 + r;
+        float4 val = *reinterpret_cast<const float4*>(stg + stg_off(r, ch));
+        if (m < M) {
+          if constexpr (EPI == EPI_RESID_F32) {
+            val.x += cur.x[it].x;
+            val.y += cur.x[it].y;
+            val.z += cur.x[it].z;
+            val.w += cur.x[it].w;
+          }
+          *reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)m * ep.ldo + col0 + ch * 4) = val;
         }
       }
-      __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)m * ep.ldo + n0 + h0;
+    } else if (EPI == EPI_ROPE_BF16 && ep.vt && col0 >= ep.v_col0) {
+      // V heads, transposed: vt[window][kv head][dim][pos]; 32 positions of a dim are contiguous
+      const int win = row0 / ep.L, pos0 = row0 % ep.L;
+      const int vi = col0 - ep.v_col0, gh = vi / ep.head_dim, dim0 = vi % ep.head_dim;
+      __nv_bfloat16* vb = ep.vt + ((size_t)(win * ep.n_kv + gh) * ep.head_dim + dim0) * ep.L + pos0;
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) store_bf16x32(dst + 32 * c, v + 32 * c);
+      for (int it = 0; it < 4; ++it) {
+        const int j = it * 8 + (lane >> 2), p0 = 8 * (lane & 3);
+        float w[8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) w[t] = *reinterpret_cast<const float*>(stg + stg_off(p0 + t, j >> 2) + (j & 3) * 4);
+        *reinterpret_cast<uint4*>(vb + (size_t)j * ep.L + p0) =
+            make_uint4(pack2_bf16(w[0], w[1]), pack2_bf16(w[2], w[3]), pack2_bf16(w[4], w[5]), pack2_bf16(w[6], w[7]));
+      }
+    } else {
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const int r = it * 8 + (lane >> 2), qd = lane & 3;
+        const int m = row0 + r;
+        const float4 a = *reinterpret_cast<const float4*>(stg + stg_off(r, 2 * qd));
+        const float4 b = *reinterpret_cast<const float4*>(stg + stg_off(r, 2 * qd + 1));
+        float w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        const int col = col0 + 8 * qd;
+        if constexpr (EPI == EPI_ROPE_BF16) {
+          if (col < ep.rope_cols) {  // head dims stored as rotation pairs (2t, 2t+1)
+            const float4 c01 = cur.x[2 * it], c23 = cur.x[2 * it + 1];
+            const float cr[4] = {c01.x, c01.z, c23.x, c23.z}, sr[4] = {c01.y, c01.w, c23.y, c23.w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const float x0 = w[2 * t], x1 = w[2 * t + 1];
+              w[2 * t] = x0 * cr[t] - x1 * sr[t];
+              w[2 * t + 1] = x1 * cr[t] + x0 * sr[t];
+            }
+          }
+        }
+        if (m < M)
+          *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)m * ep.ldo + col) =
+              make_uint4(pack2_bf16(w[0], w[1]), pack2_bf16(w[2], w[3]), pack2_bf16(w[4], w[5]), pack2_bf16(w[6], w[7]));
+      }
     }
+    __syncwarp();
+    cur = nxt;
   }
 }
 
@@ -192,6 +258,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * A_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint8_t* stg_all = smem + STAGES * STAGE_BYTES + 256;
   // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2], drain
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
@@ -212,7 +279,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
-      mbar_init(tempty0 + 8 * a, 4 * 32);
+      mbar_init(tempty0 + 8 * a, 8 * 32);
     }
     mbar_init(drain, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -308,15 +375,17 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   } else {
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
-    const int lane_base = q * 32;
+    const int half = (warp - 2) >> 2;
+    uint8_t* stg = stg_all + (warp - 2) * 32 * 128;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
-      if (!mbar_wait_bounded(tfull0 + 8 * acc, acc_phase, &abort_flag, err)) break;
+      // warp-uniform outcome: the epilogue's tcgen05.ld is warp-collective
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(tfull0 + 8 * acc, acc_phase, &abort_flag, err))) break;
       fence_after();
       const int m0 = (tile / n_tiles) * BM;
       const int n0 = (tile % n_tiles) * BN;
-      epilogue_tile<EPI>(tmem + acc * BN, lane_base, m0 + lane_base + lane, M, n0, ep);
+      epilogue_tile<EPI>(tmem + acc * BN, q, half, lane, m0, M, n0, ep, stg);
       fence_before();
       mbar_arrive(tempty0 + 8 * acc);
       if (++acc == 2) {
@@ -352,15 +421,15 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D bf16 tensor [rows x cols] row-major (ld elements per row), box
-// [box_rows x 64], 128-byte swizzle, out-of-range rows read as zero.
-static int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
-                    uint32_t box_rows) {
-  EncodeTiledFn fn = encode_fn();
+}  // namespace tc
+
+int t5::make_map_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                      uint32_t box_rows, uint32_t box_cols) {
+  tc::EncodeTiledFn fn = tc::encode_fn();
   if (!fn) return DLMZ_ECUDA;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {ld * 2};
-  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -371,6 +440,8 @@ static int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
   }
   return DLMZ_OK;
 }
+
+namespace tc {
 
 template <int EPI>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const GemmEpilogue& ep,
@@ -399,18 +470,18 @@ int gemm_bf16_tc(const __nv_bfloat16* A, int lda, const __nv_bfloat16* B, int ld
   if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) return DLMZ_EINVAL;
   if ((lda | ldb) & 7) return DLMZ_EINVAL;
   CUtensorMap ma, mb;
-  DLMZ_TRY(tc::make_map(&ma, A, M, K, lda, tc::BM));
-  DLMZ_TRY(tc::make_map(&mb, B, N, K, ldb, tc::BN));
+  DLMZ_TRY(t5::make_map_bf16(&ma, A, M, K, lda, tc::BM, tc::BK));
+  DLMZ_TRY(t5::make_map_bf16(&mb, B, N, K, ldb, tc::BN, tc::BK));
   switch (epi) {
     case EPI_BF16: return tc::launch<EPI_BF16>(ma, mb, M, N, K, ep, s);
     case EPI_F32: return tc::launch<EPI_F32>(ma, mb, M, N, K, ep, s);
     case EPI_RESID_F32: return tc::launch<EPI_RESID_F32>(ma, mb, M, N, K, ep, s);
     case EPI_SWIGLU_BF16: return tc::launch<EPI_SWIGLU_BF16>(ma, mb, M, N, K, ep, s);
     case EPI_ROPE_BF16:
-      if (ep.head_dim == 32) return tc::launch<EPI_ROPE32_BF16>(ma, mb, M, N, K, ep, s);
-      if (ep.head_dim == 64) return tc::launch<EPI_ROPE64_BF16>(ma, mb, M, N, K, ep, s);
-      if (ep.head_dim == 128) return tc::launch<EPI_ROPE128_BF16>(ma, mb, M, N, K, ep, s);
-      return DLMZ_EINVAL;
+      if (ep.head_dim % 8 || !ep.rope_cs || (reinterpret_cast<uintptr_t>(ep.rope_cs) & 15)) return DLMZ_EINVAL;
+      if (ep.vt && (ep.L % tc::BM_ALIGN_VT || M % ep.L || ep.v_col0 % 32 || (reinterpret_cast<uintptr_t>(ep.vt) & 15)))
+        return DLMZ_EINVAL;
+      return tc::launch<EPI_ROPE_BF16>(ma, mb, M, N, K, ep, s);
   }
   return DLMZ_EINVAL;
 }

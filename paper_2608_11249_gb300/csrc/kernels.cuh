@@ -13,11 +13,8 @@ enum {
   EPI_F32 = 1,         // out = acc (float32)
   EPI_RESID_F32 = 2,   // out += acc (float32 residual stream, in place)
   EPI_SWIGLU_BF16 = 3, // out[:, f] = bf16(silu(g_f) * u_f), gate/up interleaved in blocks
-  EPI_ROPE_BF16 = 4,   // out = bf16(RoPE(acc)) on columns < rope_cols, bf16(acc) beyond
-  // internal instantiations of EPI_ROPE_BF16 per head dimension
-  EPI_ROPE32_BF16 = 5,
-  EPI_ROPE64_BF16 = 6,
-  EPI_ROPE128_BF16 = 7,
+  EPI_ROPE_BF16 = 4,   // out = bf16(RoPE(acc)) on columns < rope_cols, bf16(acc) beyond; the
+                       // head dimensions are stored as rotation pairs (2t, 2t+1)
 };
 
 struct GemmEpilogue {
@@ -28,6 +25,9 @@ struct GemmEpilogue {
   int head_dim;
   int rope_cols;         // columns [0, rope_cols) get RoPE (Q and K heads)
   int gu_block;          // SwiGLU: gate/up interleave block (columns)
+  bf16* vt;              // RoPE epilogue: if set, columns >= v_col0 (the V heads) go to
+  int v_col0;            //   vt [window][kv head][dim][L] (keys contiguous) instead of `out`
+  int n_kv;
 };
 
 // tcgen05 path: N % 256 == 0, K % 64 == 0, 16-byte aligned operands.
@@ -55,6 +55,9 @@ int swiglu(const float* gu, int T_tokens, int F, int gu_block, T* out, cudaStrea
 template <typename T>
 int attention_simt(const T* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                    int head_dim, int d, T* out, cudaStream_t s);
+bool attention_tc_supported(int L, int hd);
+int attention_bf16_tc(const bf16* qkv, int ld, const bf16* vt, int n_chunks, int L, int n_heads, int n_kv_heads,
+                      int head_dim, int d, bf16* out, cudaStream_t s);
 int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                        int head_dim, int d, bf16* out, cudaStream_t s);
 

@@ -8,6 +8,10 @@
 // row-major in its logical shape.  Physical layouts: Wq|Wk|Wv stacked into
 // one [d+2 dkv x d] matrix; Wgate/Wup interleaved in blocks of gu_block rows
 // so a 256-column GEMM tile holds the gate and up rows of the same features.
+// On the tensor-core path the rows of Wq and Wk are also reordered inside each
+// head so that RoPE's rotation pairs (i, i + hd/2) become adjacent columns
+// (2i, 2i+1) of the QKV output; q.k over a head is unchanged by a permutation
+// of its dimensions applied to both q and k, and V keeps its order.
 #include <math.h>
 #include <string.h>
 
@@ -44,7 +48,7 @@ __device__ __forceinline__ __nv_bfloat16 conv_weight<__nv_bfloat16>(double x) { 
 // Element n of tensor with stream state st: pairs (2j, 2j+1) from outputs 2j, 2j+1.
 template <typename T>
 __global__ void init_kernel(T* __restrict__ dst, int64_t rows, int64_t cols, uint64_t st, int64_t grp,
-                            int64_t grp_stride, int64_t grp_off) {
+                            int64_t grp_stride, int64_t grp_off, int64_t pair_hd) {
   const int64_t n = rows * cols;
   const int64_t npairs = (n + 1) / 2;
   for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < npairs; j += (int64_t)gridDim.x * blockDim.x) {
@@ -59,7 +63,12 @@ __global__ void init_kernel(T* __restrict__ dst, int64_t rows, int64_t cols, uin
     for (int e = 0; e < 2; ++e) {
       const int64_t idx = 2 * j + e;
       if (idx >= n) break;
-      const int64_t rr = idx / cols, cc = idx % cols;
+      int64_t rr = idx / cols;
+      const int64_t cc = idx % cols;
+      if (pair_hd) {  // head row i -> 2i (i < hd/2) or 2(i - hd/2) + 1
+        const int64_t h = rr / pair_hd, i = rr % pair_hd, half = pair_hd / 2;
+        rr = h * pair_hd + (i < half ? 2 * i : 2 * (i - half) + 1);
+      }
       const int64_t drow = (rr / grp) * grp_stride + grp_off + rr % grp;
       dst[drow * cols + cc] = conv_weight<T>(0.02 * z[e]);
     }
@@ -74,13 +83,13 @@ static uint64_t tensor_state(uint64_t seed, uint64_t tid) { return mix64(seed + 
 
 template <typename T>
 static int init_tensor(void* dst, int64_t rows, int64_t cols, uint64_t seed, uint64_t tid, int64_t grp,
-                       int64_t grp_stride, int64_t grp_off) {
+                       int64_t grp_stride, int64_t grp_off, int64_t pair_hd) {
   const int64_t npairs = (rows * cols + 1) / 2;
   int64_t blocks = (npairs + 255) / 256;
   if (blocks > 65536) blocks = 65536;
   if (blocks < 1) blocks = 1;
   init_kernel<T><<<(unsigned)blocks, 256>>>(reinterpret_cast<T*>(dst), rows, cols, tensor_state(seed, tid),
-                                            grp > 0 ? grp : rows, grp > 0 ? grp_stride : 0, grp_off);
+                                            grp > 0 ? grp : rows, grp > 0 ? grp_stride : 0, grp_off, pair_hd);
   return launch_status();
 }
 
@@ -110,7 +119,7 @@ static uint64_t config_fingerprint(const dlmz_model_config& c) {
 
 size_t model_workspace_per_token(const dlmz_model* m) {
   const size_t d = m->cfg.d, F = m->cfg.ffn;
-  size_t b = 4 * d + m->esz * (2 * d + m->nqkv + F);
+  size_t b = 4 * d + m->esz * (2 * d + m->nqkv + F + m->dkv);
   if (!m->tc) b += 4 * 2 * F;  // float32 gate/up buffer of the CUDA-core path
   return b;
 }
@@ -138,6 +147,9 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
   DLMZ_TRY(w.act.ensure((size_t)Tt * F * sizeof(T)));
   if (!m->tc) DLMZ_TRY(w.gu.ensure((size_t)Tt * 2 * F * 4));
   DLMZ_TRY(w.hc.ensure((size_t)R * d * sizeof(T)));
+  // tensor-core attention reads V transposed (keys contiguous), written by the QKV epilogue
+  const bool tc_attn = m->tc && attention_tc_supported(L, hd);
+  if (tc_attn) DLMZ_TRY(w.vt.ensure((size_t)Tt * m->dkv * sizeof(T)));
   if (w.rope_L < L) {  // (cos, sin) of pos * theta^(-2i/hd), from double precision
     const int half = hd / 2;
     std::vector<float2> cs((size_t)L * half);
@@ -160,7 +172,11 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
   DLMZ_TRY(embed<T>(state, Tt, reinterpret_cast<const T*>(m->E), d, x, s));
   for (uint32_t l = 0; l < c.n_layers; ++l) {
     DLMZ_TRY(rmsnorm<T>(x, Tt, d, m->gains, c.norm_eps, h, L, 0, 0, s));
-    ep = GemmEpilogue{qkv, nq, cs, L, hd, d + m->dkv, m->gu_block};
+    ep = GemmEpilogue{qkv, nq, cs, L, hd, d + m->dkv, m->gu_block, nullptr, 0, (int)c.n_kv_heads};
+    if (tc_attn) {
+      ep.vt = w.vt.as<bf16>();
+      ep.v_col0 = d + m->dkv;
+    }
     if (m->tc) {
       DLMZ_TRY(gemm_bf16_tc(reinterpret_cast<const bf16*>(h), d, reinterpret_cast<const bf16*>(m->wqkv[l]), d, Tt,
                             nq, d, EPI_ROPE_BF16, ep, s));
@@ -170,31 +186,33 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
       DLMZ_TRY(rope_inplace<T>(qkv, Tt, nq, c.n_heads + c.n_kv_heads, hd, L, cs, s));
     }
     if constexpr (sizeof(T) == 2) {
-      if (hd == 64 || hd == 128)
+      if (tc_attn)
+        DLMZ_TRY(attention_bf16_tc(qkv, nq, w.vt.as<bf16>(), nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
+      else if (hd == 64 || hd == 128)
         DLMZ_TRY(attention_bf16_mma(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
       else
         DLMZ_TRY(attention_simt<T>(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
     } else {
       DLMZ_TRY(attention_simt<T>(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
     }
-    ep = GemmEpilogue{x, d, nullptr, L, hd, 0, m->gu_block};
+    ep = GemmEpilogue{x, d, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
     DLMZ_TRY(gemm<T>(attn, reinterpret_cast<const T*>(m->wo[l]), Tt, d, d, EPI_RESID_F32, ep, s));
     DLMZ_TRY(rmsnorm<T>(x, Tt, d, m->gains, c.norm_eps, h, L, 0, 0, s));
     if (m->tc) {
-      ep = GemmEpilogue{act, F, nullptr, L, hd, 0, m->gu_block};
+      ep = GemmEpilogue{act, F, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
       DLMZ_TRY(gemm_bf16_tc(reinterpret_cast<const bf16*>(h), d, reinterpret_cast<const bf16*>(m->wgu[l]), d, Tt,
                             2 * F, d, EPI_SWIGLU_BF16, ep, s));
     } else {
-      ep = GemmEpilogue{w.gu.p, 2 * F, nullptr, L, hd, 0, m->gu_block};
+      ep = GemmEpilogue{w.gu.p, 2 * F, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
       DLMZ_TRY(gemm<T>(h, reinterpret_cast<const T*>(m->wgu[l]), Tt, 2 * F, d, EPI_F32, ep, s));
       DLMZ_TRY(swiglu<T>(w.gu.as<float>(), Tt, F, m->gu_block, act, s));
     }
-    ep = GemmEpilogue{x, d, nullptr, L, hd, 0, m->gu_block};
+    ep = GemmEpilogue{x, d, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
     DLMZ_TRY(gemm<T>(act, reinterpret_cast<const T*>(m->wdown[l]), Tt, d, F, EPI_RESID_F32, ep, s));
   }
   T* hc = w.hc.as<T>();
   DLMZ_TRY(rmsnorm<T>(x, R, d, m->gains, c.norm_eps, hc, L, row0, rpc, s));
-  ep = GemmEpilogue{logits, V, nullptr, L, hd, 0, m->gu_block};
+  ep = GemmEpilogue{logits, V, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
   return gemm<T>(hc, reinterpret_cast<const T*>(m->head), R, V, d, EPI_F32, ep, s);
 }
 
@@ -280,18 +298,20 @@ extern "C" int dlmz_model_create(const dlmz_model_config* cfg, dlmz_model** out)
   const int64_t gb = m->gu_block;
   const size_t es = m->esz;
   int rc = DLMZ_OK;
-  auto init = [&](void* dst, int64_t rows, int64_t cols, uint64_t tid, int64_t grp, int64_t gs, int64_t go) {
+  auto init = [&](void* dst, int64_t rows, int64_t cols, uint64_t tid, int64_t grp, int64_t gs, int64_t go,
+                  int64_t pair_hd = 0) {
     if (rc != DLMZ_OK) return;
-    rc = m->bf16 ? init_tensor<bf16>(dst, rows, cols, seed, tid, grp, gs, go)
-                 : init_tensor<float>(dst, rows, cols, seed, tid, grp, gs, go);
+    rc = m->bf16 ? init_tensor<bf16>(dst, rows, cols, seed, tid, grp, gs, go, pair_hd)
+                 : init_tensor<float>(dst, rows, cols, seed, tid, grp, gs, go, pair_hd);
   };
+  const int64_t pair_hd = m->tc ? hd : 0;
   init(m->E, V + 1, d, 0, 0, 0, 0);
   init(m->head, V, d, 1, 0, 0, 0);
   for (size_t l = 0; l < nl; ++l) {
     const uint64_t t0 = 2 + 8 * l;
     uint8_t* q = reinterpret_cast<uint8_t*>(m->wqkv[l]);
-    init(q, d, d, t0 + 0, 0, 0, 0);
-    init(q + d * d * es, m->dkv, d, t0 + 1, 0, 0, 0);
+    init(q, d, d, t0 + 0, 0, 0, 0, pair_hd);
+    init(q + d * d * es, m->dkv, d, t0 + 1, 0, 0, 0, pair_hd);
     init(q + (d + m->dkv) * d * es, m->dkv, d, t0 + 2, 0, 0, 0);
     init(m->wo[l], d, d, t0 + 3, 0, 0, 0);
     init(m->wgu[l], F, d, t0 + 4, gb, 2 * gb, 0);
@@ -324,6 +344,7 @@ extern "C" void dlmz_model_destroy(dlmz_model* m) {
   m->ws.gu.release();
   m->ws.hc.release();
   m->ws.rope.release();
+  m->ws.vt.release();
   pipeline_release(m);
   delete m;
 }

@@ -34,7 +34,7 @@ struct DevBuf {
 };
 
 struct ForwardWorkspace {
-  DevBuf x, h, qkv, attn, act, gu, hc, rope;
+  DevBuf x, h, qkv, attn, act, gu, hc, rope, vt;
   int rope_L = 0;
 };
 

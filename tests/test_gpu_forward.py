@@ -19,6 +19,8 @@ MODELS = [
     (2, 256, 4, 4, 256, 256, "bf16", 192, 3, 0, 192),    # tcgen05 GEMMs (RoPE/SwiGLU/residual epilogues), mma attention hd 64
     (2, 512, 4, 2, 512, 512, "bf16", 130, 2, 2, 128),    # tcgen05 + GQA, hd 128, ragged window (130)
     (1, 256, 8, 1, 384, 300, "bf16", 77, 2, 0, 77),      # 8:1 GQA hd 32, LM head on CUDA cores (V = 300)
+    (2, 256, 4, 2, 256, 256, "bf16", 256, 2, 0, 256),    # tcgen05 attention (L % 128 == 0, hd 64), GQA 2:1
+    (2, 512, 8, 8, 512, 256, "bf16", 512, 2, 128, 128),  # byte-workload head shape: L 512, hd 64, block rows
 ]
 
 
