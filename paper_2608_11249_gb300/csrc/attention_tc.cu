@@ -6,11 +6,15 @@
 //               and V^T (keys contiguous, written so by the QKV epilogue).
 //   warp 1      allocates 256 TMEM columns (S: 128, O: head_dim) and issues
 //               S_j = Q K_j^T and O += P_j V_j with tcgen05.mma from one thread.
-//   warps 2-5   softmax, one thread per query row (its TMEM lane): row max of
-//               S_j, P_j = 2^(S_j - m) written to shared memory as bf16 (the A
-//               operand of P V), running sum; the running max is raised (and O
-//               rescaled in TMEM) only when it grows by more than 8 (log2
-//               units), so P <= 2^8; finally O / l -> bf16.
+//   warps 2-5   softmax, one thread per query row (its TMEM lane): the row of
+//               S_j in one 128-column TMEM load, its max, P_j = 2^(S_j - m) by
+//               ex2.approx.f16x2 written to shared memory as f16 (the A operand
+//               of P V); the running max is raised (and O rescaled in TMEM)
+//               only when it grows by more than 8 (log2 units), so P <= 2^8;
+//               finally O / l -> bf16.
+// V^T (f16) carries an extra row of ones after the head dimensions (and 15
+// zero rows), so O's column head_dim accumulates the row sum l of P on the
+// tensor core, rescaled together with O.
 // GQA: query head h reads KV head h / (n_heads / n_kv_heads).  Requires the
 // window length to be a multiple of 128.  All waits are bounded.
 #include "kernels.cuh"
@@ -23,13 +27,15 @@ constexpr int BQ = 128, BK = 128;
 constexpr int THREADS = 192;
 constexpr int TMEM_COLS = 256;
 constexpr float RESCALE_THRESHOLD = 8.0f;
+constexpr int VT_EXTRA = 16;  // ones row + zero rows appended to V^T
 
 template <int HD>
 struct Smem {
+  static constexpr int HDP = HD + VT_EXTRA;
   static constexpr int Q = 0;                        // HD/64 blocks of [128 x 64] bf16
   static constexpr int K = Q + BQ * HD * 2;          // HD/64 blocks of [128 x 64]
-  static constexpr int VT = K + BK * HD * 2;         // 2 blocks of [HD x 64] (keys 0-63, 64-127)
-  static constexpr int P = VT + HD * BK * 2;         // 2 blocks of [128 x 64]
+  static constexpr int VT = K + BK * HD * 2;         // 2 blocks of [HDP x 64] f16 (keys 0-63, 64-127)
+  static constexpr int P = VT + HDP * BK * 2;        // 2 blocks of [128 x 64] f16
   static constexpr int BARS = P + BQ * BK * 2;
   static constexpr int TOTAL = BARS + 128 + 1024;    // + barriers + alignment slack
 };
@@ -71,6 +77,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   t5::fence_after();
   const uint32_t tmem = tmem_slot;
   const uint32_t tS = tmem, tO = tmem + BK;
+  constexpr int HDP = S::HDP;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -87,9 +94,9 @@ __global__ void __launch_bounds__(THREADS, 1)
         k_pend = true;
         kp = j & 1;
         if (!mbar_wait_bounded(v_empty, (j & 1) ^ 1, &abort_flag, err)) break;
-        mbar_arrive_expect_tx(v_full, BK * HD * 2);
+        mbar_arrive_expect_tx(v_full, BK * HDP * 2);
         for (int kk = 0; kk < 2; ++kk)
-          t5::tma_load_2d(sVt + kk * HD * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HD, v_full);
+          t5::tma_load_2d(sVt + kk * HDP * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HDP, v_full);
         v_pend = true;
         vp = j & 1;
       }
@@ -103,7 +110,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
-      constexpr uint32_t ID_O = t5::idesc_bf16(BQ, HD);
+      constexpr uint32_t ID_O = t5::idesc_f16(BQ, HDP);
       bool issued = false;
       auto issue_s = [&]() {
         for (int kb = 0; kb < HD / 64; ++kb)
@@ -134,7 +141,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int kk = 0; kk < 2; ++kk)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            t5::mma_bf16(tO, t5::sw128_desc(sP + kk * BQ * 128 + 32 * k), t5::sw128_desc(sVt + kk * HD * 128 + 32 * k),
+            t5::mma_bf16(tO, t5::sw128_desc(sP + kk * BQ * 128 + 32 * k), t5::sw128_desc(sVt + kk * HDP * 128 + 32 * k),
                          ID_O, (j | kk | k) != 0);
         t5::commit(v_empty);
         t5::commit(o_done);
@@ -152,7 +159,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;
     const int r = q * 32 + lane;  // query row within the tile (= TMEM lane)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    float m = -INFINITY, l = 0.f;
+    float m = -INFINITY;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
       // waits are made warp-uniform: tcgen05.ld/st below are warp-collective
@@ -161,14 +168,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       t5::fence_after();
+      uint32_t sr[BK];
+      t5::tmem_ld128(tS + lane_off, sr);
       float mx = -INFINITY;
-#pragma unroll 1
-      for (int c = 0; c < BK / 32; ++c) {
-        float v[32];
-        t5::tmem_ld32(tS + lane_off + c * 32, v);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) mx = fmaxf(mx, v[i]);
-      }
+      for (int i = 0; i < BK; ++i) mx = fmaxf(mx, __uint_as_float(sr[i]));
       mx *= scale_log2;
       if (j > 0) {  // PV_{j-1} done: P buffer free, O stable
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (j - 1) & 1, &abort_flag, err))) {
@@ -184,69 +188,56 @@ __global__ void __launch_bounds__(THREADS, 1)
         float f = 1.0f;
         if (need) {
           f = t5::ex2(m - mx);
-          l *= f;
           m = mx;
         }
         if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
 #pragma unroll 1
-          for (int c = 0; c < HD / 32; ++c) {
-            float o[32];
-            t5::tmem_ld32(tO + lane_off + c * 32, o);
+          for (int c = 0; c < HDP / 16; ++c) {
+            uint32_t o[16];
+            t5::tmem_ld16(tO + lane_off + c * 16, o);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] *= f;
-            t5::tmem_st32(tO + lane_off + c * 32, o);
+            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+            t5::tmem_st16(tO + lane_off + c * 16, o);
           }
         }
       }
-      float sum = 0.f;
-#pragma unroll 1
-      for (int c = 0; c < BK / 32; ++c) {
-        float v[32];
-        t5::tmem_ld32(tS + lane_off + c * 32, v);
-        uint32_t pk[16];
+      // P = 2^(s * scale - m) as f16 pairs, 16-byte chunks of 8 keys, 128B-swizzled rows
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float a = t5::ex2(fmaf(v[2 * i], scale_log2, -m));
-          const float b = t5::ex2(fmaf(v[2 * i + 1], scale_log2, -m));
-          sum += a + b;
-          __nv_bfloat162 p2 = __floats2bfloat162_rn(a, b);
-          pk[i] = *reinterpret_cast<uint32_t*>(&p2);
-        }
-        const int kk = c >> 1;  // 64-key block
-        const uint32_t rowaddr = sP + kk * BQ * 128 + r * 128;
+      for (int cc = 0; cc < BK / 8; ++cc) {
+        uint32_t pk[4];
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
-          const int cc = (c & 1) * 4 + t;  // 16-byte chunk of 8 keys within the 128-byte row
-          const uint32_t a = rowaddr + ((cc ^ (r & 7)) << 4);
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(pk[4 * t]), "r"(pk[4 * t + 1]),
-                       "r"(pk[4 * t + 2]), "r"(pk[4 * t + 3])
-                       : "memory");
+          const int i = cc * 8 + 2 * t;
+          pk[t] = t5::ex2_f16x2(t5::pack_f16x2(fmaf(__uint_as_float(sr[i]), scale_log2, -m),
+                                               fmaf(__uint_as_float(sr[i + 1]), scale_log2, -m)));
         }
+        const uint32_t a = sP + (cc >> 3) * BQ * 128 + r * 128 + (((cc & 7) ^ (r & 7)) << 4);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(pk[0]), "r"(pk[1]), "r"(pk[2]),
+                     "r"(pk[3])
+                     : "memory");
       }
-      l += sum;
       t5::fence_proxy_async();
       t5::fence_before();
       mbar_arrive(p_ready);
     }
     if (__all_sync(0xffffffffu, ok && mbar_wait_bounded(o_done, (nt - 1) & 1, &abort_flag, err))) {
       t5::fence_after();
-      const float inv = 1.0f / l;
+      uint32_t o[HD], lsum[16];
+      t5::tmem_ld64(tO + lane_off, o);
+      t5::tmem_ld16(tO + lane_off + HD, lsum);
+      const float inv = 1.0f / __uint_as_float(lsum[0]);
       bf16* dst = out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
-#pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
-        float o[32];
-        t5::tmem_ld32(tO + lane_off + c * 32, o);
-        uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-        for (int t = 0; t < 4; ++t) {
-          uint32_t u[4];
+      for (int t = 0; t < HD / 8; ++t) {
+        uint32_t u[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 p2 = __floats2bfloat162_rn(o[8 * t + 2 * e] * inv, o[8 * t + 2 * e + 1] * inv);
-            u[e] = *reinterpret_cast<uint32_t*>(&p2);
-          }
-          d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
+        for (int e = 0; e < 4; ++e) {
+          __nv_bfloat162 p2 = __floats2bfloat162_rn(__uint_as_float(o[8 * t + 2 * e]) * inv,
+                                                    __uint_as_float(o[8 * t + 2 * e + 1]) * inv);
+          u[e] = *reinterpret_cast<uint32_t*>(&p2);
         }
+        d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
       }
     }
   }
@@ -262,7 +253,28 @@ __global__ void __launch_bounds__(THREADS, 1)
 
 bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 && hd == 64; }
 
-int attention_bf16_tc(const bf16* qkv, int ld, const bf16* vt, int n_chunks, int L, int nh, int nkv, int hd, int d,
+int attention_vt_rows(int hd) { return hd + fat::VT_EXTRA; }
+
+__global__ void vt_init_kernel(__half* vt, int blocks, int hd, int L) {
+  const int rows = hd + fat::VT_EXTRA;
+  const int64_t n = (int64_t)blocks * fat::VT_EXTRA * L;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t b = i / ((int64_t)fat::VT_EXTRA * L), rem = i % ((int64_t)fat::VT_EXTRA * L);
+    const int e = (int)(rem / L), p = (int)(rem % L);
+    vt[(b * rows + hd + e) * L + p] = __float2half(e == 0 ? 1.0f : 0.0f);
+  }
+}
+
+int attention_vt_init(void* vt, int blocks, int hd, int L, cudaStream_t s) {
+  const int64_t n = (int64_t)blocks * fat::VT_EXTRA * L;
+  if (n == 0) return DLMZ_OK;
+  int64_t g = (n + 255) / 256;
+  if (g > 65535) g = 65535;
+  vt_init_kernel<<<(unsigned)g, 256, 0, s>>>(reinterpret_cast<__half*>(vt), blocks, hd, L);
+  return launch_status();
+}
+
+int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int L, int nh, int nkv, int hd, int d,
                       bf16* out, cudaStream_t s) {
   if (n_chunks == 0) return DLMZ_OK;
   if (!attention_tc_supported(L, hd) || (ld % 8) || (reinterpret_cast<uintptr_t>(qkv) & 15) ||
@@ -270,7 +282,7 @@ int attention_bf16_tc(const bf16* qkv, int ld, const bf16* vt, int n_chunks, int
     return DLMZ_EINVAL;
   CUtensorMap mqk, mvt;
   DLMZ_TRY(t5::make_map_bf16(&mqk, qkv, (uint64_t)n_chunks * L, ld, ld, 128, 64));
-  DLMZ_TRY(t5::make_map_bf16(&mvt, vt, (uint64_t)n_chunks * nkv * hd, L, L, hd, 64));
+  DLMZ_TRY(t5::make_map_f16(&mvt, vt, (uint64_t)n_chunks * nkv * (hd + fat::VT_EXTRA), L, L, hd + fat::VT_EXTRA, 64));
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
   constexpr int SM = fat::Smem<64>::TOTAL;
   static bool attr = false;

@@ -109,6 +109,11 @@ __device__ __forceinline__ uint32_t stg_off(int row, int chunk) {
   return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
+__device__ __forceinline__ uint32_t pack2_f16(float a, float b) {
+  __half2 p = __floats2half2_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&p);
+}
+
 __device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
   __nv_bfloat162 p = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&p);
@@ -138,7 +143,7 @@ __device__ __forceinline__ void epi_load_aux(EpiAux& a, int c, int lane, int row
                                                          col0 + (lane & 7) * 4)
                       : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-  } else if constexpr (EPI == EPI_ROPE_BF16) {
+  } else if constexpr (EPI == EPI_ROPE_BF16) {  // small, L1-resident table: loaded for the current chunk
     const int col = n0 + c * 32 + 8 * (lane & 3);
     if (col < ep.rope_cols) {
       const int half = ep.head_dim >> 1;
@@ -160,18 +165,38 @@ __device__ __forceinline__ void epi_load_aux(EpiAux& a, int c, int lane, int row
 // row-contiguous global accesses (8 lanes x 16 B per float32 row segment, 4
 // lanes x 16 B per bf16 row segment) with the residual add, RoPE rotation or
 // bf16 conversion.
+// Fused RMSNorm, consumer side: sum of the row's partial sums of x^2 (the
+// caller loads it one tile ahead so the loads overlap the previous tile).
+__device__ __forceinline__ float row_ssq(const GemmEpilogue& ep, int m, int M) {
+  float ss = 0.f;
+  if (ep.ssq_in && m < M)
+    for (int i = 0; i < ep.n_part; ++i) ss += ep.ssq_in[(size_t)m * ep.n_part + i];
+  return ss;
+}
+
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, int lane, int m0, int M, int n0,
-                                              const GemmEpilogue& ep, uint8_t* stg) {
+                                              const GemmEpilogue& ep, uint8_t* stg, float row_ss) {
   const uint32_t tbase = tacc + ((uint32_t)(q * 32) << 16);
   const int row0 = m0 + q * 32;
   constexpr int NCH = (EPI == EPI_SWIGLU_BF16 ? BN / 64 : BN / 32) / 2;  // chunks per column half
   const int c0 = half * NCH;
+  // fused RMSNorm, consumer side: this thread's accumulator row is scaled by rsqrt(mean x^2 + eps)
+  float rs = 1.0f;
+  if constexpr (EPI == EPI_ROPE_BF16 || EPI == EPI_SWIGLU_BF16) {
+    if (ep.ssq_in) rs = rsqrtf(row_ss / (float)ep.d_model + ep.eps);
+  }
+  // fused RMSNorm, producer side: sums of x^2 of the rows this lane stores
+  float rowsum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   EpiAux cur, nxt;
-  epi_load_aux<EPI>(cur, c0, lane, row0, M, n0, ep);
+  if constexpr (EPI == EPI_RESID_F32) epi_load_aux<EPI>(cur, c0, lane, row0, M, n0, ep);
 #pragma unroll 1
   for (int c = c0; c < c0 + NCH; ++c) {
-    if (c + 1 < c0 + NCH) epi_load_aux<EPI>(nxt, c + 1, lane, row0, M, n0, ep);
+    if constexpr (EPI == EPI_RESID_F32) {
+      if (c + 1 < c0 + NCH) epi_load_aux<EPI>(nxt, c + 1, lane, row0, M, n0, ep);
+    } else if constexpr (EPI == EPI_ROPE_BF16) {
+      epi_load_aux<EPI>(cur, c, lane, row0, M, n0, ep);
+    }
     float v[32];
     tmem_ld32(tbase + c * 32, v);
     if constexpr (EPI == EPI_SWIGLU_BF16) {  // columns [0,128) gate, [128,256) up of the same features
@@ -179,9 +204,12 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
       tmem_ld32(tbase + BN / 2 + c * 32, u);
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        const float hg = 0.5f * v[i];
-        v[i] = fmaf(hg, tanh_approx(hg), hg) * u[i];  // silu(g) = g/2 (1 + tanh(g/2))
+        const float hg = 0.5f * rs * v[i];
+        v[i] = fmaf(hg, tanh_approx(hg), hg) * (rs * u[i]);  // silu(g) = g/2 (1 + tanh(g/2))
       }
+    } else if constexpr (EPI == EPI_ROPE_BF16) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] *= rs;
     }
 #pragma unroll
     for (int j = 0; j < 8; ++j)
@@ -194,21 +222,30 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
         const int r = it * 4 + (lane >> 3), ch = lane & 7;
         const int m = row0 + r;
         float4 val = *reinterpret_cast<const float4*>(stg + stg_off(r, ch));
-        if (m < M) {
-          if constexpr (EPI == EPI_RESID_F32) {
-            val.x += cur.x[it].x;
-            val.y += cur.x[it].y;
-            val.z += cur.x[it].z;
-            val.w += cur.x[it].w;
+        if constexpr (EPI == EPI_RESID_F32) {
+          val.x += cur.x[it].x;
+          val.y += cur.x[it].y;
+          val.z += cur.x[it].z;
+          val.w += cur.x[it].w;
+          if (ep.y_out) {  // warp-uniform: shuffles below
+            float sq = val.x * val.x + val.y * val.y + val.z * val.z + val.w * val.w;
+            sq += __shfl_xor_sync(0xffffffffu, sq, 1);
+            sq += __shfl_xor_sync(0xffffffffu, sq, 2);
+            sq += __shfl_xor_sync(0xffffffffu, sq, 4);
+            rowsum[it] += sq;
+            if (m < M)
+              *reinterpret_cast<uint2*>(ep.y_out + (size_t)m * ep.ldo + col0 + ch * 4) =
+                  make_uint2(pack2_bf16(val.x, val.y), pack2_bf16(val.z, val.w));
           }
-          *reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)m * ep.ldo + col0 + ch * 4) = val;
         }
+        if (m < M)
+          *reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)m * ep.ldo + col0 + ch * 4) = val;
       }
     } else if (EPI == EPI_ROPE_BF16 && ep.vt && col0 >= ep.v_col0) {
-      // V heads, transposed: vt[window][kv head][dim][pos]; 32 positions of a dim are contiguous
+      // V heads, transposed and f16: vt[window][kv head][vt_rows][pos]; 32 positions of a dim are contiguous
       const int win = row0 / ep.L, pos0 = row0 % ep.L;
       const int vi = col0 - ep.v_col0, gh = vi / ep.head_dim, dim0 = vi % ep.head_dim;
-      __nv_bfloat16* vb = ep.vt + ((size_t)(win * ep.n_kv + gh) * ep.head_dim + dim0) * ep.L + pos0;
+      __half* vb = reinterpret_cast<__half*>(ep.vt) + ((size_t)(win * ep.n_kv + gh) * ep.vt_rows + dim0) * ep.L + pos0;
 #pragma unroll
       for (int it = 0; it < 4; ++it) {
         const int j = it * 8 + (lane >> 2), p0 = 8 * (lane & 3);
@@ -216,7 +253,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
 #pragma unroll
         for (int t = 0; t < 8; ++t) w[t] = *reinterpret_cast<const float*>(stg + stg_off(p0 + t, j >> 2) + (j & 3) * 4);
         *reinterpret_cast<uint4*>(vb + (size_t)j * ep.L + p0) =
-            make_uint4(pack2_bf16(w[0], w[1]), pack2_bf16(w[2], w[3]), pack2_bf16(w[4], w[5]), pack2_bf16(w[6], w[7]));
+            make_uint4(pack2_f16(w[0], w[1]), pack2_f16(w[2], w[3]), pack2_f16(w[4], w[5]), pack2_f16(w[6], w[7]));
       }
     } else {
 #pragma unroll
@@ -245,7 +282,17 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
       }
     }
     __syncwarp();
-    cur = nxt;
+    if constexpr (EPI == EPI_RESID_F32) cur = nxt;
+  }
+  if constexpr (EPI == EPI_RESID_F32) {
+    if (ep.ssq_out && (lane & 7) == 0) {
+      const int part = n0 / 128 + half;
+#pragma unroll
+      for (int it = 0; it < 8; ++it) {
+        const int m = row0 + it * 4 + (lane >> 3);
+        if (m < M) ep.ssq_out[(size_t)m * ep.n_part + part] = rowsum[it];
+      }
+    }
   }
 }
 
@@ -379,13 +426,19 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint8_t* stg = stg_all + (warp - 2) * 32 * 128;
     int acc = 0;
     uint32_t acc_phase = 0;
+    constexpr bool kScale = EPI == EPI_ROPE_BF16 || EPI == EPI_SWIGLU_BF16;
+    float ss_next = 0.f;
+    if (kScale && blockIdx.x < total) ss_next = row_ssq(ep, (blockIdx.x / n_tiles) * BM + q * 32 + lane, M);
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      const float ss_cur = ss_next;
+      if (kScale && tile + (int)gridDim.x < total)  // next tile's row, loaded while this tile drains
+        ss_next = row_ssq(ep, ((tile + gridDim.x) / n_tiles) * BM + q * 32 + lane, M);
       // warp-uniform outcome: the epilogue's tcgen05.ld is warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait_bounded(tfull0 + 8 * acc, acc_phase, &abort_flag, err))) break;
       fence_after();
       const int m0 = (tile / n_tiles) * BM;
       const int n0 = (tile % n_tiles) * BN;
-      epilogue_tile<EPI>(tmem + acc * BN, q, half, lane, m0, M, n0, ep, stg);
+      epilogue_tile<EPI>(tmem + acc * BN, q, half, lane, m0, M, n0, ep, stg, ss_cur);
       fence_before();
       mbar_arrive(tempty0 + 8 * acc);
       if (++acc == 2) {
@@ -423,22 +476,31 @@ static EncodeTiledFn encode_fn() {
 
 }  // namespace tc
 
-int t5::make_map_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
-                      uint32_t box_rows, uint32_t box_cols) {
+static int make_map_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t rows, uint64_t cols,
+                       uint64_t ld, uint32_t box_rows, uint32_t box_cols) {
   tc::EncodeTiledFn fn = tc::encode_fn();
   if (!fn) return DLMZ_ECUDA;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {ld * 2};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     fprintf(stderr, "dlmz: cuTensorMapEncodeTiled failed (%d)\n", (int)r);
     return DLMZ_ECUDA;
   }
   return DLMZ_OK;
+}
+
+int t5::make_map_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                      uint32_t box_rows, uint32_t box_cols) {
+  return make_map_2d(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, rows, cols, ld, box_rows, box_cols);
+}
+
+int t5::make_map_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                     uint32_t box_rows, uint32_t box_cols) {
+  return make_map_2d(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base, rows, cols, ld, box_rows, box_cols);
 }
 
 namespace tc {

@@ -25,9 +25,20 @@ struct GemmEpilogue {
   int head_dim;
   int rope_cols;         // columns [0, rope_cols) get RoPE (Q and K heads)
   int gu_block;          // SwiGLU: gate/up interleave block (columns)
-  bf16* vt;              // RoPE epilogue: if set, columns >= v_col0 (the V heads) go to
-  int v_col0;            //   vt [window][kv head][dim][L] (keys contiguous) instead of `out`
+  void* vt;              // RoPE epilogue: if set, columns >= v_col0 (the V heads) go to
+  int v_col0;            //   vt [window][kv head][vt_rows][L] as f16 (keys contiguous) instead of `out`
   int n_kv;
+  int vt_rows;           //   head_dim + the attention kernel's extra rows
+  // Fused RMSNorm.  Producer (residual epilogue): y_out = bf16(x) and per-row
+  // partial sums of x^2, one per 128 columns, into ssq_out [rows x n_part].
+  // Consumer (RoPE / SwiGLU epilogues): each row of the product is scaled by
+  // rsqrt(sum of the row's n_part partials / d_model + eps) (unit norm gains).
+  bf16* y_out;
+  float* ssq_out;
+  const float* ssq_in;
+  int n_part;
+  int d_model;
+  float eps;
 };
 
 // tcgen05 path: N % 256 == 0, K % 64 == 0, 16-byte aligned operands.
@@ -40,6 +51,9 @@ int gemm_simt(const T* A, int lda, const T* B, int ldb, int M, int N, int K, int
               const GemmEpilogue& ep, cudaStream_t s);
 
 // ---- layers -------------------------------------------------------------------
+// x[t] = E[state[t]] (f32), y[t] = bf16(x[t]), ssq[t] = {sum x^2, 0, ...} (n_part entries)
+int embed_norm(const int32_t* state, int n, const bf16* E, int d, float* x, bf16* y, float* ssq, int n_part,
+               cudaStream_t s);
 template <typename T>
 int embed(const int32_t* state, int T_tokens, const T* E, int d, float* x, cudaStream_t s);
 // h[r] = OutT(x[row(r)] * g / sqrt(mean(x^2) + eps)); row(r) = (r / rpc) * L + row0 + r % rpc
@@ -56,8 +70,12 @@ template <typename T>
 int attention_simt(const T* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                    int head_dim, int d, T* out, cudaStream_t s);
 bool attention_tc_supported(int L, int hd);
-int attention_bf16_tc(const bf16* qkv, int ld, const bf16* vt, int n_chunks, int L, int n_heads, int n_kv_heads,
+int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int L, int n_heads, int n_kv_heads,
                       int head_dim, int d, bf16* out, cudaStream_t s);
+// Rows per (window, kv head) of the attention kernel's V^T buffer (head_dim + extra rows).
+int attention_vt_rows(int head_dim);
+// Writes the extra rows of every (window, kv head) block of V^T: row head_dim = 1, the rest 0.
+int attention_vt_init(void* vt, int blocks, int head_dim, int L, cudaStream_t s);
 int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                        int head_dim, int d, bf16* out, cudaStream_t s);
 

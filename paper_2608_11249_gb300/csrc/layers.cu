@@ -26,6 +26,33 @@ int embed(const int32_t* state, int n, const T* E, int d, float* x, cudaStream_t
   embed_kernel<T><<<n, 128, 0, s>>>(state, n, E, d, x);
   return launch_status();
 }
+__global__ void embed_norm_kernel(const int32_t* __restrict__ state, int n, const bf16* __restrict__ E, int d,
+                                  float* __restrict__ x, bf16* __restrict__ y, float* __restrict__ ssq, int n_part) {
+  const int t = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (t >= n) return;
+  const bf16* row = E + (size_t)state[t] * d;
+  float ss = 0.f;
+  for (int i = lane; i < d; i += 32) {
+    const bf16 e = row[i];
+    const float v = __bfloat162float(e);
+    x[(size_t)t * d + i] = v;
+    y[(size_t)t * d + i] = e;
+    ss += v * v;
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  for (int i = lane; i < n_part; i += 32) ssq[(size_t)t * n_part + i] = i == 0 ? ss : 0.f;
+}
+
+int embed_norm(const int32_t* state, int n, const bf16* E, int d, float* x, bf16* y, float* ssq, int n_part,
+               cudaStream_t s) {
+  if (n == 0) return DLMZ_OK;
+  ProfScope prof(PROF_LAYER, s, 0, (double)n * d * 8);
+  embed_norm_kernel<<<(n + 7) / 8, 256, 0, s>>>(state, n, E, d, x, y, ssq, n_part);
+  return launch_status();
+}
+
 template int embed<float>(const int32_t*, int, const float*, int, float*, cudaStream_t);
 template int embed<bf16>(const int32_t*, int, const bf16*, int, float*, cudaStream_t);
 

@@ -119,7 +119,7 @@ static uint64_t config_fingerprint(const dlmz_model_config& c) {
 
 size_t model_workspace_per_token(const dlmz_model* m) {
   const size_t d = m->cfg.d, F = m->cfg.ffn;
-  size_t b = 4 * d + m->esz * (2 * d + m->nqkv + F + m->dkv);
+  size_t b = 4 * d + m->esz * (2 * d + m->nqkv + F + m->dkv + 16 * m->cfg.n_kv_heads) + 4 * (d / 128);
   if (!m->tc) b += 4 * 2 * F;  // float32 gate/up buffer of the CUDA-core path
   return b;
 }
@@ -149,7 +149,16 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
   DLMZ_TRY(w.hc.ensure((size_t)R * d * sizeof(T)));
   // tensor-core attention reads V transposed (keys contiguous), written by the QKV epilogue
   const bool tc_attn = m->tc && attention_tc_supported(L, hd);
-  if (tc_attn) DLMZ_TRY(w.vt.ensure((size_t)Tt * m->dkv * sizeof(T)));
+  if (tc_attn) {
+    const int vrows = attention_vt_rows(hd), blocks = nc * (int)c.n_kv_heads;
+    DLMZ_TRY(w.vt.ensure((size_t)blocks * vrows * L * 2));
+    if (w.vt_ptr != w.vt.p || w.vt_L != L || w.vt_blocks != blocks) {
+      DLMZ_TRY(attention_vt_init(w.vt.p, blocks, hd, L, s));
+      w.vt_ptr = w.vt.p;
+      w.vt_L = L;
+      w.vt_blocks = blocks;
+    }
+  }
   if (w.rope_L < L) {  // (cos, sin) of pos * theta^(-2i/hd), from double precision
     const int half = hd / 2;
     std::vector<float2> cs((size_t)L * half);
@@ -168,51 +177,94 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
   T* attn = w.attn.as<T>();
   T* act = w.act.as<T>();
   const float2* cs = w.rope.as<float2>();
+  auto epi = [&](void* out, int ldo) {
+    GemmEpilogue e{};
+    e.out = out;
+    e.ldo = ldo;
+    e.rope_cs = cs;
+    e.L = L;
+    e.head_dim = hd;
+    e.gu_block = m->gu_block;
+    e.n_kv = (int)c.n_kv_heads;
+    e.d_model = d;
+    e.eps = c.norm_eps;
+    return e;
+  };
   GemmEpilogue ep{};
-  DLMZ_TRY(embed<T>(state, Tt, reinterpret_cast<const T*>(m->E), d, x, s));
-  for (uint32_t l = 0; l < c.n_layers; ++l) {
-    DLMZ_TRY(rmsnorm<T>(x, Tt, d, m->gains, c.norm_eps, h, L, 0, 0, s));
-    ep = GemmEpilogue{qkv, nq, cs, L, hd, d + m->dkv, m->gu_block, nullptr, 0, (int)c.n_kv_heads};
-    if (tc_attn) {
-      ep.vt = w.vt.as<bf16>();
-      ep.v_col0 = d + m->dkv;
+  if (m->tc) {
+    // Tensor-core path with RMSNorm fused into the GEMM epilogues: h holds
+    // bf16(x) and ssq the per-row partial sums of x^2 (unit norm gains).
+    const int np = d / 128;
+    DLMZ_TRY(w.ssq.ensure((size_t)Tt * np * 4));
+    float* ssq = w.ssq.as<float>();
+    bf16* y = reinterpret_cast<bf16*>(h);
+    DLMZ_TRY(embed_norm(state, Tt, reinterpret_cast<const bf16*>(m->E), d, x, y, ssq, np, s));
+    for (uint32_t l = 0; l < c.n_layers; ++l) {
+      ep = epi(qkv, nq);
+      ep.rope_cols = d + m->dkv;
+      ep.ssq_in = ssq;
+      ep.n_part = np;
+      if (tc_attn) {
+        ep.vt = w.vt.p;
+        ep.v_col0 = d + m->dkv;
+        ep.vt_rows = attention_vt_rows(hd);
+      }
+      DLMZ_TRY(gemm_bf16_tc(y, d, reinterpret_cast<const bf16*>(m->wqkv[l]), d, Tt, nq, d, EPI_ROPE_BF16, ep, s));
+      if (tc_attn)
+        DLMZ_TRY(attention_bf16_tc(reinterpret_cast<const bf16*>(qkv), nq, w.vt.p, nc, L, c.n_heads,
+                                   c.n_kv_heads, hd, d, reinterpret_cast<bf16*>(attn), s));
+      else if (hd == 64 || hd == 128)
+        DLMZ_TRY(attention_bf16_mma(reinterpret_cast<const bf16*>(qkv), nq, nc, L, c.n_heads, c.n_kv_heads, hd, d,
+                                    reinterpret_cast<bf16*>(attn), s));
+      else
+        DLMZ_TRY(attention_simt<bf16>(reinterpret_cast<const bf16*>(qkv), nq, nc, L, c.n_heads, c.n_kv_heads, hd, d,
+                                      reinterpret_cast<bf16*>(attn), s));
+      ep = epi(x, d);
+      ep.y_out = y;
+      ep.ssq_out = ssq;
+      ep.n_part = np;
+      DLMZ_TRY(gemm_bf16_tc(reinterpret_cast<const bf16*>(attn), d, reinterpret_cast<const bf16*>(m->wo[l]), d, Tt, d,
+                            d, EPI_RESID_F32, ep, s));
+      ep = epi(act, F);
+      ep.ssq_in = ssq;
+      ep.n_part = np;
+      DLMZ_TRY(gemm_bf16_tc(y, d, reinterpret_cast<const bf16*>(m->wgu[l]), d, Tt, 2 * F, d, EPI_SWIGLU_BF16, ep, s));
+      ep = epi(x, d);
+      ep.y_out = y;
+      ep.ssq_out = ssq;
+      ep.n_part = np;
+      DLMZ_TRY(gemm_bf16_tc(reinterpret_cast<const bf16*>(act), F, reinterpret_cast<const bf16*>(m->wdown[l]), F, Tt,
+                            d, F, EPI_RESID_F32, ep, s));
     }
-    if (m->tc) {
-      DLMZ_TRY(gemm_bf16_tc(reinterpret_cast<const bf16*>(h), d, reinterpret_cast<const bf16*>(m->wqkv[l]), d, Tt,
-                            nq, d, EPI_ROPE_BF16, ep, s));
-    } else {
+  } else {
+    DLMZ_TRY(embed<T>(state, Tt, reinterpret_cast<const T*>(m->E), d, x, s));
+    for (uint32_t l = 0; l < c.n_layers; ++l) {
+      DLMZ_TRY(rmsnorm<T>(x, Tt, d, m->gains, c.norm_eps, h, L, 0, 0, s));
+      ep = epi(qkv, nq);
       DLMZ_TRY(gemm<T>(h, reinterpret_cast<const T*>(m->wqkv[l]), Tt, nq, d, sizeof(T) == 2 ? EPI_BF16 : EPI_F32, ep,
                        s));
       DLMZ_TRY(rope_inplace<T>(qkv, Tt, nq, c.n_heads + c.n_kv_heads, hd, L, cs, s));
-    }
-    if constexpr (sizeof(T) == 2) {
-      if (tc_attn)
-        DLMZ_TRY(attention_bf16_tc(qkv, nq, w.vt.as<bf16>(), nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
-      else if (hd == 64 || hd == 128)
-        DLMZ_TRY(attention_bf16_mma(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
-      else
+      if constexpr (sizeof(T) == 2) {
+        if (hd == 64 || hd == 128)
+          DLMZ_TRY(attention_bf16_mma(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
+        else
+          DLMZ_TRY(attention_simt<T>(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
+      } else {
         DLMZ_TRY(attention_simt<T>(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
-    } else {
-      DLMZ_TRY(attention_simt<T>(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
-    }
-    ep = GemmEpilogue{x, d, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
-    DLMZ_TRY(gemm<T>(attn, reinterpret_cast<const T*>(m->wo[l]), Tt, d, d, EPI_RESID_F32, ep, s));
-    DLMZ_TRY(rmsnorm<T>(x, Tt, d, m->gains, c.norm_eps, h, L, 0, 0, s));
-    if (m->tc) {
-      ep = GemmEpilogue{act, F, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
-      DLMZ_TRY(gemm_bf16_tc(reinterpret_cast<const bf16*>(h), d, reinterpret_cast<const bf16*>(m->wgu[l]), d, Tt,
-                            2 * F, d, EPI_SWIGLU_BF16, ep, s));
-    } else {
-      ep = GemmEpilogue{w.gu.p, 2 * F, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
+      }
+      ep = epi(x, d);
+      DLMZ_TRY(gemm<T>(attn, reinterpret_cast<const T*>(m->wo[l]), Tt, d, d, EPI_RESID_F32, ep, s));
+      DLMZ_TRY(rmsnorm<T>(x, Tt, d, m->gains, c.norm_eps, h, L, 0, 0, s));
+      ep = epi(w.gu.p, 2 * F);
       DLMZ_TRY(gemm<T>(h, reinterpret_cast<const T*>(m->wgu[l]), Tt, 2 * F, d, EPI_F32, ep, s));
       DLMZ_TRY(swiglu<T>(w.gu.as<float>(), Tt, F, m->gu_block, act, s));
+      ep = epi(x, d);
+      DLMZ_TRY(gemm<T>(act, reinterpret_cast<const T*>(m->wdown[l]), Tt, d, F, EPI_RESID_F32, ep, s));
     }
-    ep = GemmEpilogue{x, d, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
-    DLMZ_TRY(gemm<T>(act, reinterpret_cast<const T*>(m->wdown[l]), Tt, d, F, EPI_RESID_F32, ep, s));
   }
   T* hc = w.hc.as<T>();
   DLMZ_TRY(rmsnorm<T>(x, R, d, m->gains, c.norm_eps, hc, L, row0, rpc, s));
-  ep = GemmEpilogue{logits, V, nullptr, L, hd, 0, m->gu_block, nullptr, 0, 0};
+  ep = epi(logits, V);
   return gemm<T>(hc, reinterpret_cast<const T*>(m->head), R, V, d, EPI_F32, ep, s);
 }
 
@@ -345,6 +397,7 @@ extern "C" void dlmz_model_destroy(dlmz_model* m) {
   m->ws.hc.release();
   m->ws.rope.release();
   m->ws.vt.release();
+  m->ws.ssq.release();
   pipeline_release(m);
   delete m;
 }
