@@ -211,11 +211,22 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] *= rs;
     }
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      *reinterpret_cast<float4*>(stg + stg_off(lane, j)) = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-    __syncwarp();
     const int col0 = (EPI == EPI_SWIGLU_BF16 ? n0 / 2 : n0) + c * 32;
+    // V heads of the QKV projection are staged transposed ([dim][token], a
+    // thread writes its token down a column, each dim row rotated by
+    // 4 * (dim mod 8) floats so both the 4-byte writes and the 16-byte reads of
+    // token runs are free of bank conflicts); everything else is staged
+    // [token][dim] with 16-byte chunks swizzled by row.
+    const bool vt_chunk = EPI == EPI_ROPE_BF16 && ep.vt && col0 >= ep.v_col0;
+    if (vt_chunk) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) reinterpret_cast<float*>(stg)[j * 32 + ((lane + 4 * (j & 7)) & 31)] = v[j];
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        *reinterpret_cast<float4*>(stg + stg_off(lane, j)) = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+    }
+    __syncwarp();
     if constexpr (EPI == EPI_F32 || EPI == EPI_RESID_F32) {
 #pragma unroll
       for (int it = 0; it < 8; ++it) {
@@ -241,7 +252,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
         if (m < M)
           *reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)m * ep.ldo + col0 + ch * 4) = val;
       }
-    } else if (EPI == EPI_ROPE_BF16 && ep.vt && col0 >= ep.v_col0) {
+    } else if (vt_chunk) {
       // V heads, transposed and f16: vt[window][kv head][vt_rows][pos]; 32 positions of a dim are contiguous
       const int win = row0 / ep.L, pos0 = row0 % ep.L;
       const int vi = col0 - ep.v_col0, gh = vi / ep.head_dim, dim0 = vi % ep.head_dim;
@@ -249,9 +260,9 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
 #pragma unroll
       for (int it = 0; it < 4; ++it) {
         const int j = it * 8 + (lane >> 2), p0 = 8 * (lane & 3);
-        float w[8];
-#pragma unroll
-        for (int t = 0; t < 8; ++t) w[t] = *reinterpret_cast<const float*>(stg + stg_off(p0 + t, j >> 2) + (j & 3) * 4);
+        const float4 a = *reinterpret_cast<const float4*>(stg + (j * 32 + ((p0 + 4 * (j & 7)) & 31)) * 4);
+        const float4 b = *reinterpret_cast<const float4*>(stg + (j * 32 + ((p0 + 4 + 4 * (j & 7)) & 31)) * 4);
+        const float w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
         *reinterpret_cast<uint4*>(vb + (size_t)j * ep.L + p0) =
             make_uint4(pack2_f16(w[0], w[1]), pack2_f16(w[2], w[3]), pack2_f16(w[4], w[5]), pack2_f16(w[6], w[7]));
       }
