@@ -2,8 +2,9 @@
 // every position attends to every position of its window, no mask).
 //
 // CTA = (128 queries, head, window), 6 warps:
-//   warp 0      TMA: Q once; per key tile of 128: K (into a single buffer)
-//               and V^T (keys contiguous, written so by the QKV epilogue).
+//   warp 0      TMA: Q once; per key tile of 128: K (2-stage ring, requested
+//               one tile ahead of V) and V^T (keys contiguous, written so by
+//               the QKV epilogue; single buffer).
 //   warp 1      allocates 256 TMEM columns (S: 128, O: head_dim) and issues
 //               S_j = Q K_j^T and O += P_j V_j with tcgen05.mma from one thread.
 //   warps 2-5   softmax, one thread per query row (its TMEM lane): the row of
@@ -33,8 +34,9 @@ template <int HD>
 struct Smem {
   static constexpr int HDP = HD + VT_EXTRA;
   static constexpr int Q = 0;                        // HD/64 blocks of [128 x 64] bf16
-  static constexpr int K = Q + BQ * HD * 2;          // HD/64 blocks of [128 x 64]
-  static constexpr int VT = K + BK * HD * 2;         // 2 blocks of [HDP x 64] f16 (keys 0-63, 64-127)
+  static constexpr int KT = BK * HD * 2;             // one key tile: HD/64 blocks of [128 x 64]
+  static constexpr int K = Q + BQ * HD * 2;          // 2 key tiles
+  static constexpr int VT = K + 2 * KT;              // 2 blocks of [HDP x 64] f16 (keys 0-63, 64-127)
   static constexpr int P = VT + HDP * BK * 2;        // 2 blocks of [128 x 64] f16
   static constexpr int BARS = P + BQ * BK * 2;
   static constexpr int TOTAL = BARS + 128 + 1024;    // + barriers + alignment slack
@@ -52,8 +54,10 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t base = smem_u32(sm);
   const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT, sP = base + S::P;
   const uint32_t bar = base + S::BARS;
-  const uint32_t q_full = bar, k_full = bar + 8, k_empty = bar + 16, v_full = bar + 24, v_empty = bar + 32,
-                 s_full = bar + 40, p_ready = bar + 48, o_done = bar + 56;
+  const uint32_t q_full = bar, v_full = bar + 24, v_empty = bar + 32, s_full = bar + 40, p_ready = bar + 48,
+                 o_done = bar + 56;
+  auto k_full = [&](int st) { return st ? bar + 72 : bar + 8; };   // per key stage
+  auto k_empty = [&](int st) { return st ? bar + 80 : bar + 16; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int w = blockIdx.z, h = blockIdx.y, q0 = blockIdx.x * BQ;
   const int g = h / (nh / nkv);
@@ -62,8 +66,10 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (threadIdx.x == 0) {
     abort_flag = 0;
     mbar_init(q_full, 1);
-    mbar_init(k_full, 1);
-    mbar_init(k_empty, 1);
+    for (int st = 0; st < 2; ++st) {
+      mbar_init(k_full(st), 1);
+      mbar_init(k_empty(st), 1);
+    }
     mbar_init(v_full, 1);
     mbar_init(v_empty, 1);
     mbar_init(s_full, 1);
@@ -84,26 +90,35 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int row0 = w * L;
       mbar_arrive_expect_tx(q_full, BQ * HD * 2);
       for (int kb = 0; kb < HD / 64; ++kb) t5::tma_load_2d(sQ + kb * BQ * 128, &tmQK, h * HD + kb * 64, row0 + q0, q_full);
-      bool k_pend = false, v_pend = false;
-      uint32_t kp = 0, vp = 0;
-      for (int j = 0; j < nt && !abort_flag; ++j) {
-        if (!mbar_wait_bounded(k_empty, (j & 1) ^ 1, &abort_flag, err)) break;
-        mbar_arrive_expect_tx(k_full, BK * HD * 2);
-        for (int kb = 0; kb < HD / 64; ++kb)
-          t5::tma_load_2d(sK + kb * BK * 128, &tmQK, d + g * HD + kb * 64, row0 + j * BK, k_full);
-        k_pend = true;
-        kp = j & 1;
-        if (!mbar_wait_bounded(v_empty, (j & 1) ^ 1, &abort_flag, err)) break;
-        mbar_arrive_expect_tx(v_full, BK * HDP * 2);
-        for (int kk = 0; kk < 2; ++kk)
-          t5::tma_load_2d(sVt + kk * HDP * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HDP, v_full);
-        v_pend = true;
-        vp = j & 1;
+      uint32_t kpend = 0, kpar[2] = {0, 0}, vp = 0;
+      bool v_pend = false;
+      // K_j is requested before V_{j-1}: K runs one tile ahead through its 2-stage ring
+      for (int j = 0; j <= nt && !abort_flag; ++j) {
+        if (j < nt) {
+          const int st = j & 1;
+          const uint32_t ph = (j >> 1) & 1;
+          if (!mbar_wait_bounded(k_empty(st), ph ^ 1, &abort_flag, err)) break;
+          mbar_arrive_expect_tx(k_full(st), BK * HD * 2);
+          for (int kb = 0; kb < HD / 64; ++kb)
+            t5::tma_load_2d(sK + st * S::KT + kb * BK * 128, &tmQK, d + g * HD + kb * 64, row0 + j * BK, k_full(st));
+          kpend |= 1u << st;
+          kpar[st] = ph;
+        }
+        if (j >= 1) {
+          const int jv = j - 1;
+          if (!mbar_wait_bounded(v_empty, (jv & 1) ^ 1, &abort_flag, err)) break;
+          mbar_arrive_expect_tx(v_full, BK * HDP * 2);
+          for (int kk = 0; kk < 2; ++kk)
+            t5::tma_load_2d(sVt + kk * HDP * 128, &tmVt, jv * BK + kk * 64, (w * nkv + g) * HDP, v_full);
+          v_pend = true;
+          vp = jv & 1;
+        }
       }
       if (abort_flag) {  // let our own copies land before the CTA can exit
         volatile int never = 0;
         mbar_wait_bounded(q_full, 0, &never, err, 100000000ull);
-        if (k_pend) mbar_wait_bounded(k_full, kp, &never, err, 100000000ull);
+        for (int st = 0; st < 2; ++st)
+          if (kpend & (1u << st)) mbar_wait_bounded(k_full(st), kpar[st], &never, err, 100000000ull);
         if (v_pend) mbar_wait_bounded(v_full, vp, &never, err, 100000000ull);
       }
     }
@@ -112,28 +127,29 @@ __global__ void __launch_bounds__(THREADS, 1)
       constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
       constexpr uint32_t ID_O = t5::idesc_f16(BQ, HDP);
       bool issued = false;
-      auto issue_s = [&]() {
+      auto issue_s = [&](int st) {
         for (int kb = 0; kb < HD / 64; ++kb)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            t5::mma_bf16(tS, t5::sw128_desc(sQ + kb * BQ * 128 + 32 * k), t5::sw128_desc(sK + kb * BK * 128 + 32 * k),
-                         ID_S, (kb | k) != 0);
+            t5::mma_bf16(tS, t5::sw128_desc(sQ + kb * BQ * 128 + 32 * k),
+                         t5::sw128_desc(sK + st * S::KT + kb * BK * 128 + 32 * k), ID_S, (kb | k) != 0);
         t5::commit(s_full);
-        t5::commit(k_empty);
+        t5::commit(k_empty(st));
         issued = true;
       };
-      bool ok = mbar_wait_bounded(q_full, 0, &abort_flag, err) && mbar_wait_bounded(k_full, 0, &abort_flag, err);
+      bool ok = mbar_wait_bounded(q_full, 0, &abort_flag, err) && mbar_wait_bounded(k_full(0), 0, &abort_flag, err);
       if (ok) {
         t5::fence_after();
-        issue_s();
+        issue_s(0);
       }
       for (int j = 0; ok && j < nt; ++j) {
         if (!mbar_wait_bounded(p_ready, j & 1, &abort_flag, err)) break;
         t5::fence_after();
         if (j + 1 < nt) {
-          if (!mbar_wait_bounded(k_full, (j + 1) & 1, &abort_flag, err)) break;
+          const int st1 = (j + 1) & 1;
+          if (!mbar_wait_bounded(k_full(st1), ((j + 1) >> 1) & 1, &abort_flag, err)) break;
           t5::fence_after();
-          issue_s();
+          issue_s(st1);
         }
         if (!mbar_wait_bounded(v_full, j & 1, &abort_flag, err)) break;
         t5::fence_after();
@@ -148,7 +164,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (abort_flag && issued) {
         volatile int never = 0;
-        const uint32_t drain = bar + 64;
+        const uint32_t drain = bar + 88;
         mbar_init(drain, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         t5::commit(drain);
@@ -170,9 +186,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       t5::fence_after();
       uint32_t sr[BK];
       t5::tmem_ld128(tS + lane_off, sr);
-      float mx = -INFINITY;
+      float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};  // 4 independent chains
 #pragma unroll
-      for (int i = 0; i < BK; ++i) mx = fmaxf(mx, __uint_as_float(sr[i]));
+      for (int i = 0; i < BK; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sr[i]));
+      float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       mx *= scale_log2;
       if (j > 0) {  // PV_{j-1} done: P buffer free, O stable
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (j - 1) & 1, &abort_flag, err))) {
