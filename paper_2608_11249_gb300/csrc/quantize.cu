@@ -266,6 +266,222 @@ __global__ void __launch_bounds__(QT) quantize_cta_kernel(const float* __restric
   if (threadIdx.x == 0) cr[0] = 0;
 }
 
+// ---- large vocabularies (V % 4 == 0): persistent, CPS CTAs of NT threads per SM ----------
+// A CTA walks rows r = blockIdx.x, blockIdx.x + gridDim.x, ...; with CPS rows
+// per SM in flight the row stays in L2 after the first pass (from HBM), and
+// the CTAs of an SM drift apart, so one row's compute-heavy CDF pass overlaps
+// another's HBM-bound first pass.  Every per-element quantity is a function
+// of the integer code q in [0, 8191] alone, so the second pass only builds a
+// histogram of q: W = sum hist[q] w(q), A = sum hist[q] w(q) q and the
+// remainder D = R - sum hist[q] floor(w(q) R / W) come from the 8192 bins, and
+// the CDF pass looks floor(w(q) R / W) up in the same shared table, rewritten
+// in place.  Every CDF partial sum is at most 2^P <= 2^24, so the scan runs
+// in 32-bit integers.
+// floor(w R / W) without a division: K = floor(R 2^64 / W) per row (R < W), the
+// estimate (w K) >> 64 is floor(w R / W) or one less, and (e + 1) W <= w R
+// (both sides < 2^64) decides which.
+constexpr int NQ = 8192;       // codes q = 0 .. 8191
+constexpr int QNT = 256;       // threads per CTA
+constexpr int QCPS = 4;        // CTAs per SM (4 x 33 KB shared memory, 64 registers per thread)
+
+__device__ __forceinline__ uint32_t floor_wr_over_w(uint32_t w, uint32_t R, uint64_t Wsum, uint64_t K) {
+  const uint64_t lo = (uint64_t)w * (uint32_t)K;          // w * K_lo
+  const uint64_t hi = (uint64_t)w * (uint32_t)(K >> 32);  // w * K_hi
+  const uint32_t est = (uint32_t)((hi + (lo >> 32)) >> 32);
+  const uint64_t x = (uint64_t)w * R;
+  return est + (((uint64_t)(est + 1) * Wsum) <= x ? 1u : 0u);
+}
+
+template <int NT, int CPS>
+__global__ void __launch_bounds__(NT, CPS)
+    quantize_persist_kernel(const float* __restrict__ logits, int rows, int V, int P, uint32_t* __restrict__ cdf,
+                            uint64_t* __restrict__ Wout, uint64_t* __restrict__ Aout, int32_t* __restrict__ Hq,
+                            int32_t* __restrict__ topout, float* __restrict__ mxout, int* err) {
+  constexpr int NW = NT / 32;
+  static_assert(NT % 32 == 0 && NW <= 32 && NQ % NT == 0, "block shape");
+  __shared__ uint32_t T[256];
+  __shared__ uint32_t tab[NQ];  // histogram of q, then floor(w(q) R / W)
+  __shared__ float redf[NW];
+  __shared__ int redi[NW];
+  __shared__ uint64_t redu[NW], redu2[NW];
+  __shared__ uint32_t wtot[2][NW];
+  __shared__ uint64_t s_K, s_W;
+  __shared__ uint32_t s_D;
+  __shared__ float s_m;
+  __shared__ int s_top;
+  for (int i = threadIdx.x; i < 256; i += NT) T[i] = c_exp_table[i];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n4 = V >> 2;
+  const uint32_t R = (1u << P) - (uint32_t)V;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    const float4* l4 = reinterpret_cast<const float4*>(logits + (size_t)r * V);
+    // pass 1 (HBM): max; x - x is NaN exactly for non-finite x
+    float m = -INFINITY, nf = 0.f;
+    {
+      constexpr int U = 4;  // independent 16-byte loads in flight per thread
+      int i0 = threadIdx.x;
+      for (; i0 + (U - 1) * NT < n4; i0 += U * NT) {
+        float4 xv[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) xv[u] = l4[i0 + u * NT];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const float4 x = xv[u];
+          m = fmaxf(fmaxf(m, x.x), fmaxf(fmaxf(x.y, x.z), x.w));
+          nf += (x.x - x.x) + (x.y - x.y) + (x.z - x.z) + (x.w - x.w);
+        }
+      }
+      for (; i0 < n4; i0 += NT) {
+        const float4 x = l4[i0];
+        m = fmaxf(fmaxf(m, x.x), fmaxf(fmaxf(x.y, x.z), x.w));
+        nf += (x.x - x.x) + (x.y - x.y) + (x.z - x.z) + (x.w - x.w);
+      }
+    }
+    int bad = !(nf == 0.f);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+      bad |= __shfl_xor_sync(0xffffffffu, bad, o);
+    }
+    __syncthreads();  // previous row done with the shared state
+    for (int b = threadIdx.x; b < NQ; b += NT) tab[b] = 0;
+    if (lane == 0) {
+      redf[warp] = m;
+      redi[warp] = bad;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      float m2 = lane < NW ? redf[lane] : -INFINITY;
+      int b2 = lane < NW ? redi[lane] : 0;
+#pragma unroll
+      for (int o = 16; o; o >>= 1) {
+        m2 = fmaxf(m2, __shfl_xor_sync(0xffffffffu, m2, o));
+        b2 |= __shfl_xor_sync(0xffffffffu, b2, o);
+      }
+      if (lane == 0) {
+        if (b2) {
+          atomicOr(err, ERR_NONFINITE);  // the call fails; outputs stay defined
+          m2 = 0.f;
+        }
+        s_m = m2;
+      }
+    }
+    __syncthreads();
+    m = s_m;
+    // pass 2 (L2): histogram of q, lowest index of the maximum
+    int topc = 0x7fffffff;
+    for (int i0 = threadIdx.x; i0 < n4; i0 += 2 * NT) {
+      const bool two = i0 + NT < n4;
+      const float4 xa = l4[i0];
+      const float4 xb = two ? l4[i0 + NT] : xa;
+      const float xs[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        if (e < 4 || two) {
+          if (xs[e] == m) topc = min(topc, 4 * (e < 4 ? i0 : i0 + NT) + (e & 3));
+          atomicAdd(&tab[quant_q(m, xs[e])], 1u);
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) topc = min(topc, __shfl_xor_sync(0xffffffffu, topc, o));
+    if (lane == 0) redi[warp] = topc;
+    __syncthreads();
+    // per-row sums over the bins (each thread owns bins threadIdx.x + k NT here and below)
+    uint64_t Ws = 0, As = 0;
+    for (int b = threadIdx.x; b < NQ; b += NT) {
+      const uint64_t hw = (uint64_t)tab[b] * quant_w(T, b);
+      Ws += hw;
+      As += hw * (uint32_t)b;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      Ws += __shfl_xor_sync(0xffffffffu, Ws, o);
+      As += __shfl_xor_sync(0xffffffffu, As, o);
+    }
+    if (lane == 0) {
+      redu[warp] = Ws;
+      redu2[warp] = As;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      uint64_t tw = 0, ta = 0;
+      int tp = 0x7fffffff;
+      for (int i = 0; i < NW; ++i) {
+        tw += redu[i];
+        ta += redu2[i];
+        tp = min(tp, redi[i]);
+      }
+      if (tp == 0x7fffffff) tp = 0;  // only for rows flagged non-finite
+      s_top = tp;
+      s_K = (uint64_t)(((unsigned __int128)R << 64) / tw);
+      s_W = tw;
+      Wout[r] = tw;
+      if (Aout) Aout[r] = ta;
+      Hq[r] = entropy_q(tw, ta);
+      if (topout) topout[r] = tp;
+      if (mxout) mxout[r] = m;
+    }
+    __syncthreads();
+    if (!cdf) continue;
+    const uint64_t Wr = s_W, K = s_K;
+    const int top = s_top;
+    // floor(w(q) R / W) per code, over its own bin's count, and the histogram-weighted sum
+    uint32_t fsum = 0;  // <= R
+    for (int b = threadIdx.x; b < NQ; b += NT) {
+      const uint32_t f = floor_wr_over_w(quant_w(T, b), R, Wr, K);
+      fsum += tab[b] * f;
+      tab[b] = f;
+    }
+    fsum = __reduce_add_sync(0xffffffffu, fsum);
+    if (lane == 0) redi[warp] = (int)fsum;
+    __syncthreads();  // the floor table complete
+    const uint32_t D = R - __reduce_add_sync(0xffffffffu, lane < NW ? (uint32_t)redi[lane] : 0u);
+    // CDF[v+1] = (v+1) + sum_{u<=v} floor(w_u R / W) + (v >= top ? D : 0), scanned in
+    // block-wide tiles of 4 NT elements (a float4 per thread, from L2); the next
+    // tile's load is issued before this tile's barrier
+    uint32_t* cr = cdf + (size_t)r * (V + 1);
+    if (threadIdx.x == 0) cr[0] = 0;
+    uint32_t carry = 0;
+    int buf = 0;
+    float4 xn = threadIdx.x < n4 ? __ldcs(l4 + threadIdx.x) : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int base = 0; base < n4; base += NT) {
+      const int i = base + threadIdx.x;
+      const float4 x = xn;
+      if (i + NT < n4) xn = __ldcs(l4 + i + NT);
+      uint32_t f0 = 0, f1 = 0, f2 = 0, f3 = 0;
+      if (i < n4) {
+        f0 = tab[quant_q(m, x.x)];
+        f1 = tab[quant_q(m, x.y)];
+        f2 = tab[quant_q(m, x.z)];
+        f3 = tab[quant_q(m, x.w)];
+      }
+      const uint32_t c1 = f0 + f1, c2 = c1 + f2, lsum = c2 + f3;
+      uint32_t inc = lsum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += t;
+      }
+      if (lane == 31) wtot[buf][warp] = inc;
+      __syncthreads();
+      const uint32_t tv = lane < NW ? wtot[buf][lane] : 0u;
+      const uint32_t pre = __reduce_add_sync(0xffffffffu, lane < warp ? tv : 0u);
+      const uint32_t basev = carry + pre + (inc - lsum);
+      carry += __reduce_add_sync(0xffffffffu, tv);
+      buf ^= 1;
+      if (i < n4) {
+        const int v = 4 * i;
+        const uint32_t c0 = (uint32_t)v + 1u + basev;
+        __stcs(cr + v + 1, c0 + f0 + (v >= top ? D : 0u));
+        __stcs(cr + v + 2, c0 + 1u + c1 + (v + 1 >= top ? D : 0u));
+        __stcs(cr + v + 3, c0 + 2u + c2 + (v + 2 >= top ? D : 0u));
+        __stcs(cr + v + 4, c0 + 3u + lsum + (v + 3 >= top ? D : 0u));
+      }
+    }
+  }
+}
+
 int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, uint64_t* W, uint64_t* A, int32_t* Hq,
                   int32_t* top, float* mx, cudaStream_t s) {
   if (rows == 0) return DLMZ_OK;
@@ -277,7 +493,12 @@ int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, ui
   else if (V <= 128) quantize_warp_kernel<4><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V <= 256) quantize_warp_kernel<8><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V <= 512) quantize_warp_kernel<16><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
-  else quantize_cta_kernel<<<rows, QT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  else if (V % 4 == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0) {
+    const int g = rows < QCPS * num_sms() ? rows : QCPS * num_sms();
+    quantize_persist_kernel<QNT, QCPS><<<g, QNT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  } else {
+    quantize_cta_kernel<<<rows, QT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+  }
   return launch_status();
 }
 

@@ -18,7 +18,7 @@ def _rows(V, n, seed):
     return np.concatenate([l, np.array(extra, dtype=np.float32)]).astype(np.float32)
 
 
-@pytest.mark.parametrize("V,n", [(2, 9), (4, 33), (37, 70), (256, 300), (300, 50), (512, 40), (1000, 20),
+@pytest.mark.parametrize("V,n", [(2, 9), (4, 33), (37, 70), (256, 300), (300, 50), (512, 40), (1000, 20), (1001, 7),
                                  (5000, 17), (126464, 5), (152064, 3)])
 def test_quantize_bit_exact(dev, V, n):
     import torch
