@@ -87,9 +87,10 @@ __global__ void __launch_bounds__(256) quantize_warp_kernel(const float* __restr
     const int i2 = __shfl_xor_sync(0xffffffffu, mi, o);
     argmax_merge(m, mi, m2, i2);
   }
-  if (!__all_sync(0xffffffffu, finite)) {
+  const bool bad = !__all_sync(0xffffffffu, finite);
+  if (bad) {  // the call reports EBADINPUT; m = +inf sends every code to 8191, W is pinned below
     if (lane == 0) atomicOr(err, ERR_NONFINITE);
-    m = 0.f;  // keep going with defined values; the call reports EBADINPUT
+    m = INFINITY;
   }
   uint32_t w[NPL];
   uint64_t Ws = 0, As = 0;
@@ -109,6 +110,10 @@ __global__ void __launch_bounds__(256) quantize_warp_kernel(const float* __restr
   for (int o = 16; o; o >>= 1) {
     Ws += __shfl_xor_sync(0xffffffffu, Ws, o);
     As += __shfl_xor_sync(0xffffffffu, As, o);
+  }
+  if (bad) {  // every w is 0: any W >= 2^31 keeps the tables defined
+    Ws = 1ull << 31;
+    As = 0;
   }
   if (lane == 0) {
     Wout[r] = Ws;
@@ -202,9 +207,9 @@ __global__ void __launch_bounds__(QT) quantize_cta_kernel(const float* __restric
     bad |= redi[i] < 0;
     argmax_merge(m, mi, redf[i], redi[i] & 0x7fffffff);
   }
-  if (bad) {
+  if (bad) {  // as in the warp kernel: every code 8191, W pinned to 2^31
     if (threadIdx.x == 0) atomicOr(err, ERR_NONFINITE);
-    m = 0.f;
+    m = INFINITY;
   }
   // pass 2: W, A
   uint64_t Ws = 0, As = 0;
@@ -217,6 +222,10 @@ __global__ void __launch_bounds__(QT) quantize_cta_kernel(const float* __restric
   }
   Ws = block_sum(Ws, redu);
   As = block_sum(As, redu);
+  if (bad) {
+    Ws = 1ull << 31;
+    As = 0;
+  }
   if (threadIdx.x == 0) {
     Wout[r] = Ws;
     if (Aout) Aout[r] = As;
@@ -281,6 +290,9 @@ __global__ void __launch_bounds__(QT) quantize_cta_kernel(const float* __restric
 // estimate (w K) >> 64 is floor(w R / W) or one less, and (e + 1) W <= w R
 // (both sides < 2^64) decides which.
 constexpr int NQ = 8192;       // codes q = 0 .. 8191
+// w(q) = T[q & 255] >> (q >> 8) is 0 for q > 7936 (T[j] < 2^31 for j >= 1; w(7936) = T[0] >> 31 = 1):
+// those codes add nothing to W, A or D and need no bin
+constexpr int QW0 = 31 * 256 + 1;
 constexpr int QNT = 256;       // threads per CTA
 constexpr int QCPS = 4;        // CTAs per SM (4 x 33 KB shared memory, 64 registers per thread)
 
@@ -304,11 +316,10 @@ __global__ void __launch_bounds__(NT, CPS)
   __shared__ float redf[NW];
   __shared__ int redi[NW];
   __shared__ uint64_t redu[NW], redu2[NW];
-  __shared__ uint32_t wtot[2][NW];
+  __shared__ uint32_t wtot[2][4][NW];
   __shared__ uint64_t s_K, s_W;
-  __shared__ uint32_t s_D;
   __shared__ float s_m;
-  __shared__ int s_top;
+  __shared__ int s_top, s_bad;
   for (int i = threadIdx.x; i < 256; i += NT) T[i] = c_exp_table[i];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n4 = V >> 2;
@@ -360,31 +371,39 @@ __global__ void __launch_bounds__(NT, CPS)
       }
       if (lane == 0) {
         if (b2) {
-          atomicOr(err, ERR_NONFINITE);  // the call fails; outputs stay defined
-          m2 = 0.f;
+          // the call fails; m = +inf sends every code to 8191 (in range) and W is pinned below
+          atomicOr(err, ERR_NONFINITE);
+          m2 = INFINITY;
         }
         s_m = m2;
+        s_bad = b2;
       }
     }
     __syncthreads();
     m = s_m;
-    // pass 2 (L2): histogram of q, lowest index of the maximum
+    // pass 2 (L2): histogram of the codes q < QW0 (the others weigh nothing), lowest index of the maximum
     int topc = 0x7fffffff;
-    for (int i0 = threadIdx.x; i0 < n4; i0 += 2 * NT) {
-      const bool two = i0 + NT < n4;
-      const float4 xa = l4[i0];
-      const float4 xb = two ? l4[i0 + NT] : xa;
-      const float xs[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+    for (int i0 = threadIdx.x; i0 < n4; i0 += 4 * NT) {
+      float4 xv[4];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        if (e < 4 || two) {
-          if (xs[e] == m) topc = min(topc, 4 * (e < 4 ? i0 : i0 + NT) + (e & 3));
-          atomicAdd(&tab[quant_q(m, xs[e])], 1u);
+      for (int k = 0; k < 4; ++k)
+        if (i0 + k * NT < n4) xv[k] = l4[i0 + k * NT];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = i0 + k * NT;
+        if (i < n4) {
+          const float4 x = xv[k];
+          if (x.x == m || x.y == m || x.z == m || x.w == m)
+            topc = min(topc, 4 * i + (x.x == m ? 0 : x.y == m ? 1 : x.z == m ? 2 : 3));
+          const int q0 = quant_q(m, x.x), q1 = quant_q(m, x.y), q2 = quant_q(m, x.z), q3 = quant_q(m, x.w);
+          if (q0 < QW0) atomicAdd(&tab[q0], 1u);
+          if (q1 < QW0) atomicAdd(&tab[q1], 1u);
+          if (q2 < QW0) atomicAdd(&tab[q2], 1u);
+          if (q3 < QW0) atomicAdd(&tab[q3], 1u);
         }
       }
     }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) topc = min(topc, __shfl_xor_sync(0xffffffffu, topc, o));
+    topc = __reduce_min_sync(0xffffffffu, topc);
     if (lane == 0) redi[warp] = topc;
     __syncthreads();
     // per-row sums over the bins (each thread owns bins threadIdx.x + k NT here and below)
@@ -413,6 +432,10 @@ __global__ void __launch_bounds__(NT, CPS)
         tp = min(tp, redi[i]);
       }
       if (tp == 0x7fffffff) tp = 0;  // only for rows flagged non-finite
+      if (s_bad) {                   // all codes 8191 (w = 0): any W >= 2^31 keeps the tables defined
+        tw = 1ull << 31;
+        ta = 0;
+      }
       s_top = tp;
       s_K = (uint64_t)(((unsigned __int128)R << 64) / tw);
       s_W = tw;
@@ -437,47 +460,95 @@ __global__ void __launch_bounds__(NT, CPS)
     if (lane == 0) redi[warp] = (int)fsum;
     __syncthreads();  // the floor table complete
     const uint32_t D = R - __reduce_add_sync(0xffffffffu, lane < NW ? (uint32_t)redi[lane] : 0u);
-    // CDF[v+1] = (v+1) + sum_{u<=v} floor(w_u R / W) + (v >= top ? D : 0), scanned in
-    // block-wide tiles of 4 NT elements (a float4 per thread, from L2); the next
-    // tile's load is issued before this tile's barrier
+    // CDF[v+1] = (v+1) + sum_{u<=v} (floor(w_u R / W) + (u == top ? D : 0)), scanned in
+    // tiles of 4 NT float4s: sub-tile k holds float4s base + k NT + thread, so the
+    // loads coalesce and the four warp scans run side by side; one barrier per tile
     uint32_t* cr = cdf + (size_t)r * (V + 1);
     if (threadIdx.x == 0) cr[0] = 0;
+    // CDF entry 1 + 4 i + e starts a 16-byte quad when e == sh
+    const int sh = (int)((0u - (uint32_t)(reinterpret_cast<uintptr_t>(cr + 1) >> 2)) & 3u);
     uint32_t carry = 0;
-    int buf = 0;
-    float4 xn = threadIdx.x < n4 ? __ldcs(l4 + threadIdx.x) : make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int base = 0; base < n4; base += NT) {
-      const int i = base + threadIdx.x;
-      const float4 x = xn;
-      if (i + NT < n4) xn = __ldcs(l4 + i + NT);
-      uint32_t f0 = 0, f1 = 0, f2 = 0, f3 = 0;
-      if (i < n4) {
-        f0 = tab[quant_q(m, x.x)];
-        f1 = tab[quant_q(m, x.y)];
-        f2 = tab[quant_q(m, x.z)];
-        f3 = tab[quant_q(m, x.w)];
+    int wb = 0;
+    for (int base = 0; base < n4; base += 4 * NT) {
+      uint32_t f[4][4], ts[4], inc[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = base + k * NT + threadIdx.x;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < n4) x = __ldcs(l4 + i);
+        const bool ok = i < n4;
+        f[k][0] = ok ? tab[quant_q(m, x.x)] : 0u;
+        f[k][1] = ok ? tab[quant_q(m, x.y)] : 0u;
+        f[k][2] = ok ? tab[quant_q(m, x.z)] : 0u;
+        f[k][3] = ok ? tab[quant_q(m, x.w)] : 0u;
+        const uint32_t dt = (uint32_t)(top - 4 * i);  // the remainder joins the element at top and every prefix after it
+        if (dt < 4u) {
+          f[k][0] += dt == 0 ? D : 0u;
+          f[k][1] += dt == 1 ? D : 0u;
+          f[k][2] += dt == 2 ? D : 0u;
+          f[k][3] += dt == 3 ? D : 0u;
+        }
+        ts[k] = f[k][0] + f[k][1] + f[k][2] + f[k][3];
+        inc[k] = ts[k];
       }
-      const uint32_t c1 = f0 + f1, c2 = c1 + f2, lsum = c2 + f3;
-      uint32_t inc = lsum;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
-        if (lane >= o) inc += t;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint32_t t = __shfl_up_sync(0xffffffffu, inc[k], o);
+          if (lane >= o) inc[k] += t;
+        }
       }
-      if (lane == 31) wtot[buf][warp] = inc;
+      if (lane == 31) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) wtot[wb][k][warp] = inc[k];
+      }
       __syncthreads();
-      const uint32_t tv = lane < NW ? wtot[buf][lane] : 0u;
-      const uint32_t pre = __reduce_add_sync(0xffffffffu, lane < warp ? tv : 0u);
-      const uint32_t basev = carry + pre + (inc - lsum);
-      carry += __reduce_add_sync(0xffffffffu, tv);
-      buf ^= 1;
-      if (i < n4) {
+      uint32_t run = carry;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t tv = lane < NW ? wtot[wb][k][lane] : 0u;
+        const uint32_t pre = __reduce_add_sync(0xffffffffu, lane < warp ? tv : 0u);
+        const int i = base + k * NT + threadIdx.x;
         const int v = 4 * i;
-        const uint32_t c0 = (uint32_t)v + 1u + basev;
-        __stcs(cr + v + 1, c0 + f0 + (v >= top ? D : 0u));
-        __stcs(cr + v + 2, c0 + 1u + c1 + (v + 1 >= top ? D : 0u));
-        __stcs(cr + v + 3, c0 + 2u + c2 + (v + 2 >= top ? D : 0u));
-        __stcs(cr + v + 4, c0 + 3u + lsum + (v + 3 >= top ? D : 0u));
+        uint32_t o[4];  // o[e] = CDF[v + e + 1]
+        uint32_t c = (uint32_t)v + run + pre + (inc[k] - ts[k]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          c += 1u + f[k][e];
+          o[e] = c;
+        }
+        run += __reduce_add_sync(0xffffffffu, tv);
+        const uint32_t n0 = __shfl_down_sync(0xffffffffu, o[0], 1);
+        const uint32_t n1 = __shfl_down_sync(0xffffffffu, o[1], 1);
+        const uint32_t n2 = __shfl_down_sync(0xffffffffu, o[2], 1);
+        if (i < n4) {
+          uint32_t* dst = cr + 1 + v;
+          if (sh == 0) {
+            __stcs(reinterpret_cast<uint4*>(dst), make_uint4(o[0], o[1], o[2], o[3]));
+          } else {
+            // lanes 0..30 write the quad that starts at their element sh and ends in the
+            // next lane's float4; a warp's first elements and its last lane's tail go singly
+            if (lane == 0) {
+#pragma unroll
+              for (int e = 0; e < 3; ++e)
+                if (e < sh) __stcs(dst + e, o[e]);
+            }
+            if (lane < 31 && i + 1 < n4) {
+              const uint4 qv = sh == 1 ? make_uint4(o[1], o[2], o[3], n0)
+                             : sh == 2 ? make_uint4(o[2], o[3], n0, n1)
+                                       : make_uint4(o[3], n0, n1, n2);
+              __stcs(reinterpret_cast<uint4*>(dst + sh), qv);
+            } else {
+#pragma unroll
+              for (int e = 1; e < 4; ++e)
+                if (e >= sh) __stcs(dst + e, o[e]);
+            }
+          }
+        }
       }
+      carry = run;
+      wb ^= 1;
     }
   }
 }

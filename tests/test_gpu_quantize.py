@@ -58,15 +58,27 @@ def test_quantize_isolated_workload_rows(dev):
     assert np.array_equal(Hq.cpu().numpy(), ref["Hq"].astype(np.int32))
 
 
-def test_quantize_rejects_non_finite(dev):
+@pytest.mark.parametrize("V", [64, 1000, 1001, 5000, 126464])
+def test_quantize_rejects_non_finite(dev, V):
+    """NaN / +inf / -inf among positive and negative logits: EBADINPUT, tables in range, context usable."""
     import torch
     d = dlmz()
-    l = np.zeros((3, 64), dtype=np.float32)
+    l = np.linspace(-5, 5, 6 * V, dtype=np.float32).reshape(6, V)
     l[1, 5] = np.nan
-    W = torch.empty(3, dtype=torch.int64, device="cuda")
-    Hq = torch.empty(3, dtype=torch.int32, device="cuda")
-    d.quantize(ptr(to_dev(l)), 3, 64, 16, 0, ptr(W), 0, ptr(Hq), 0)
+    l[2, V - 1] = np.inf
+    l[3, 0] = -np.inf
+    l[4, [1, V // 2]] = [np.nan, np.inf]
+    P = Q.precision_for_vocab(V)
+    cdf = torch.empty(6, V + 1, dtype=torch.int32, device="cuda")
+    W = torch.empty(6, dtype=torch.int64, device="cuda")
+    Hq = torch.empty(6, dtype=torch.int32, device="cuda")
+    d.quantize(ptr(to_dev(l)), 6, V, P, ptr(cdf), ptr(W), 0, ptr(Hq), 0)
     with pytest.raises(d.DlmzError) as e:
         d.check()
     assert e.value.code == d.EBADINPUT
     d.check()  # flag cleared
+    c = cdf.cpu().numpy().view(np.uint32).astype(np.int64)
+    ref = Q.quantize(l[[0, 5]], P)  # the finite rows are still exact
+    assert np.array_equal(c[[0, 5]], ref["cdf"].astype(np.int64))
+    for i in (1, 2, 3, 4):  # the others stay non-decreasing tables within [0, 2^P]
+        assert c[i, 0] == 0 and c[i, -1] <= (1 << P) and np.all(np.diff(c[i]) >= 0)
