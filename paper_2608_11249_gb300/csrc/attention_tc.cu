@@ -55,7 +55,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT, sP = base + S::P;
   const uint32_t bar = base + S::BARS;
   const uint32_t q_full = bar, v_full = bar + 24, v_empty = bar + 32, s_full = bar + 40, p_ready = bar + 48,
-                 o_done = bar + 56;
+                 o_done = bar + 56, s_free = bar + 96;
   auto k_full = [&](int st) { return st ? bar + 72 : bar + 8; };   // per key stage
   auto k_empty = [&](int st) { return st ? bar + 80 : bar + 16; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -74,6 +74,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(v_empty, 1);
     mbar_init(s_full, 1);
     mbar_init(p_ready, 4 * 32);
+    mbar_init(s_free, 4 * 32);
     mbar_init(o_done, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -143,14 +144,16 @@ __global__ void __launch_bounds__(THREADS, 1)
         issue_s(0);
       }
       for (int j = 0; ok && j < nt; ++j) {
-        if (!mbar_wait_bounded(p_ready, j & 1, &abort_flag, err)) break;
-        t5::fence_after();
+        // S_{j+1} goes as soon as the softmax has S_j in registers, so it runs under P_j's exponentials
         if (j + 1 < nt) {
           const int st1 = (j + 1) & 1;
+          if (!mbar_wait_bounded(s_free, j & 1, &abort_flag, err)) break;
           if (!mbar_wait_bounded(k_full(st1), ((j + 1) >> 1) & 1, &abort_flag, err)) break;
           t5::fence_after();
           issue_s(st1);
         }
+        if (!mbar_wait_bounded(p_ready, j & 1, &abort_flag, err)) break;
+        t5::fence_after();
         if (!mbar_wait_bounded(v_full, j & 1, &abort_flag, err)) break;
         t5::fence_after();
 #pragma unroll
@@ -186,6 +189,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       t5::fence_after();
       uint32_t sr[BK];
       t5::tmem_ld128(tS + lane_off, sr);
+      t5::fence_before();
+      mbar_arrive(s_free);  // S_j is in registers: the MMA warp may overwrite it with S_{j+1}
       float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};  // 4 independent chains
 #pragma unroll
       for (int i = 0; i < BK; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sr[i]));
