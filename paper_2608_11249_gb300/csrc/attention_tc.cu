@@ -1,7 +1,7 @@
 // Bidirectional attention on the 5th-generation tensor cores (Definition 3:
 // every position attends to every position of its window, no mask).
 //
-// CTA = (128 queries, head, window), 6 warps:
+// Persistent CTAs (two per SM) walk work items (128 queries, head, window); 6 warps:
 //   warp 0      TMA: Q once; per key tile of 128: K (2-stage ring, requested
 //               one tile ahead of V) and V^T (keys contiguous, written so by
 //               the QKV epilogue; single buffer).
@@ -43,9 +43,9 @@ struct Smem {
 };
 
 template <int HD>
-__global__ void __launch_bounds__(THREADS, 1)
-    fa_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt, int L, int nh,
-                 int nkv, int d, bf16* __restrict__ out, float scale_log2, int* err) {
+__global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 registers per thread
+    fa_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt, int n_chunks,
+                 int L, int nh, int nkv, int d, bf16* __restrict__ out, float scale_log2, int* err) {
   using S = Smem<HD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -55,17 +55,28 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT, sP = base + S::P;
   const uint32_t bar = base + S::BARS;
   const uint32_t q_full = bar, v_full = bar + 24, v_empty = bar + 32, s_full = bar + 40, p_ready = bar + 48,
-                 o_done = bar + 56, s_free = bar + 96;
+                 o_done = bar + 56, s_free = bar + 96, q_empty = bar + 104, o_free = bar + 112;
   auto k_full = [&](int st) { return st ? bar + 72 : bar + 8; };   // per key stage
   auto k_empty = [&](int st) { return st ? bar + 80 : bar + 16; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int w = blockIdx.z, h = blockIdx.y, q0 = blockIdx.x * BQ;
-  const int g = h / (nh / nkv);
-  const int nt = L / BK;
+  const int nt = L / BK, nqt = L / BQ;
+  // work items (query tile, head, window), query tile fastest; this CTA takes
+  // items blockIdx.x, blockIdx.x + gridDim.x, ...  Tiles are counted across
+  // items (J), so every barrier's phase is a function of J or of the item count.
+  const int items = n_chunks * nh * nqt;
+  const int n_my = blockIdx.x < items ? (items - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  const int total = n_my * nt;
+  auto item_of = [&](int it, int& w, int& h, int& q0) {
+    const int id = (int)blockIdx.x + it * (int)gridDim.x;
+    q0 = (id % nqt) * BQ;
+    h = (id / nqt) % nh;
+    w = id / (nqt * nh);
+  };
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
     mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
     for (int st = 0; st < 2; ++st) {
       mbar_init(k_full(st), 1);
       mbar_init(k_empty(st), 1);
@@ -76,6 +87,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(p_ready, 4 * 32);
     mbar_init(s_free, 4 * 32);
     mbar_init(o_done, 1);
+    mbar_init(o_free, 4 * 32);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) t5::tmem_alloc(smem_u32(&tmem_slot), TMEM_COLS);
@@ -88,38 +100,53 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      const int row0 = w * L;
-      mbar_arrive_expect_tx(q_full, BQ * HD * 2);
-      for (int kb = 0; kb < HD / 64; ++kb) t5::tma_load_2d(sQ + kb * BQ * 128, &tmQK, h * HD + kb * 64, row0 + q0, q_full);
-      uint32_t kpend = 0, kpar[2] = {0, 0}, vp = 0;
-      bool v_pend = false;
-      // K_j is requested before V_{j-1}: K runs one tile ahead through its 2-stage ring
-      for (int j = 0; j <= nt && !abort_flag; ++j) {
-        if (j < nt) {
-          const int st = j & 1;
-          const uint32_t ph = (j >> 1) & 1;
+      uint32_t kpend = 0, kpar0 = 0, kpar1 = 0, vp = 0;
+      bool v_pend = false, q_pend = false;
+      uint32_t qp = 0;
+      // per global tile J: (item's Q when J starts an item), K_J, then V_{J-1};
+      // K runs one tile ahead of V through its 2-stage ring
+      for (int J = 0; J <= total && !abort_flag; ++J) {
+        if (J < total) {
+          const int it = J / nt, j = J % nt;
+          int w, h, q0;
+          item_of(it, w, h, q0);
+          const int g = h / (nh / nkv);
+          if (j == 0) {  // the previous item's last QK^T has read Q
+            if (it > 0 && !mbar_wait_bounded(q_empty, (it - 1) & 1, &abort_flag, err)) break;
+            mbar_arrive_expect_tx(q_full, BQ * HD * 2);
+            for (int kb = 0; kb < HD / 64; ++kb)
+              t5::tma_load_2d(sQ + kb * BQ * 128, &tmQK, h * HD + kb * 64, w * L + q0, q_full);
+            q_pend = true;
+            qp = it & 1;
+          }
+          const int st = J & 1;
+          const uint32_t ph = (J >> 1) & 1;
           if (!mbar_wait_bounded(k_empty(st), ph ^ 1, &abort_flag, err)) break;
           mbar_arrive_expect_tx(k_full(st), BK * HD * 2);
           for (int kb = 0; kb < HD / 64; ++kb)
-            t5::tma_load_2d(sK + st * S::KT + kb * BK * 128, &tmQK, d + g * HD + kb * 64, row0 + j * BK, k_full(st));
+            t5::tma_load_2d(sK + st * S::KT + kb * BK * 128, &tmQK, d + g * HD + kb * 64, w * L + j * BK, k_full(st));
           kpend |= 1u << st;
-          kpar[st] = ph;
+          if (st) kpar1 = ph;
+          else kpar0 = ph;
         }
-        if (j >= 1) {
-          const int jv = j - 1;
-          if (!mbar_wait_bounded(v_empty, (jv & 1) ^ 1, &abort_flag, err)) break;
+        if (J >= 1) {
+          const int Jv = J - 1, it = Jv / nt, j = Jv % nt;
+          int w, h, q0;
+          item_of(it, w, h, q0);
+          const int g = h / (nh / nkv);
+          if (!mbar_wait_bounded(v_empty, (Jv & 1) ^ 1, &abort_flag, err)) break;
           mbar_arrive_expect_tx(v_full, BK * HDP * 2);
           for (int kk = 0; kk < 2; ++kk)
-            t5::tma_load_2d(sVt + kk * HDP * 128, &tmVt, jv * BK + kk * 64, (w * nkv + g) * HDP, v_full);
+            t5::tma_load_2d(sVt + kk * HDP * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HDP, v_full);
           v_pend = true;
-          vp = jv & 1;
+          vp = Jv & 1;
         }
       }
       if (abort_flag) {  // let our own copies land before the CTA can exit
         volatile int never = 0;
-        mbar_wait_bounded(q_full, 0, &never, err, 100000000ull);
-        for (int st = 0; st < 2; ++st)
-          if (kpend & (1u << st)) mbar_wait_bounded(k_full(st), kpar[st], &never, err, 100000000ull);
+        if (q_pend) mbar_wait_bounded(q_full, qp, &never, err, 100000000ull);
+        if (kpend & 1u) mbar_wait_bounded(k_full(0), kpar0, &never, err, 100000000ull);
+        if (kpend & 2u) mbar_wait_bounded(k_full(1), kpar1, &never, err, 100000000ull);
         if (v_pend) mbar_wait_bounded(v_full, vp, &never, err, 100000000ull);
       }
     }
@@ -128,7 +155,13 @@ __global__ void __launch_bounds__(THREADS, 1)
       constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
       constexpr uint32_t ID_O = t5::idesc_f16(BQ, HDP);
       bool issued = false;
-      auto issue_s = [&](int st) {
+      // S_J = Q K_J^T; the first tile of an item waits for that item's Q, the
+      // last one releases Q to the next item's load
+      auto issue_s = [&](int J) -> bool {
+        const int st = J & 1;
+        if (J % nt == 0 && !mbar_wait_bounded(q_full, (J / nt) & 1, &abort_flag, err)) return false;
+        if (!mbar_wait_bounded(k_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
+        t5::fence_after();
         for (int kb = 0; kb < HD / 64; ++kb)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
@@ -136,25 +169,23 @@ __global__ void __launch_bounds__(THREADS, 1)
                          t5::sw128_desc(sK + st * S::KT + kb * BK * 128 + 32 * k), ID_S, (kb | k) != 0);
         t5::commit(s_full);
         t5::commit(k_empty(st));
+        if (J % nt == nt - 1) t5::commit(q_empty);
         issued = true;
+        return true;
       };
-      bool ok = mbar_wait_bounded(q_full, 0, &abort_flag, err) && mbar_wait_bounded(k_full(0), 0, &abort_flag, err);
-      if (ok) {
-        t5::fence_after();
-        issue_s(0);
-      }
-      for (int j = 0; ok && j < nt; ++j) {
-        // S_{j+1} goes as soon as the softmax has S_j in registers, so it runs under P_j's exponentials
-        if (j + 1 < nt) {
-          const int st1 = (j + 1) & 1;
-          if (!mbar_wait_bounded(s_free, j & 1, &abort_flag, err)) break;
-          if (!mbar_wait_bounded(k_full(st1), ((j + 1) >> 1) & 1, &abort_flag, err)) break;
-          t5::fence_after();
-          issue_s(st1);
+      bool ok = total == 0 || issue_s(0);
+      for (int J = 0; ok && J < total; ++J) {
+        const int it = J / nt, j = J % nt;
+        // S_{J+1} goes as soon as the softmax has S_J in registers, so it runs under P_J's exponentials
+        // (across items too: the next item's first QK^T overlaps this item's last softmax and epilogue)
+        if (J + 1 < total) {
+          if (!mbar_wait_bounded(s_free, J & 1, &abort_flag, err)) break;
+          if (!issue_s(J + 1)) break;
         }
-        if (!mbar_wait_bounded(p_ready, j & 1, &abort_flag, err)) break;
-        t5::fence_after();
-        if (!mbar_wait_bounded(v_full, j & 1, &abort_flag, err)) break;
+        if (!mbar_wait_bounded(p_ready, J & 1, &abort_flag, err)) break;
+        if (!mbar_wait_bounded(v_full, J & 1, &abort_flag, err)) break;
+        // the first PV of an item overwrites O: the softmax warps must have read the previous item's O
+        if (j == 0 && it > 0 && !mbar_wait_bounded(o_free, (it - 1) & 1, &abort_flag, err)) break;
         t5::fence_after();
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk)
@@ -179,33 +210,26 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int r = q * 32 + lane;  // query row within the tile (= TMEM lane)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     float m = -INFINITY;
-    bool ok = true;
-    for (int j = 0; j < nt; ++j) {
+    for (int J = 0; J < total; ++J) {
+      const int j = J % nt;
       // waits are made warp-uniform: tcgen05.ld/st below are warp-collective
-      if (!__all_sync(0xffffffffu, mbar_wait_bounded(s_full, j & 1, &abort_flag, err))) {
-        ok = false;
-        break;
-      }
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(s_full, J & 1, &abort_flag, err))) break;
       t5::fence_after();
       uint32_t sr[BK];
       t5::tmem_ld128(tS + lane_off, sr);
       t5::fence_before();
-      mbar_arrive(s_free);  // S_j is in registers: the MMA warp may overwrite it with S_{j+1}
+      mbar_arrive(s_free);  // S_J is in registers: the MMA warp may overwrite it with S_{J+1}
       float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};  // 4 independent chains
 #pragma unroll
       for (int i = 0; i < BK; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sr[i]));
       float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       mx *= scale_log2;
-      if (j > 0) {  // PV_{j-1} done: P buffer free, O stable
-        if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (j - 1) & 1, &abort_flag, err))) {
-          ok = false;
-          break;
-        }
-        t5::fence_after();
-      }
-      if (j == 0) {
+      if (j == 0) {  // P buffer and O were released by this item's predecessor's epilogue
         m = mx;
       } else {
+        // PV_{J-1} done: P buffer free, O stable
+        if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (J - 1) & 1, &abort_flag, err))) break;
+        t5::fence_after();
         const bool need = mx > m + RESCALE_THRESHOLD;
         float f = 1.0f;
         if (need) {
@@ -241,25 +265,30 @@ __global__ void __launch_bounds__(THREADS, 1)
       t5::fence_proxy_async();
       t5::fence_before();
       mbar_arrive(p_ready);
-    }
-    if (__all_sync(0xffffffffu, ok && mbar_wait_bounded(o_done, (nt - 1) & 1, &abort_flag, err))) {
-      t5::fence_after();
-      uint32_t o[HD], lsum[16];
-      t5::tmem_ld64(tO + lane_off, o);
-      t5::tmem_ld16(tO + lane_off + HD, lsum);
-      const float inv = 1.0f / __uint_as_float(lsum[0]);
-      bf16* dst = out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
-      uint4* d4 = reinterpret_cast<uint4*>(dst);
+      if (j == nt - 1) {  // this item's epilogue: O / l -> bf16
+        if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, J & 1, &abort_flag, err))) break;
+        t5::fence_after();
+        uint32_t o[HD], lsum[16];
+        t5::tmem_ld64(tO + lane_off, o);
+        t5::tmem_ld16(tO + lane_off + HD, lsum);
+        t5::fence_before();
+        mbar_arrive(o_free);  // O is in registers: the next item's first PV may overwrite it
+        int w, h, q0;
+        item_of(J / nt, w, h, q0);
+        const float inv = 1.0f / __uint_as_float(lsum[0]);
+        bf16* dst = out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
+        uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-      for (int t = 0; t < HD / 8; ++t) {
-        uint32_t u[4];
+        for (int t = 0; t < HD / 8; ++t) {
+          uint32_t u[4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          __nv_bfloat162 p2 = __floats2bfloat162_rn(__uint_as_float(o[8 * t + 2 * e]) * inv,
-                                                    __uint_as_float(o[8 * t + 2 * e + 1]) * inv);
-          u[e] = *reinterpret_cast<uint32_t*>(&p2);
+          for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 p2 = __floats2bfloat162_rn(__uint_as_float(o[8 * t + 2 * e]) * inv,
+                                                      __uint_as_float(o[8 * t + 2 * e + 1]) * inv);
+            u[e] = *reinterpret_cast<uint32_t*>(&p2);
+          }
+          d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
         }
-        d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
       }
     }
   }
@@ -312,9 +341,13 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
     DLMZ_CUDA_TRY(cudaFuncSetAttribute(fat::fa_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM));
     attr = true;
   }
-  dim3 grid(L / fat::BQ, nh, n_chunks);
+  // persistent: two CTAs per SM (shared memory and 256 TMEM columns each) walk the work items
+  const int64_t items = (int64_t)n_chunks * nh * (L / fat::BQ);
+  if (items > 0x7fffffff) return DLMZ_EINVAL;
+  const int grid = items < 2 * num_sms() ? (int)items : 2 * num_sms();
   ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
-  fat::fa_tc_kernel<64><<<grid, fat::THREADS, SM, s>>>(mqk, mvt, L, nh, nkv, d, out, scale_log2, device_error_word());
+  fat::fa_tc_kernel<64><<<grid, fat::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
+                                                      device_error_word());
   return launch_status();
 }
 

@@ -21,6 +21,7 @@ MODELS = [
     (1, 256, 8, 1, 384, 300, "bf16", 77, 2, 0, 77),      # 8:1 GQA hd 32, LM head on CUDA cores (V = 300)
     (2, 256, 4, 2, 256, 256, "bf16", 256, 2, 0, 256),    # tcgen05 attention (L % 128 == 0, hd 64), GQA 2:1
     (2, 512, 8, 8, 512, 256, "bf16", 512, 2, 128, 128),  # byte-workload head shape: L 512, hd 64, block rows
+    (1, 256, 4, 2, 256, 256, "bf16", 256, 80, 0, 256),   # 640 attention work items: persistent CTAs take 2-3 each
 ]
 
 
