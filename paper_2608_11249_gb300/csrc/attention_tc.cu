@@ -224,18 +224,25 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       for (int i = 0; i < BK; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sr[i]));
       float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       mx *= scale_log2;
+      // the running max first (P needs only m); P_J is computed in registers while PV_{J-1} may still run
+      float f = 1.0f;
+      bool need = false;
       if (j == 0) {  // P buffer and O were released by this item's predecessor's epilogue
         m = mx;
-      } else {
+      } else if (mx > m + RESCALE_THRESHOLD) {
+        need = true;
+        f = t5::ex2(m - mx);
+        m = mx;
+      }
+      // P = 2^(s * scale - m) as f16 pairs (in place of S)
+#pragma unroll
+      for (int c = 0; c < BK / 2; ++c)
+        sr[c] = t5::ex2_f16x2(t5::pack_f16x2(fmaf(__uint_as_float(sr[2 * c]), scale_log2, -m),
+                                             fmaf(__uint_as_float(sr[2 * c + 1]), scale_log2, -m)));
+      if (j > 0) {
         // PV_{J-1} done: P buffer free, O stable
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (J - 1) & 1, &abort_flag, err))) break;
         t5::fence_after();
-        const bool need = mx > m + RESCALE_THRESHOLD;
-        float f = 1.0f;
-        if (need) {
-          f = t5::ex2(m - mx);
-          m = mx;
-        }
         if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
 #pragma unroll 1
           for (int c = 0; c < HDP / 16; ++c) {
@@ -247,19 +254,12 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
           }
         }
       }
-      // P = 2^(s * scale - m) as f16 pairs, 16-byte chunks of 8 keys, 128B-swizzled rows
+      // 16-byte chunks of 8 keys, 128B-swizzled rows
 #pragma unroll
       for (int cc = 0; cc < BK / 8; ++cc) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-          const int i = cc * 8 + 2 * t;
-          pk[t] = t5::ex2_f16x2(t5::pack_f16x2(fmaf(__uint_as_float(sr[i]), scale_log2, -m),
-                                               fmaf(__uint_as_float(sr[i + 1]), scale_log2, -m)));
-        }
         const uint32_t a = sP + (cc >> 3) * BQ * 128 + r * 128 + (((cc & 7) ^ (r & 7)) << 4);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(pk[0]), "r"(pk[1]), "r"(pk[2]),
-                     "r"(pk[3])
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(sr[4 * cc]), "r"(sr[4 * cc + 1]),
+                     "r"(sr[4 * cc + 2]), "r"(sr[4 * cc + 3])
                      : "memory");
       }
       t5::fence_proxy_async();
