@@ -20,7 +20,9 @@ Diffusion LMs for Lossless Compression"):
                    entropy scores (Sec. 3.3 entropy equation; rANS-style
                    statistical coding of Sec. 2.1 / Sec. 4).
 * ``selector``  -- commitment schedules of Sec. 3.3 (max-confidence top-k in
-                   left-to-right blocks, entropy threshold with minimum m).
+                   left-to-right blocks, entropy threshold with minimum m,
+                   uniform block, progressive).
+* ``context``   -- initial context of Sec. 3.4 (contiguous, random).
 * ``coder``     -- range coder with minimal termination (statistical coding,
                    Sec. 2.1 and Sec. 4 "Implementation Details").
 * ``container`` -- compressed-file header (Sec. 3.3 last paragraph, Sec. 4).

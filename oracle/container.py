@@ -7,9 +7,10 @@ Details") are stored so the decompressor replays every decision.  Layout
 
     off size field
       0   4  magic "DLMZ"
-      4   2  version (1)
+      4   2  version (1; 2 when the windows carry an initial context)
       6   1  P, CDF precision bits
-      7   1  policy kind (0 = top-k confidence, 1 = entropy)
+      7   1  policy kind (0 = top-k confidence, 1 = entropy, 2 = uniform block,
+             3 = progressive; for 3 the block field holds r in 16.16 fixed point)
       8   8  model fingerprint (FNV-1a 64 of the model configuration)
      16   4  V (vocabulary size)
      20   4  chunk_len (the window w)
@@ -20,7 +21,13 @@ Details") are stored so the decompressor replays every decision.  Layout
      56   4  n_chunks
      60   4  checksum: CRC-32 (IEEE) of the little-endian CRC-32s of the
              windows' input bytes, window by window
-     64   -  n_chunks LEB128 varints: bit length of each chunk's stream
+   version 2 only (initial context, Sec. 3.4: the visible symbols are stored):
+     64   4  context kind (1 = contiguous, 2 = random)
+     68   4  c, context symbols per window
+     72   8  seed of the random positions
+     80   -  the context symbols, window by window (min(c, window length) each,
+             ascending position; 1 byte each when V <= 256, else u32)
+      -   -  n_chunks LEB128 varints: bit length of each chunk's stream
       -   -  streams, chunk by chunk, ceil(bits / 8) bytes each
 
 Parity: pinned by parse(write(h)) == h and by the corruption tests
@@ -32,8 +39,10 @@ from dataclasses import dataclass
 
 MAGIC = b"DLMZ"
 VERSION = 1
+VERSION_CONTEXT = 2
 HEADER = struct.Struct("<4sHBBQIIIIIIIIQII")
-assert HEADER.size == 64
+EXT = struct.Struct("<IIQ")
+assert HEADER.size == 64 and EXT.size == 16
 
 
 class ContainerError(Exception):
@@ -77,6 +86,10 @@ class Header:
     n_symbols: int
     n_chunks: int
     crc32: int
+    ctx_kind: int = 0
+    ctx_c: int = 0
+    ctx_seed: int = 0
+    ctx_data: bytes = b""
 
 
 def varint(n):
@@ -107,9 +120,12 @@ def read_varint(buf, pos):
 
 def write(h, streams):
     """``streams``: list of (bits, bytes) per chunk."""
+    ver = VERSION_CONTEXT if h.ctx_c else VERSION
     out = bytearray(HEADER.pack(
-        MAGIC, VERSION, h.P, h.kind, h.fingerprint, h.vocab, h.chunk_len, h.batch_chunks, h.k,
+        MAGIC, ver, h.P, h.kind, h.fingerprint, h.vocab, h.chunk_len, h.batch_chunks, h.k,
         h.block, h.tau_q, h.k_min, h.k_max, h.n_symbols, h.n_chunks, h.crc32))
+    if ver == VERSION_CONTEXT:
+        out += EXT.pack(h.ctx_kind, h.ctx_c, h.ctx_seed) + h.ctx_data
     for bits, _ in streams:
         out += varint(bits)
     for bits, data in streams:
@@ -125,7 +141,7 @@ def read(buf):
     f = HEADER.unpack_from(buf, 0)
     if f[0] != MAGIC:
         raise ContainerError("bad magic")
-    if f[1] != VERSION:
+    if f[1] not in (VERSION, VERSION_CONTEXT):
         raise ContainerError("unsupported version")
     h = Header(*f[2:])
     if h.chunk_len == 0 and h.n_symbols:
@@ -134,6 +150,20 @@ def read(buf):
     if h.n_chunks != exp_chunks:
         raise ContainerError("chunk count does not match the symbol count")
     pos = HEADER.size
+    if f[1] == VERSION_CONTEXT:
+        if len(buf) < pos + EXT.size:
+            raise ContainerError("truncated header")
+        h.ctx_kind, h.ctx_c, h.ctx_seed = EXT.unpack_from(buf, pos)
+        pos += EXT.size
+        if h.ctx_kind not in (1, 2) or h.ctx_c == 0:
+            raise ContainerError("bad context")
+        sb = 1 if h.vocab <= 256 else 4
+        full, tail = divmod(h.n_symbols, h.chunk_len)
+        nb = sb * (full * min(h.ctx_c, h.chunk_len) + min(h.ctx_c, tail))
+        if pos + nb > len(buf):
+            raise ContainerError("truncated context")
+        h.ctx_data = bytes(buf[pos:pos + nb])
+        pos += nb
     lens = []
     for _ in range(h.n_chunks):
         n, pos = read_varint(buf, pos)

@@ -1,6 +1,6 @@
 """Symbol commitment schedules (oracle side), Sec. 3.3.
 
-Two schedules are on the path:
+Four schedules:
 
 * ``TOPK_CONF`` -- max-confidence top-k inside left-to-right blocks.  The
   paper builds on LLaDA (Sec. 1, Sec. 4) and the workloads here commit k
@@ -16,7 +16,19 @@ Two schedules are on the path:
   An optional cap ``k_max`` (0 = none) keeps only the k_max lowest-entropy
   positions of the selection.
 
-Both are deterministic given their hyper-parameters, so the decoder replays
+* ``UNIFORM`` -- uniform block schedule (Sec. 3.3, paragraph 1): with K = ``k``
+  steps, u = floor(n / K) symbols are committed per step in contiguous
+  left-to-right order (n = masked positions of the window).  Reading: K is
+  capped at n, and the last step commits the remainder n - (K - 1) u, so
+  exactly K forwards cover the window.
+* ``PROGRESSIVE`` -- geometric schedule (Sec. 3.3, paragraph 2): u_k =
+  round(u_1 r^(k-1)) symbols left to right, u_1 = ``k``.  Reading: r is
+  carried as a 16.16 fixed-point integer ``growth_q16`` and the sequence as
+  x_1 = u_1 2^16, x_(k+1) = floor(x_k r_q / 2^16) (exact integers, so every
+  implementation agrees); u_k = max(1, floor((x_k + 2^15) / 2^16)), and the
+  last step takes what remains.  r = 1 gives u_k = u_1 (uniform steps).
+
+All are deterministic given their hyper-parameters, so the decoder replays
 them from the header alone (Sec. 3.3, last paragraph).  Within a step the
 committed symbols are coded in ascending position.
 
@@ -30,6 +42,8 @@ import numpy as np
 
 TOPK_CONF = 0
 ENTROPY = 1
+UNIFORM = 2
+PROGRESSIVE = 3
 
 
 @dataclass(frozen=True)
@@ -40,6 +54,32 @@ class Policy:
     tau_bits: float = 0.0
     k_min: int = 1
     k_max: int = 0
+    growth_q16: int = 65536
+
+
+def schedule_sizes(n, policy):
+    """u_1, ..., u_K of the left-to-right schedules for n masked positions (sum = n)."""
+    if n <= 0:
+        return []
+    if policy.kind == UNIFORM:
+        K = min(policy.k, n)
+        u = n // K
+        return [u] * (K - 1) + [n - (K - 1) * u]
+    if policy.kind == PROGRESSIVE:
+        sizes, rem, x = [], n, policy.k << 16
+        while rem > 0:
+            u = max(1, (x + (1 << 15)) >> 16)
+            u = min(u, rem)
+            sizes.append(u)
+            rem -= u
+            x = min((x * policy.growth_q16) >> 16, n << 16)
+        return sizes
+    raise ValueError("not a left-to-right schedule")
+
+
+def leftmost(masked, count):
+    """The ``count`` leftmost masked positions."""
+    return np.flatnonzero(np.asarray(masked, dtype=bool))[:count]
 
 
 def active_block(masked, block):
