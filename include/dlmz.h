@@ -81,17 +81,32 @@ DLMZ_API uint64_t dlmz_model_fingerprint(const dlmz_model* m);
 /* Copy the model configuration into *cfg. */
 DLMZ_API int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg);
 
-/* ---- commitment schedule (Sec. 3.3) ---------------------------------- */
-#define DLMZ_TOPK_CONF 0u /* k most confident masked positions of the leftmost incomplete block */
-#define DLMZ_ENTROPY 1u   /* all masked positions with entropy <= tau; at least k_min, at most k_max */
+/* ---- commitment schedule (Sec. 3.3) and initial context (Sec. 3.4) ---- */
+#define DLMZ_TOPK_CONF 0u   /* k most confident masked positions of the leftmost incomplete block */
+#define DLMZ_ENTROPY 1u     /* all masked positions with entropy <= tau; at least k_min, at most k_max */
+#define DLMZ_UNIFORM 2u     /* uniform block (Sec. 3.3 par. 1): K = k steps of floor(n/K) masked positions,
+                               left to right, the last step taking the remainder */
+#define DLMZ_PROGRESSIVE 3u /* progressive (Sec. 3.3 par. 2): u_k = round(u_1 r^(k-1)) left to right,
+                               u_1 = k, r = growth_q16 / 65536 (exact 16.16 fixed-point sequence) */
+
+#define DLMZ_CONTEXT_NONE 0u       /* every position starts masked (c = 0) */
+#define DLMZ_CONTEXT_CONTIGUOUS 1u /* the first c symbols of each window stay visible */
+#define DLMZ_CONTEXT_RANDOM 2u     /* c positions per window drawn from context_seed (SplitMix64,
+                                      partial Fisher-Yates); symbols stored raw in the file */
 
 typedef struct {
   uint32_t kind;
-  uint32_t k;       /* TOPK_CONF: positions per step (>= 1) */
-  uint32_t block;   /* TOPK_CONF: block length; 0 = the whole window */
-  float tau_bits;   /* ENTROPY: threshold tau in bits (entropy base 2) */
-  uint32_t k_min;   /* ENTROPY: m, minimum positions per step (>= 1) */
-  uint32_t k_max;   /* ENTROPY: cap per step; 0 = no cap */
+  uint32_t k;            /* TOPK_CONF: positions per step; UNIFORM: K steps; PROGRESSIVE: u_1 (all >= 1) */
+  uint32_t block;        /* TOPK_CONF: block length; 0 = the whole window */
+  float tau_bits;        /* ENTROPY: threshold tau in bits (entropy base 2) */
+  uint32_t k_min;        /* ENTROPY: m, minimum positions per step (>= 1) */
+  uint32_t k_max;        /* ENTROPY: cap per step; 0 = no cap */
+  uint32_t growth_q16;   /* PROGRESSIVE: growth ratio r in 16.16 fixed point, 1 .. 64 * 65536 */
+  uint32_t context;      /* DLMZ_CONTEXT_*: initial context of every window (compress only; the
+                            decompressor reads it from the file) */
+  uint32_t context_c;    /* c, symbols per window left visible (0 exactly when context is NONE) */
+  uint32_t reserved;     /* 0 */
+  uint64_t context_seed; /* RANDOM: seed of the positions */
 } dlmz_k_policy;
 
 /* ---- whole-file API, host buffers ------------------------------------ */
@@ -101,7 +116,9 @@ typedef struct {
  * malloc'd container of *out_bytes bytes, released with dlmz_free; on error
  * *out is NULL.  batch_chunks = 0 picks the default batch (<= 1024 windows
  * per forward batch, bounded by device memory); the value used is stored in
- * the header so the decoder replays the same batches. */
+ * the header so the decoder replays the same batches.  The policy's context
+ * fields select an initial context (Sec. 3.4): those symbols are stored raw
+ * in the file and not coded. */
 DLMZ_API int dlmz_compress(const dlmz_model* m, const void* in, size_t in_bytes, uint32_t chunk_len,
                   const dlmz_k_policy* policy, uint8_t** out, size_t* out_bytes);
 DLMZ_API int dlmz_compress_ex(const dlmz_model* m, const void* in, size_t in_bytes, uint32_t chunk_len,
@@ -199,7 +216,10 @@ DLMZ_API int dlmz_coder_load_decoder(dlmz_coder* c, const uint8_t* d_bytes, cons
  * order into each window's stream (encoder: true symbols from d_symbols
  * [n_chunks x L]; decoder: decoded) and reveal them in d_state.
  * d_committed (may be NULL) receives the number of positions committed per
- * window [n_chunks]. */
+ * window [n_chunks].  For UNIFORM and PROGRESSIVE the caller runs the
+ * schedule: policy->k is this step's u_k, and the step commits the u_k
+ * leftmost masked positions inside the rows (the logits' scores are not used).
+ * The policy's context fields are ignored here (the caller sets d_state). */
 DLMZ_API int dlmz_encode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits,
                      uint32_t row0, uint32_t rows_per_chunk, const int32_t* d_symbols,
                      int32_t* d_state, int32_t* d_committed, void* stream);

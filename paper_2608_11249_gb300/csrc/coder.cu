@@ -4,8 +4,9 @@
 //
 // Selection: every schedule here commits the n smallest candidates under
 // (key, position): top-k confidence (key W, n = min(k, #candidates) of the
-// leftmost incomplete block) and the entropy threshold (key H_q, n = #{H_q <=
-// tau} or m if fewer, capped by k_max).  A CTA per window ranks its
+// leftmost incomplete block), the entropy threshold (key H_q, n = #{H_q <=
+// tau} or m if fewer, capped by k_max), and the left-to-right uniform-block and
+// progressive schedules (no key: the n = u_k leftmost masked positions).  A CTA per window ranks its
 // candidates, so the result does not depend on thread order.
 //
 // Range coder: 64-bit low/range, 16-bit output units stored big-endian,
@@ -33,7 +34,7 @@ __global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask
   int nv = 0, nb = 0;
   for (int i = threadIdx.x; i < rpc; i += blockDim.x) {
     const bool ok = state ? state[(size_t)c * L + row0 + i] == mask_id : true;
-    const uint64_t key = (uint64_t)(int64_t)keys[(size_t)c * rpc + i];
+    const uint64_t key = keys ? (uint64_t)(int64_t)keys[(size_t)c * rpc + i] : 0;  // null: position order
     skey[i] = key;
     valid[i] = ok;
     nv += ok;

@@ -2,9 +2,9 @@
 //
 // compress: the input is cut into non-overlapping windows of chunk_len
 // symbols (w, Sec. 4); windows of equal length run as a batch.  Each batch
-// starts fully masked (c = 0) and repeats forward -> quantise -> select ->
-// code -> reveal until every position is committed (coverage sum u_k = n,
-// Sec. 3.3).  Each window owns one range-coder stream.  decompress replays
+// starts masked -- fully, or with c context symbols per window left visible
+// (Sec. 3.4) -- and repeats forward -> quantise -> select -> code -> reveal
+// until every masked position is committed (coverage sum u_k = n, Sec. 3.3).  Each window owns one range-coder stream.  decompress replays
 // the same batches and schedule from the header alone (Sec. 3.3, last
 // paragraph): the selection of a step never depends on the symbols that
 // step codes, so the decoder sees the same logits at every step.
@@ -14,10 +14,15 @@
 // tau_q, k_min, k_max, n_symbols, n_chunks, checksum), one LEB128 varint per
 // window with its stream's bit length, then the streams (ceil(bits/8) bytes
 // each).  The checksum is the CRC-32 (IEEE) of the windows' CRC-32s.
+// Version 2 (a context, Sec. 3.4) extends the header by 16 bytes (context
+// kind, c, seed) and puts the context symbols (min(c, window) per window,
+// ascending position, 1 or 4 bytes each) between the header and the lengths.
+// For the progressive schedule the block field holds r in 16.16 fixed point.
 #include <math.h>
 #include <stdlib.h>
 #include <string.h>
 
+#include <algorithm>
 #include <vector>
 
 #include "coder.cuh"
@@ -132,6 +137,35 @@ __global__ void sum_i32_kernel(const int32_t* v, int n, unsigned long long* out)
   }
 }
 
+// Initial context (Sec. 3.4) of windows [0, nc) (each L long): the ce context
+// positions of window w (pos[w*ce + i], or i itself when pos is null) take their
+// symbol -- from `symbols` when compressing (also written to out_syms, sb bytes
+// little-endian each, for the file) or from the file's bytes when decompressing
+// (a symbol >= V there marks the file corrupt and is replaced by 0).
+__global__ void context_kernel(int32_t* state, int nc, int L, int ce, const int32_t* pos, const int32_t* symbols,
+                               const uint8_t* file_syms, uint8_t* out_syms, int sb, int V, int* err) {
+  const int64_t n = (int64_t)nc * ce;
+  for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < n; idx += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t w = idx / ce;
+    const int p = pos ? pos[idx] : (int)(idx % ce);
+    int32_t v;
+    if (symbols) {
+      v = symbols[w * L + p];
+    } else {
+      uint32_t u = 0;
+      for (int b = 0; b < sb; ++b) u |= (uint32_t)file_syms[idx * sb + b] << (8 * b);
+      if (u >= (uint32_t)V) {
+        atomicOr(err, ERR_CORRUPT);
+        u = 0;
+      }
+      v = (int32_t)u;
+    }
+    state[w * L + p] = v;
+    if (out_syms)
+      for (int b = 0; b < sb; ++b) out_syms[idx * sb + b] = (uint8_t)((uint32_t)v >> (8 * b));
+  }
+}
+
 static unsigned grid_for(int64_t n, int threads = 256) {
   int64_t b = (n + threads - 1) / threads;
   if (b < 1) b = 1;
@@ -147,6 +181,80 @@ static uint32_t crc32_host(const uint8_t* p, size_t n) {
   }
   return ~crc;
 }
+
+// ---- left-to-right schedules (Sec. 3.3, paragraphs 1-2) --------------------------------
+// Uniform block: K = min(k, n) steps of floor(n / K), the last taking the remainder.
+// Progressive: x_1 = u_1 2^16, x_(k+1) = floor(x_k r_q / 2^16) (capped at n 2^16, which
+// changes no step), u_k = max(1, floor((x_k + 2^15) / 2^16)), at most what remains.
+static std::vector<int> schedule_sizes(int n, const dlmz_k_policy& p) {
+  std::vector<int> u;
+  if (n <= 0) return u;
+  if (p.kind == DLMZ_UNIFORM) {
+    const int K = (int64_t)p.k < n ? (int)p.k : n;
+    const int q = n / K;
+    u.assign(K - 1, q);
+    u.push_back(n - (K - 1) * q);
+    return u;
+  }
+  unsigned __int128 x = (unsigned __int128)p.k << 16;
+  const unsigned __int128 cap = (unsigned __int128)n << 16;
+  for (int rem = n; rem > 0;) {
+    unsigned __int128 v = (x + (1u << 15)) >> 16;
+    if (v < 1) v = 1;
+    const int take = v < (unsigned __int128)rem ? (int)v : rem;
+    u.push_back(take);
+    rem -= take;
+    x = (x * p.growth_q16) >> 16;
+    if (x > cap) x = cap;
+  }
+  return u;
+}
+
+// ---- initial context positions (Sec. 3.4) ----------------------------------------------
+// Random: partial Fisher-Yates (Durstenfeld) of [0, n) with output i of the
+// SplitMix64 stream (Steele, Lea & Flood 2014) whose state is output `window` of
+// the stream seeded by `seed`; output j of a stream with state s is mix(s + (j+1) gamma).
+static uint64_t sm64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+static constexpr uint64_t SM64_GAMMA = 0x9E3779B97F4A7C15ull;
+
+static int context_count(const dlmz_k_policy& p, int n) {
+  return p.context == DLMZ_CONTEXT_NONE ? 0 : ((int64_t)p.context_c < n ? (int)p.context_c : n);
+}
+
+static void context_positions(const dlmz_k_policy& p, int n, uint64_t window, int32_t* out) {
+  const int ce = context_count(p, n);
+  if (p.context == DLMZ_CONTEXT_CONTIGUOUS) {
+    for (int i = 0; i < ce; ++i) out[i] = i;
+    return;
+  }
+  if (ce == 0) return;
+  const uint64_t st = sm64_mix(p.context_seed + (window + 1) * SM64_GAMMA);
+  std::vector<int32_t> slot(n);
+  for (int i = 0; i < n; ++i) slot[i] = i;
+  for (int i = 0; i < ce; ++i) {
+    const uint64_t o = sm64_mix(st + (uint64_t)(i + 1) * SM64_GAMMA);
+    const int j = i + (int)(o % (uint64_t)(n - i));
+    const int32_t t = slot[i];
+    slot[i] = slot[j];
+    slot[j] = t;
+  }
+  std::sort(slot.begin(), slot.begin() + ce);
+  for (int i = 0; i < ce; ++i) out[i] = slot[i];
+}
+
+// Context of one batch: ce positions per window (host and device copies).
+struct BatchContext {
+  int ce = 0;                   // context symbols per window of this batch
+  std::vector<int32_t> pos;     // nc x ce, ascending per window (empty when contiguous)
+  const int32_t* d_pos = nullptr;
+  const uint8_t* file_syms = nullptr;  // decompress: the batch's symbols in the file
+  uint8_t* out_syms = nullptr;         // compress: where the batch's symbols go
+  int sb = 1;                          // bytes per stored symbol
+};
 
 // ---- per-batch step state ---------------------------------------------------------
 struct StepBufs {
@@ -170,7 +278,7 @@ struct StepBufs {
 };
 
 static int kcap_for(const dlmz_k_policy& p, int rpc) {
-  int k = p.kind == DLMZ_TOPK_CONF ? (int)p.k : (p.k_max ? (int)p.k_max : rpc);
+  int k = p.kind != DLMZ_ENTROPY ? (int)p.k : (p.k_max ? (int)p.k_max : rpc);
   if (p.kind == DLMZ_ENTROPY && (int)p.k_min > k) k = (int)p.k_min;
   return k < rpc ? k : rpc;
 }
@@ -187,9 +295,10 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
   DLMZ_TRY(sb.ensure(rows, 1, nc, kcap));
   DLMZ_TRY(quantize_rows(logits, rows, V, P, nullptr, sb.W.as<uint64_t>(), nullptr, sb.Hq.as<int32_t>(),
                          sb.top.as<int32_t>(), sb.mx.as<float>(), s));
-  if (pol.kind == DLMZ_TOPK_CONF)
-    DLMZ_TRY(select_rows<uint64_t>(state, nc, L, V, row0, rpc, sb.W.as<uint64_t>(), 0, (int)pol.k, 0, 0, 0, kcap,
-                                   sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), s));
+  if (pol.kind != DLMZ_ENTROPY)  // left-to-right schedules: the k leftmost masked rows (keys ignored)
+    DLMZ_TRY(select_rows<uint64_t>(state, nc, L, V, row0, rpc,
+                                   pol.kind == DLMZ_TOPK_CONF ? sb.W.as<uint64_t>() : nullptr, 0, (int)pol.k, 0, 0,
+                                   0, kcap, sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), s));
   else
     DLMZ_TRY(select_rows<int32_t>(state, nc, L, V, row0, rpc, sb.Hq.as<int32_t>(), 1, 0, tau_q_of(pol.tau_bits),
                                   (int)pol.k_min, (int)pol.k_max, kcap, sb.sel_count.as<int32_t>(),
@@ -222,7 +331,11 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
 
 static int validate_policy(const dlmz_k_policy* p) {
   if (!p) return DLMZ_EINVAL;
-  if (p->kind == DLMZ_TOPK_CONF) return p->k >= 1 ? DLMZ_OK : DLMZ_EINVAL;
+  if (p->context > DLMZ_CONTEXT_RANDOM || (p->context == DLMZ_CONTEXT_NONE) != (p->context_c == 0) || p->reserved)
+    return DLMZ_EINVAL;
+  if (p->kind == DLMZ_TOPK_CONF || p->kind == DLMZ_UNIFORM) return p->k >= 1 ? DLMZ_OK : DLMZ_EINVAL;
+  if (p->kind == DLMZ_PROGRESSIVE)
+    return p->k >= 1 && p->growth_q16 >= 1 && p->growth_q16 <= (64u << 16) ? DLMZ_OK : DLMZ_EINVAL;
   if (p->kind == DLMZ_ENTROPY) {
     if (p->k_min < 1) return DLMZ_EINVAL;
     if (p->k_max && p->k_max < p->k_min) return DLMZ_EINVAL;
@@ -242,26 +355,79 @@ static uint64_t cap_bytes_for(uint32_t L, int P) {
 // One batch of nc windows of length Lb through all steps.
 static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int nc, int Lb, const int32_t* symbols,
                      int32_t* state, CoderState* cst, uint8_t* ebytes, uint64_t cap_bytes, const uint8_t* in_bytes,
-                     const uint64_t* in_off, const uint32_t* in_bits, bool decode, cudaStream_t s) {
+                     const uint64_t* in_off, const uint32_t* in_bits, bool decode, const BatchContext& bx,
+                     cudaStream_t s) {
   const int V = (int)m->cfg.vocab, P = precision_for(m->cfg.vocab);
+  const int ce = bx.ce;
   fill_i32<<<grid_for((int64_t)nc * Lb), 256, 0, s>>>(state, (int64_t)nc * Lb, V);
   DLMZ_TRY(launch_status());
+  if (ce > 0) {
+    context_kernel<<<grid_for((int64_t)nc * ce), 256, 0, s>>>(state, nc, Lb, ce, bx.d_pos, decode ? nullptr : symbols,
+                                                             bx.file_syms, decode ? nullptr : bx.out_syms, bx.sb, V,
+                                                             device_error_word());
+    DLMZ_TRY(launch_status());
+  }
   if (decode) DLMZ_TRY(coder_load(cst, nc, in_bytes, in_off, in_bits, s));
   else DLMZ_TRY(coder_reset(cst, nc, s));
+  // context positions of window w inside [a, b)
+  auto ctx_in = [&](int w, int a, int b) -> int {
+    if (ce == 0) return 0;
+    if (bx.pos.empty()) return std::max(0, std::min(b, ce) - a);  // contiguous: [0, ce)
+    const int32_t* p = bx.pos.data() + (size_t)w * ce;
+    return (int)(std::lower_bound(p, p + ce, b) - std::lower_bound(p, p + ce, a));
+  };
   if (pol.kind == DLMZ_TOPK_CONF) {
     const int B = pol.block ? (int)pol.block : Lb;
     for (int b0 = 0; b0 < Lb; b0 += B) {
       const int Bl = B < Lb - b0 ? B : Lb - b0;
+      // steps for this block: the window with the most masked positions in it decides
+      int most = 0;
+      for (int w = 0; w < (bx.pos.empty() ? 1 : nc); ++w) most = std::max(most, Bl - ctx_in(w, b0, b0 + Bl));
+      const int steps = (most + (int)pol.k - 1) / (int)pol.k;
+      if (steps == 0) continue;
       DLMZ_TRY(sb.ensure((size_t)nc * Bl, V, nc, kcap_for(pol, Bl)));
-      for (int rem = Bl; rem > 0; rem -= ((int)pol.k < rem ? (int)pol.k : rem)) {
+      for (int t = 0; t < steps; ++t) {
         DLMZ_TRY(model_forward(m, state, nc, Lb, b0, Bl, sb.logits.as<float>(), s));
         DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, pol, b0, Bl, symbols, state, cst, ebytes,
                           cap_bytes, in_bytes, in_off, in_bits, decode, nullptr, s));
       }
     }
+  } else if (pol.kind == DLMZ_UNIFORM || pol.kind == DLMZ_PROGRESSIVE) {
+    // every window has n = Lb - ce masked positions, so one schedule serves the batch; step k
+    // commits masked positions [t, t + u_k) of each window, whose rows span [lo, hi) over the batch
+    const int n = Lb - ce;
+    const std::vector<int> sizes = schedule_sizes(n, pol);
+    std::vector<int32_t> masked;  // nc x n masked positions, ascending (random context only)
+    if (!bx.pos.empty()) {
+      masked.resize((size_t)nc * n);
+      for (int w = 0; w < nc; ++w) {
+        const int32_t* p = bx.pos.data() + (size_t)w * ce;
+        int q = 0, j = 0;
+        for (int x = 0; x < Lb; ++x) {
+          if (j < ce && p[j] == x) ++j;
+          else masked[(size_t)w * n + q++] = x;
+        }
+      }
+    }
+    auto mpos = [&](int w, int t) -> int { return masked.empty() ? ce + t : masked[(size_t)w * n + t]; };
+    int t = 0;
+    for (const int u : sizes) {
+      int lo = Lb, hi = 0;
+      for (int w = 0; w < (masked.empty() ? 1 : nc); ++w) {
+        lo = std::min(lo, mpos(w, t));
+        hi = std::max(hi, mpos(w, t + u - 1) + 1);
+      }
+      dlmz_k_policy sp = pol;
+      sp.k = (uint32_t)u;
+      DLMZ_TRY(sb.ensure((size_t)nc * (hi - lo), V, nc, kcap_for(sp, hi - lo)));
+      DLMZ_TRY(model_forward(m, state, nc, Lb, lo, hi - lo, sb.logits.as<float>(), s));
+      DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, sp, lo, hi - lo, symbols, state, cst, ebytes,
+                        cap_bytes, in_bytes, in_off, in_bits, decode, nullptr, s));
+      t += u;
+    }
   } else {
     DLMZ_TRY(sb.ensure((size_t)nc * Lb, V, nc, kcap_for(pol, Lb)));
-    int64_t remaining = (int64_t)nc * Lb;
+    int64_t remaining = (int64_t)nc * (Lb - ce);
     for (int64_t step = 0; remaining > 0; ++step) {
       if (step > (int64_t)Lb) return DLMZ_ECORRUPT;  // every step commits >= 1 per live window
       DLMZ_TRY(model_forward(m, state, nc, Lb, 0, Lb, sb.logits.as<float>(), s));
@@ -281,10 +447,10 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
 
 struct PipeWs {
   StepBufs sb;
-  DevBuf symbols, state, cst, staging, bits, crcs, offsets, hin, hout;
+  DevBuf symbols, state, cst, staging, bits, crcs, offsets, hin, hout, ctxpos, ctxsyms;
   void release() {
     sb.release(); symbols.release(); state.release(); cst.release(); staging.release(); bits.release();
-    crcs.release(); offsets.release(); hin.release(); hout.release();
+    crcs.release(); offsets.release(); hin.release(); hout.release(); ctxpos.release(); ctxsyms.release();
   }
 };
 
@@ -310,6 +476,16 @@ static int default_batch(const dlmz_model* m, uint32_t L, uint32_t n_chunks) {
 struct Header {
   uint32_t P, kind, vocab, chunk_len, batch_chunks, k, block, tau_q, k_min, k_max, n_chunks, crc;
   uint64_t fingerprint, n_symbols;
+  uint32_t ctx_kind = 0, ctx_c = 0;  // version 2: initial context (Sec. 3.4)
+  uint64_t ctx_seed = 0;
+  size_t size() const { return ctx_c ? 80 : 64; }
+  // bytes of the stored context symbols (after the header)
+  uint64_t ctx_bytes() const {
+    if (!ctx_c || !chunk_len) return 0;
+    const uint64_t full = n_symbols / chunk_len, tail = n_symbols % chunk_len;
+    const uint64_t per = ctx_c < chunk_len ? ctx_c : chunk_len;
+    return (full * per + (ctx_c < tail ? ctx_c : tail)) * (vocab > 256 ? 4 : 1);
+  }
 };
 
 static void put32(uint8_t* p, uint32_t v) { for (int i = 0; i < 4; ++i) p[i] = (uint8_t)(v >> (8 * i)); }
@@ -319,7 +495,7 @@ static uint64_t get64(const uint8_t* p) { uint64_t v = 0; for (int i = 0; i < 8;
 
 static void write_header(uint8_t* o, const Header& h) {
   memcpy(o, "DLMZ", 4);
-  o[4] = 1;
+  o[4] = h.ctx_c ? 2 : 1;
   o[5] = 0;
   o[6] = (uint8_t)h.P;
   o[7] = (uint8_t)h.kind;
@@ -335,11 +511,17 @@ static void write_header(uint8_t* o, const Header& h) {
   put64(o + 48, h.n_symbols);
   put32(o + 56, h.n_chunks);
   put32(o + 60, h.crc);
+  if (h.ctx_c) {
+    put32(o + 64, h.ctx_kind);
+    put32(o + 68, h.ctx_c);
+    put64(o + 72, h.ctx_seed);
+  }
 }
 
+// o holds the first min(n, 80) bytes of the file
 static int read_header(const uint8_t* o, size_t n, Header& h) {
   if (n < 64) return DLMZ_ECORRUPT;
-  if (memcmp(o, "DLMZ", 4) || o[4] != 1 || o[5] != 0) return DLMZ_ECORRUPT;
+  if (memcmp(o, "DLMZ", 4) || (o[4] != 1 && o[4] != 2) || o[5] != 0) return DLMZ_ECORRUPT;
   h.P = o[6];
   h.kind = o[7];
   h.fingerprint = get64(o + 8);
@@ -357,6 +539,33 @@ static int read_header(const uint8_t* o, size_t n, Header& h) {
   if (h.chunk_len == 0 && h.n_symbols) return DLMZ_ECORRUPT;
   const uint64_t exp = h.chunk_len ? (h.n_symbols + h.chunk_len - 1) / h.chunk_len : 0;
   if (exp != h.n_chunks) return DLMZ_ECORRUPT;
+  if (o[4] == 2) {
+    if (n < 80) return DLMZ_ECORRUPT;
+    h.ctx_kind = get32(o + 64);
+    h.ctx_c = get32(o + 68);
+    h.ctx_seed = get64(o + 72);
+    if ((h.ctx_kind != DLMZ_CONTEXT_CONTIGUOUS && h.ctx_kind != DLMZ_CONTEXT_RANDOM) || h.ctx_c == 0)
+      return DLMZ_ECORRUPT;
+  }
+  return DLMZ_OK;
+}
+
+// The batch's context: positions (host + device) and where its symbols are in the file.
+static int batch_context(const dlmz_k_policy& pol, int c0, int nc, int Lb, int sb, DevBuf& dpos, uint64_t sym_off,
+                         const uint8_t* file, uint8_t* out, cudaStream_t s, BatchContext& bx) {
+  bx = BatchContext{};
+  bx.ce = context_count(pol, Lb);
+  bx.sb = sb;
+  if (bx.ce == 0) return DLMZ_OK;
+  bx.file_syms = file ? file + sym_off * sb : nullptr;
+  bx.out_syms = out ? out + sym_off * sb : nullptr;
+  if (pol.context == DLMZ_CONTEXT_RANDOM) {
+    bx.pos.resize((size_t)nc * bx.ce);
+    for (int w = 0; w < nc; ++w) context_positions(pol, Lb, (uint64_t)(c0 + w), bx.pos.data() + (size_t)w * bx.ce);
+    DLMZ_TRY(dpos.ensure(bx.pos.size() * 4));
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(dpos.p, bx.pos.data(), bx.pos.size() * 4, cudaMemcpyHostToDevice, s));
+    bx.d_pos = dpos.as<int32_t>();
+  }
   return DLMZ_OK;
 }
 
@@ -411,14 +620,28 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
     window_crc_kernel<<<(n_chunks + 127) / 128, 128, 0, s>>>(d_in, in_bytes, wbytes, n_chunks, w.crcs.as<uint32_t>());
     DLMZ_TRY(launch_status());
   }
+  Header h{};
+  h.ctx_kind = pol->context_c ? pol->context : 0;
+  h.ctx_c = pol->context_c;
+  h.ctx_seed = pol->context_seed;
+  h.chunk_len = L;
+  h.n_symbols = n_sym;
+  h.vocab = V;
+  const uint64_t ctx_bytes = h.ctx_bytes();
+  const int sbytes = tok ? 4 : 1;
+  DLMZ_TRY(w.ctxsyms.ensure(ctx_bytes + 16));
+  const uint64_t ce_full = (uint64_t)context_count(*pol, (int)L);
   for (const BatchPlan& b : plan_batches(n_sym, L, bc)) {
     const int64_t nsym_b = (int64_t)b.nc * b.L;
     symbols_in_kernel<<<grid_for(nsym_b), 256, 0, s>>>(d_in, (int64_t)b.c0 * L, nsym_b, tok, (int)V,
                                                        w.symbols.as<int32_t>(), device_error_word());
     DLMZ_TRY(launch_status());
     uint8_t* eb = w.staging.as<uint8_t>() + (size_t)b.c0 * cap;
+    BatchContext bx;
+    DLMZ_TRY(batch_context(*pol, b.c0, b.nc, b.L, sbytes, w.ctxpos, (uint64_t)b.c0 * ce_full, nullptr,
+                           w.ctxsyms.as<uint8_t>(), s, bx));
     DLMZ_TRY(run_batch(m, w.sb, *pol, b.nc, b.L, w.symbols.as<int32_t>(), w.state.as<int32_t>(),
-                       w.cst.as<CoderState>(), eb, cap, nullptr, nullptr, nullptr, false, s));
+                       w.cst.as<CoderState>(), eb, cap, nullptr, nullptr, nullptr, false, bx, s));
     DLMZ_TRY(coder_finish(w.cst.as<CoderState>(), b.nc, eb, cap, w.bits.as<uint32_t>() + b.c0, nullptr, nullptr, s));
   }
   DLMZ_TRY(check_device(s));
@@ -429,26 +652,23 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
   }
   std::vector<uint8_t> crcb((size_t)n_chunks * 4);
   for (int c = 0; c < n_chunks; ++c) put32(crcb.data() + 4 * c, crcs[c]);
-  Header h{};
   h.P = P;
   h.kind = pol->kind;
-  h.vocab = V;
-  h.chunk_len = L;
   h.batch_chunks = bc;
   h.k = pol->k;
-  h.block = pol->block;
+  h.block = pol->kind == DLMZ_PROGRESSIVE ? pol->growth_q16 : pol->block;
   h.tau_q = (uint32_t)tau_q_of(pol->tau_bits);
   h.k_min = pol->k_min;
   h.k_max = pol->k_max;
   h.n_chunks = n_chunks;
   h.crc = crc32_host(crcb.data(), crcb.size());
   h.fingerprint = m->fingerprint;
-  h.n_symbols = n_sym;
-  std::vector<uint8_t> head(64);
+  std::vector<uint8_t> head(h.size());
   write_header(head.data(), h);
-  for (int c = 0; c < n_chunks; ++c) put_varint(head, bits[c]);
+  std::vector<uint8_t> lens;
+  for (int c = 0; c < n_chunks; ++c) put_varint(lens, bits[c]);
   std::vector<uint64_t> offs(n_chunks);
-  uint64_t pos = head.size();
+  uint64_t pos = head.size() + ctx_bytes + lens.size();
   for (int c = 0; c < n_chunks; ++c) {
     offs[c] = pos;
     pos += (bits[c] + 7) / 8;
@@ -457,6 +677,10 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
   if (pos > out_cap) return DLMZ_ECAPACITY;
   if (!d_out) return DLMZ_EINVAL;
   DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out, head.data(), head.size(), cudaMemcpyHostToDevice, s));
+  if (ctx_bytes)
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out + head.size(), w.ctxsyms.p, ctx_bytes, cudaMemcpyDeviceToDevice, s));
+  if (!lens.empty())
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out + head.size() + ctx_bytes, lens.data(), lens.size(), cudaMemcpyHostToDevice, s));
   if (n_chunks) {
     DLMZ_CUDA_TRY(cudaMemcpyAsync(w.offsets.p, offs.data(), (size_t)n_chunks * 8, cudaMemcpyHostToDevice, s));
     gather_streams_kernel<<<n_chunks, 128, 0, s>>>(w.staging.as<uint8_t>(), cap, w.bits.as<uint32_t>(),
@@ -471,15 +695,27 @@ static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes
   if (!m || !d_in || !out_bytes) return DLMZ_EINVAL;
   DLMZ_TRY(device_error_word() ? DLMZ_OK : DLMZ_ENOMEM);
   DLMZ_TRY(clear_device_error(s));
-  uint8_t hb[64];
+  uint8_t hb[80];
   if (in_bytes < 64) return DLMZ_ECORRUPT;
-  DLMZ_CUDA_TRY(cudaMemcpy(hb, d_in, 64, cudaMemcpyDeviceToHost));
+  DLMZ_CUDA_TRY(cudaMemcpy(hb, d_in, in_bytes < 80 ? in_bytes : 80, cudaMemcpyDeviceToHost));
   Header h{};
   DLMZ_TRY(read_header(hb, in_bytes, h));
   if (h.fingerprint != m->fingerprint) return DLMZ_EMODEL;
   if (h.vocab != m->cfg.vocab || (int)h.P != precision_for(h.vocab)) return DLMZ_ECORRUPT;
-  dlmz_k_policy pol{h.kind, h.k, h.block, (float)(h.tau_q / 65536.0), h.k_min, h.k_max};
+  dlmz_k_policy pol{};
+  pol.kind = h.kind;
+  pol.k = h.k;
+  pol.block = h.kind == DLMZ_PROGRESSIVE ? 0 : h.block;
+  pol.growth_q16 = h.kind == DLMZ_PROGRESSIVE ? h.block : 65536;
+  pol.tau_bits = (float)(h.tau_q / 65536.0);
+  pol.k_min = h.k_min;
+  pol.k_max = h.k_max;
+  pol.context = h.ctx_kind;
+  pol.context_c = h.ctx_c;
+  pol.context_seed = h.ctx_seed;
   if (validate_policy(&pol) != DLMZ_OK) return DLMZ_ECORRUPT;
+  const uint64_t hsize = h.size(), ctx_bytes = h.ctx_bytes();
+  if (hsize + ctx_bytes > in_bytes) return DLMZ_ECORRUPT;
   if (h.n_symbols && h.batch_chunks == 0) return DLMZ_ECORRUPT;
   const int tok = h.vocab > 256;
   const uint64_t out_need = h.n_symbols * (tok ? 4 : 1);
@@ -487,9 +723,10 @@ static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes
   if (out_need > out_cap) return DLMZ_ECAPACITY;
   if (out_need && !d_out) return DLMZ_EINVAL;
   const int n_chunks = (int)h.n_chunks;
-  const size_t vmax = (size_t)n_chunks * 5 < in_bytes - 64 ? (size_t)n_chunks * 5 : in_bytes - 64;
+  const uint64_t lens0 = hsize + ctx_bytes;  // the length table follows the context symbols
+  const size_t vmax = (size_t)n_chunks * 5 < in_bytes - lens0 ? (size_t)n_chunks * 5 : in_bytes - lens0;
   std::vector<uint8_t> vb(vmax);
-  if (vmax) DLMZ_CUDA_TRY(cudaMemcpy(vb.data(), d_in + 64, vmax, cudaMemcpyDeviceToHost));
+  if (vmax) DLMZ_CUDA_TRY(cudaMemcpy(vb.data(), d_in + lens0, vmax, cudaMemcpyDeviceToHost));
   std::vector<uint32_t> bits(n_chunks);
   size_t p = 0;
   for (int c = 0; c < n_chunks; ++c) {
@@ -506,7 +743,7 @@ static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes
     bits[c] = (uint32_t)v;
   }
   std::vector<uint64_t> offs(n_chunks);
-  uint64_t pos = 64 + p;
+  uint64_t pos = lens0 + p;
   for (int c = 0; c < n_chunks; ++c) {
     offs[c] = pos;
     pos += (bits[c] + 7) / 8;
@@ -525,9 +762,13 @@ static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes
   const size_t bl = (size_t)(bc < n_chunks ? bc : (n_chunks ? n_chunks : 1)) * L;
   DLMZ_TRY(w.state.ensure(bl * 4));
   DLMZ_TRY(w.cst.ensure((size_t)bc * sizeof(CoderState)));
+  const uint64_t ce_full = (uint64_t)context_count(pol, (int)L);
   for (const BatchPlan& b : plan_batches(h.n_symbols, L, bc)) {
+    BatchContext bx;
+    DLMZ_TRY(batch_context(pol, b.c0, b.nc, b.L, tok ? 4 : 1, w.ctxpos, (uint64_t)b.c0 * ce_full, d_in + hsize,
+                           nullptr, s, bx));
     DLMZ_TRY(run_batch(m, w.sb, pol, b.nc, b.L, nullptr, w.state.as<int32_t>(), w.cst.as<CoderState>(), nullptr, 0,
-                       d_in, w.offsets.as<uint64_t>() + b.c0, w.bits.as<uint32_t>() + b.c0, true, s));
+                       d_in, w.offsets.as<uint64_t>() + b.c0, w.bits.as<uint32_t>() + b.c0, true, bx, s));
     const int64_t nsym_b = (int64_t)b.nc * b.L;
     symbols_out_kernel<<<grid_for(nsym_b), 256, 0, s>>>(w.state.as<int32_t>(), (int64_t)b.c0 * L, nsym_b, tok, d_out);
     DLMZ_TRY(launch_status());

@@ -20,7 +20,8 @@ lib = ctypes.CDLL(_LIB_PATH)
 
 OK, EINVAL, EBADINPUT, ECORRUPT, EMODEL, ENOMEM, ECUDA, ETIMEOUT, ECAPACITY = 0, -1, -2, -3, -4, -5, -6, -7, -8
 FP32, BF16 = 0, 1
-TOPK_CONF, ENTROPY = 0, 1
+TOPK_CONF, ENTROPY, UNIFORM, PROGRESSIVE = 0, 1, 2, 3
+CONTEXT_NONE, CONTEXT_CONTIGUOUS, CONTEXT_RANDOM = 0, 1, 2
 
 
 class DlmzError(RuntimeError):
@@ -37,7 +38,8 @@ class ModelConfig(Structure):
 
 class KPolicy(Structure):
     _fields_ = [("kind", c_uint32), ("k", c_uint32), ("block", c_uint32), ("tau_bits", c_float),
-                ("k_min", c_uint32), ("k_max", c_uint32)]
+                ("k_min", c_uint32), ("k_max", c_uint32), ("growth_q16", c_uint32), ("context", c_uint32),
+                ("context_c", c_uint32), ("reserved", c_uint32), ("context_seed", c_uint64)]
 
 
 class Profile(Structure):
@@ -94,8 +96,9 @@ def strerror(code):
     return lib.dlmz_strerror(code).decode()
 
 
-def policy(kind=TOPK_CONF, k=1, block=0, tau_bits=0.0, k_min=1, k_max=0):
-    return KPolicy(kind, k, block, tau_bits, k_min, k_max)
+def policy(kind=TOPK_CONF, k=1, block=0, tau_bits=0.0, k_min=1, k_max=0, growth_q16=65536,
+           context=CONTEXT_NONE, context_c=0, context_seed=0):
+    return KPolicy(kind, k, block, tau_bits, k_min, k_max, growth_q16, context, context_c, 0, context_seed)
 
 
 class Model:

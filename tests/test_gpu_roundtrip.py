@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 
 from oracle import container as OC
+from oracle import context as OX
 from oracle import model as OM
 from oracle import pipeline as OP
 from oracle import selector as S
@@ -50,6 +51,65 @@ def test_roundtrip_and_size_vs_oracle(dev, ci):
     w = OM.Weights(OM.ModelConfig(*spec, seed=40 + ci))
     oblob = OP.compress(w, data, L, opol)
     assert abs(len(blob) - len(oblob)) <= 0.005 * len(oblob) + 8, (len(blob), len(oblob))
+
+
+LR_CASES = [
+    # model, data kind, n, chunk_len, oracle policy, context (kind, c, seed), batch_chunks
+    ((1, 32, 2, 2, 64, 256, "f32"), "bytes", 1500, 512, S.Policy(kind=S.UNIFORM, k=16), (OX.NONE, 0, 0), 0),
+    ((2, 256, 4, 4, 256, 256, "bf16"), "bytes", 1100, 256, S.Policy(kind=S.PROGRESSIVE, k=2, growth_q16=98304),
+     (OX.RANDOM, 8, 5), 3),
+    ((1, 64, 4, 2, 128, 5000, "f32"), "tokens", 300, 100, S.Policy(kind=S.UNIFORM, k=7), (OX.CONTIGUOUS, 5, 0), 0),
+    ((2, 256, 4, 4, 256, 256, "bf16"), "bytes", 600, 200, S.Policy(kind=S.TOPK_CONF, k=8, block=64),
+     (OX.RANDOM, 16, 9), 2),
+    ((2, 256, 4, 4, 256, 256, "bf16"), "bytes", 600, 200, S.Policy(kind=S.ENTROPY, tau_bits=6.0, k_min=2, k_max=16),
+     (OX.CONTIGUOUS, 3, 0), 2),
+    ((1, 32, 2, 2, 64, 256, "f32"), "bytes", 700, 64, S.Policy(kind=S.PROGRESSIVE, k=1, growth_q16=2 << 16),
+     (OX.RANDOM, 100, 3), 0),  # c > window: whole windows stored as context
+]
+
+
+@pytest.mark.parametrize("ci", range(len(LR_CASES)))
+def test_schedules_and_context_vs_oracle(dev, ci):
+    """Uniform/progressive schedules (Sec. 3.3) and initial context (Sec. 3.4): round trip, the stored
+    context symbols bit for bit, and the container size against the oracle's own compression."""
+    d = dlmz()
+    spec, kind, n, L, opol, ctx, bc = LR_CASES[ci]
+    m = _model(d, spec, 60 + ci)
+    data = _data(kind, n, spec[5])
+    pol = d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max, opol.growth_q16,
+                   ctx[0], ctx[1], ctx[2])
+    blob = m.compress(data, L, pol, bc)
+    assert m.decompress(blob) == data
+    h, streams = OC.read(blob)
+    assert (h.ctx_kind, h.ctx_c, h.ctx_seed) == (ctx if ctx[1] else (0, 0, 0))
+    sym = np.frombuffer(data, dtype=np.uint8 if kind == "bytes" else "<u4").astype(np.int64)
+    want = []
+    for c in range(h.n_chunks):
+        win = sym[c * L:(c + 1) * L]
+        want.append(win[OX.positions(ctx[0], ctx[1], ctx[2], win.size, c)])
+    want = np.concatenate(want) if want else np.zeros(0, dtype=np.int64)
+    assert h.ctx_data == (want.astype(np.uint8).tobytes() if kind == "bytes" else want.astype("<u4").tobytes())
+    w = OM.Weights(OM.ModelConfig(*spec, seed=60 + ci))
+    oblob = OP.compress(w, data, L, opol, context=ctx)
+    assert abs(len(blob) - len(oblob)) <= 0.005 * len(oblob) + 8, (len(blob), len(oblob))
+
+
+def test_bad_schedule_and_context_rejected(dev):
+    d = dlmz()
+    m = _model(d, (1, 32, 2, 2, 64, 256, "f32"), 1)
+    for pol in (d.policy(d.UNIFORM, 0), d.policy(d.PROGRESSIVE, 1, growth_q16=0),
+                d.policy(d.PROGRESSIVE, 1, growth_q16=(64 << 16) + 1), d.policy(d.TOPK_CONF, 2, context=d.CONTEXT_RANDOM),
+                d.policy(d.TOPK_CONF, 2, context=7, context_c=1), d.policy(d.TOPK_CONF, 2, context_c=3)):
+        with pytest.raises(d.DlmzError) as e:
+            m.compress(b"abcdef", 4, pol)
+        assert e.value.code == d.EINVAL
+    blob = m.compress(b"abcdefgh", 4, d.policy(d.UNIFORM, 2, context=d.CONTEXT_RANDOM, context_c=2, context_seed=1))
+    # bad context kind, truncated extension, an edited context symbol (the checksum catches it)
+    for bad in (blob[:64] + b"\x09" + blob[65:], blob[:79], blob[:80] + bytes([blob[80] ^ 1]) + blob[81:]):
+        with pytest.raises(d.DlmzError) as e:
+            m.decompress(bad)
+        assert e.value.code == d.ECORRUPT
+    d.check()
 
 
 def test_edge_inputs(dev):
