@@ -143,7 +143,7 @@ __device__ __forceinline__ void epi_load_aux(EpiAux& a, int c, int lane, int row
                                                          col0 + (lane & 7) * 4)
                       : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-  } else if constexpr (EPI == EPI_ROPE_BF16) {  // small, L1-resident table: loaded for the current chunk
+  } else if constexpr (EPI == EPI_ROPE_BF16) {  // this lane's (cos, sin) pairs: 4 rows x 4 rotation pairs
     const int col = n0 + c * 32 + 8 * (lane & 3);
     if (col < ep.rope_cols) {
       const int half = ep.head_dim >> 1;
@@ -190,12 +190,20 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
   float rowsum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   EpiAux cur, nxt;
   if constexpr (EPI == EPI_RESID_F32) epi_load_aux<EPI>(cur, c0, lane, row0, M, n0, ep);
+  // RoPE: a warp takes every other chunk (c = half, half + 2, ...), so with head_dim 64 all its
+  // chunks rotate the same pairs and the (cos, sin) table is loaded once per tile
+  int rope_t = -1;
 #pragma unroll 1
-  for (int c = c0; c < c0 + NCH; ++c) {
+  for (int ci = 0; ci < NCH; ++ci) {
+    const int c = EPI == EPI_ROPE_BF16 ? half + 2 * ci : c0 + ci;
     if constexpr (EPI == EPI_RESID_F32) {
-      if (c + 1 < c0 + NCH) epi_load_aux<EPI>(nxt, c + 1, lane, row0, M, n0, ep);
+      if (ci + 1 < NCH) epi_load_aux<EPI>(nxt, c + 1, lane, row0, M, n0, ep);
     } else if constexpr (EPI == EPI_ROPE_BF16) {
-      epi_load_aux<EPI>(cur, c, lane, row0, M, n0, ep);
+      const int t = (n0 + c * 32) % ep.head_dim;
+      if (t != rope_t && n0 + c * 32 < ep.rope_cols) {
+        epi_load_aux<EPI>(cur, c, lane, row0, M, n0, ep);
+        rope_t = t;
+      }
     }
     float v[32];
     tmem_ld32(tbase + c * 32, v);
