@@ -25,6 +25,7 @@ Diffusion LMs for Lossless Compression"):
 * ``context``   -- initial context of Sec. 3.4 (contiguous, random).
 * ``coder``     -- range coder with minimal termination (statistical coding,
                    Sec. 2.1 and Sec. 4 "Implementation Details").
+* ``rans``      -- rANS coder (64-bit state, 32-bit words), the paper's coder.
 * ``container`` -- compressed-file header (Sec. 3.3 last paragraph, Sec. 4).
 * ``pipeline``  -- the iterative pipeline S^(k+1) = f_theta(S^(k)) of
                    Sec. 3.2, compress and decompress.

@@ -7,7 +7,8 @@ Details") are stored so the decompressor replays every decision.  Layout
 
     off size field
       0   4  magic "DLMZ"
-      4   2  version (1; 2 when the windows carry an initial context)
+      4   1  version (1; 2 when the windows carry an initial context)
+      5   1  coder (0 = range coder, 1 = rANS)
       6   1  P, CDF precision bits
       7   1  policy kind (0 = top-k confidence, 1 = entropy, 2 = uniform block,
              3 = progressive; for 3 the block field holds r in 16.16 fixed point)
@@ -40,7 +41,7 @@ from dataclasses import dataclass
 MAGIC = b"DLMZ"
 VERSION = 1
 VERSION_CONTEXT = 2
-HEADER = struct.Struct("<4sHBBQIIIIIIIIQII")
+HEADER = struct.Struct("<4sBBBBQIIIIIIIIQII")
 EXT = struct.Struct("<IIQ")
 assert HEADER.size == 64 and EXT.size == 16
 
@@ -86,6 +87,7 @@ class Header:
     n_symbols: int
     n_chunks: int
     crc32: int
+    coder: int = 0
     ctx_kind: int = 0
     ctx_c: int = 0
     ctx_seed: int = 0
@@ -122,7 +124,7 @@ def write(h, streams):
     """``streams``: list of (bits, bytes) per chunk."""
     ver = VERSION_CONTEXT if h.ctx_c else VERSION
     out = bytearray(HEADER.pack(
-        MAGIC, ver, h.P, h.kind, h.fingerprint, h.vocab, h.chunk_len, h.batch_chunks, h.k,
+        MAGIC, ver, h.coder, h.P, h.kind, h.fingerprint, h.vocab, h.chunk_len, h.batch_chunks, h.k,
         h.block, h.tau_q, h.k_min, h.k_max, h.n_symbols, h.n_chunks, h.crc32))
     if ver == VERSION_CONTEXT:
         out += EXT.pack(h.ctx_kind, h.ctx_c, h.ctx_seed) + h.ctx_data
@@ -143,7 +145,9 @@ def read(buf):
         raise ContainerError("bad magic")
     if f[1] not in (VERSION, VERSION_CONTEXT):
         raise ContainerError("unsupported version")
-    h = Header(*f[2:])
+    if f[2] not in (0, 1):
+        raise ContainerError("unknown coder")
+    h = Header(*f[3:], coder=f[2])
     if h.chunk_len == 0 and h.n_symbols:
         raise ContainerError("zero chunk length")
     exp_chunks = (h.n_symbols + h.chunk_len - 1) // h.chunk_len if h.chunk_len else 0

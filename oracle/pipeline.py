@@ -23,8 +23,13 @@ from . import container as C
 from . import context as X
 from . import model as M
 from . import quantizer as Q
+from . import rans
 from . import selector as S
 from .coder import Decoder, Encoder
+
+RANGE, RANS = 0, 1  # statistical coders: range coder, rANS (Sec. 2.1)
+_ENC = {RANGE: Encoder, RANS: rans.Encoder}
+_DEC = {RANGE: Decoder, RANS: rans.Decoder}
 
 
 class BadInput(ValueError):
@@ -70,14 +75,14 @@ def _key(qz, policy):
     return qz["W"] if policy.kind == S.TOPK_CONF else qz["Hq"]
 
 
-def encode_window(symbols, V, logits_fn, policy, P, trace=None, ctx=()):
+def encode_window(symbols, V, logits_fn, policy, P, trace=None, ctx=(), coder=RANGE):
     """Compress one window; return ((bits, bytes), steps).  ``ctx``: context positions."""
     symbols = np.asarray(symbols, dtype=np.int64)
     n = symbols.size
     state = np.full(n, V, dtype=np.int64)
     ctx = np.asarray(ctx, dtype=np.int64)
     state[ctx] = symbols[ctx]
-    enc = Encoder(P)
+    enc = _ENC[coder](P)
     tq = Q.tau_q(policy.tau_bits)
     sizes = S.schedule_sizes(int(np.sum(state == V)), policy) if policy.kind in (S.UNIFORM, S.PROGRESSIVE) else None
     step = 0
@@ -105,10 +110,10 @@ def encode_window(symbols, V, logits_fn, policy, P, trace=None, ctx=()):
     return enc.finish(), step
 
 
-def decode_window(stream, n, V, logits_fn, policy, P, ctx=(), ctx_symbols=()):
+def decode_window(stream, n, V, logits_fn, policy, P, ctx=(), ctx_symbols=(), coder=RANGE):
     """Decompress one window of ``n`` symbols from (bits, bytes)."""
     bits, data = stream
-    dec = Decoder(data, bits, P)
+    dec = _DEC[coder](data, bits, P)
     state = np.full(n, V, dtype=np.int64)
     state[np.asarray(ctx, dtype=np.int64)] = np.asarray(ctx_symbols, dtype=np.int64)
     tq = Q.tau_q(policy.tau_bits)
@@ -137,10 +142,11 @@ def model_logits_fn(wts):
     return lambda step, state, rows: M.forward(wts, state, rows)
 
 
-def compress(wts, data, chunk_len, policy, batch_chunks=1, context=(X.NONE, 0, 0)):
+def compress(wts, data, chunk_len, policy, batch_chunks=1, context=(X.NONE, 0, 0), coder=RANGE):
     """Compress ``data`` with the DLM ``wts``; return the container bytes.
 
     ``context`` = (kind, c, seed): c symbols per window left visible (Sec. 3.4).
+    ``coder``: RANGE or RANS.
     """
     cfg = wts.cfg
     V = cfg.vocab
@@ -160,7 +166,9 @@ def compress(wts, data, chunk_len, policy, batch_chunks=1, context=(X.NONE, 0, 0
         win = sym[c * chunk_len:(c + 1) * chunk_len]
         ctx = X.positions(ckind, cc, cseed, win.size, c)
         ctx_sym.append(win[ctx])
-        (bits, byts), _ = encode_window(win, V, fn, policy, P, ctx=ctx)
+        if coder not in _ENC:
+            raise BadInput("unknown coder")
+        (bits, byts), _ = encode_window(win, V, fn, policy, P, ctx=ctx, coder=coder)
         streams.append((bits, byts))
     block = policy.growth_q16 if policy.kind == S.PROGRESSIVE else policy.block
     h = C.Header(P=P, kind=policy.kind, fingerprint=C.fingerprint(cfg), vocab=V, chunk_len=chunk_len,
@@ -168,7 +176,7 @@ def compress(wts, data, chunk_len, policy, batch_chunks=1, context=(X.NONE, 0, 0
                  tau_q=Q.tau_q(policy.tau_bits), k_min=policy.k_min, k_max=policy.k_max,
                  n_symbols=n, n_chunks=nchunks,
                  crc32=C.window_checksum(bytes(data), chunk_len * (1 if V <= 256 else 4)),
-                 ctx_kind=ckind, ctx_c=cc, ctx_seed=cseed,
+                 coder=coder, ctx_kind=ckind, ctx_c=cc, ctx_seed=cseed,
                  ctx_data=bytes_from_symbols(np.concatenate(ctx_sym) if ctx_sym else [], V))
     return C.write(h, streams)
 
@@ -195,7 +203,7 @@ def decompress(wts, blob):
     for c, st in enumerate(streams):
         n = min(h.chunk_len, h.n_symbols - c * h.chunk_len)
         ctx = X.positions(h.ctx_kind, h.ctx_c, h.ctx_seed, n, c)
-        out.append(decode_window(st, n, cfg.vocab, fn, policy, h.P, ctx, ctx_all[used:used + ctx.size]))
+        out.append(decode_window(st, n, cfg.vocab, fn, policy, h.P, ctx, ctx_all[used:used + ctx.size], h.coder))
         used += ctx.size
     sym = np.concatenate(out) if out else np.zeros(0, dtype=np.int64)
     data = bytes_from_symbols(sym, cfg.vocab)
