@@ -89,6 +89,9 @@ DLMZ_API int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg);
 #define DLMZ_PROGRESSIVE 3u /* progressive (Sec. 3.3 par. 2): u_k = round(u_1 r^(k-1)) left to right,
                                u_1 = k, r = growth_q16 / 65536 (exact 16.16 fixed-point sequence) */
 
+#define DLMZ_CODER_RANGE 0u /* range coder, minimal termination: ideal length + at most ~1 bit per window */
+#define DLMZ_CODER_RANS 1u  /* rANS, 64-bit state, 32-bit words: ideal length + at most 96 bits per window */
+
 #define DLMZ_CONTEXT_NONE 0u       /* every position starts masked (c = 0) */
 #define DLMZ_CONTEXT_CONTIGUOUS 1u /* the first c symbols of each window stay visible */
 #define DLMZ_CONTEXT_RANDOM 2u     /* c positions per window drawn from context_seed (SplitMix64,
@@ -105,7 +108,7 @@ typedef struct {
   uint32_t context;      /* DLMZ_CONTEXT_*: initial context of every window (compress only; the
                             decompressor reads it from the file) */
   uint32_t context_c;    /* c, symbols per window left visible (0 exactly when context is NONE) */
-  uint32_t reserved;     /* 0 */
+  uint32_t coder;        /* DLMZ_CODER_RANGE (default) or DLMZ_CODER_RANS (the paper's rANS, Sec. 2.1) */
   uint64_t context_seed; /* RANDOM: seed of the positions */
 } dlmz_k_policy;
 
@@ -203,6 +206,11 @@ DLMZ_API int dlmz_select_smallest_noalloc(const uint64_t* d_keys, uint32_t group
 typedef struct dlmz_coder dlmz_coder;
 /* Allocate coder state for n_chunks windows of length L with P-bit tables. */
 DLMZ_API int dlmz_coder_create(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, dlmz_coder** out);
+/* As dlmz_coder_create with the statistical coder chosen (DLMZ_CODER_*); the
+ * policies given to its steps must name the same coder (else EINVAL).  rANS
+ * keeps each window's (c, f) pairs until dlmz_coder_finish codes them. */
+DLMZ_API int dlmz_coder_create_ex(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, uint32_t coder,
+                                  dlmz_coder** out);
 DLMZ_API void dlmz_coder_destroy(dlmz_coder* c);
 /* Encoder: reset every stream to the empty state.  Decoder: read stream c
  * from d_bytes + d_offsets[c] (big-endian 16-bit units, d_bits[c] bits long;

@@ -13,6 +13,11 @@
 // renormalisation below 2^48, carries propagated into the emitted units,
 // minimal termination.  The decoder keeps val = code - low and reads units
 // beyond the stream's length as zero (never past its buffer).
+// rANS (the paper's coder, Sec. 2.1): 64-bit state in [2^31, 2^63), 32-bit
+// words; encode x = floor(x/f) 2^P + x mod f + c after emitting the low word
+// when x >= 2^(63-P) f.  Last in, first out: the steps buffer a window's
+// (c, f) pairs and the finish kernel codes them in reverse; the stream is the
+// final state (8 bytes big-endian) then the words in reverse emission order.
 #include "kernels.cuh"
 #include "coder.cuh"
 #include "exp_table.inc"
@@ -126,6 +131,15 @@ __device__ __forceinline__ uint32_t unit_at(const uint8_t* b, uint64_t nbytes, u
   return (hi << 8) | lo;
 }
 
+// big-endian 32-bit word at byte offset o (bytes at or past nbytes read as 0)
+__device__ __forceinline__ uint64_t word_at(const uint8_t* b, uint64_t nbytes, uint64_t o) {
+  uint64_t w = 0;
+  for (int i = 0; i < 4; ++i) w = (w << 8) | (o + i < nbytes ? b[o + i] : 0u);
+  return w;
+}
+
+constexpr uint64_t RANS_L = 1ull << 31;
+
 __device__ __forceinline__ void put_unit(uint8_t* b, uint32_t i, uint32_t u) {
   b[2 * i] = (uint8_t)(u >> 8);
   b[2 * i + 1] = (uint8_t)u;
@@ -231,20 +245,30 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       __syncthreads();
       if (threadIdx.x == 0) {
         CoderState t = st;
-        enc_symbol(t, ebuf, a.cap_bytes / 2, P, s_cs, s_fs, a.err);
+        if (a.rans) {  // buffered; coded in reverse when the window is finished
+          if (t.n_units < (uint32_t)a.pair_cap) a.pairs[(size_t)c * a.pair_cap + t.n_units] = (s_cs << 32) | s_fs;
+          else atomicOr(a.err, ERR_CAPACITY);
+          t.n_units++;
+        } else {
+          enc_symbol(t, ebuf, a.cap_bytes / 2, P, s_cs, s_fs, a.err);
+        }
         st = t;
         a.state[(size_t)c * a.L + pos] = sym;
       }
       __syncthreads();
     } else {
       if (threadIdx.x == 0) {
-        const uint64_t r = st.rng >> P;
-        uint64_t slot = st.low / r;  // decoder keeps val in .low
-        if (slot >= (1ull << P)) {
-          atomicOr(a.err, ERR_CORRUPT);
-          slot = (1ull << P) - 1;
+        if (a.rans) {
+          s_slot = st.low & ((1ull << P) - 1);  // x mod 2^P
+        } else {
+          const uint64_t r = st.rng >> P;
+          uint64_t slot = st.low / r;  // decoder keeps val in .low
+          if (slot >= (1ull << P)) {
+            atomicOr(a.err, ERR_CORRUPT);
+            slot = (1ull << P) - 1;
+          }
+          s_slot = slot;
         }
-        s_slot = slot;
       }
       __syncthreads();
       const uint64_t slot = s_slot;
@@ -266,12 +290,20 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       __syncthreads();
       if (threadIdx.x == 0) {
         CoderState t = st;
-        const uint64_t r = t.rng >> P;
-        t.low -= r * s_cs;
-        t.rng = r * s_fs;
-        while (t.rng < RENORM) {
-          t.low = (t.low << 16) | unit_at(dbuf, dn, t.n_units++);
-          t.rng <<= 16;
+        if (a.rans) {
+          t.low = s_fs * (t.low >> P) + slot - s_cs;
+          if (t.low < RANS_L) {
+            t.low = (t.low << 32) | word_at(dbuf, dn, 8 + 4ull * t.n_units);
+            t.n_units++;
+          }
+        } else {
+          const uint64_t r = t.rng >> P;
+          t.low -= r * s_cs;
+          t.rng = r * s_fs;
+          while (t.rng < RENORM) {
+            t.low = (t.low << 16) | unit_at(dbuf, dn, t.n_units++);
+            t.rng <<= 16;
+          }
         }
         st = t;
         a.state[(size_t)c * a.L + pos] = s_sym;
@@ -303,16 +335,64 @@ __global__ void coder_reset_kernel(CoderState* st, int n) {
 }
 
 __global__ void coder_load_kernel(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets,
-                                  const uint32_t* bits) {
+                                  const uint32_t* bits, int rans) {
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= n) return;
   const uint8_t* b = bytes + (offsets ? offsets[c] : 0);
   const uint64_t nb = (bits[c] + 7) / 8;
   uint64_t v = 0;
-  for (int i = 0; i < 4; ++i) v = (v << 16) | unit_at(b, nb, i);
+  if (rans) {  // the final state of the encoder leads the stream
+    v = (word_at(b, nb, 0) << 32) | word_at(b, nb, 4);
+    st[c].n_units = 0;
+  } else {
+    for (int i = 0; i < 4; ++i) v = (v << 16) | unit_at(b, nb, i);
+    st[c].n_units = 4;
+  }
   st[c].low = v;
   st[c].rng = ~0ull;
-  st[c].n_units = 4;
+}
+
+// rANS: code window c's buffered pairs in reverse.  Words go down from the end
+// of the window's buffer; the state goes below them; the stream is then moved
+// to the front of the buffer.
+__global__ void rans_finish_kernel(CoderState* st, int n, const uint64_t* pairs, int pair_cap, int P, uint8_t* bytes,
+                                   uint64_t cap_bytes, uint32_t* bits_out, uint8_t* out, const uint64_t* offsets,
+                                   int* err) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n) return;
+  uint8_t* buf = bytes + (size_t)c * cap_bytes;
+  const uint32_t np = st[c].n_units < (uint32_t)pair_cap ? st[c].n_units : (uint32_t)pair_cap;
+  const uint64_t* pr = pairs + (size_t)c * pair_cap;
+  uint64_t x = RANS_L, pos = cap_bytes & ~3ull;  // next word ends at pos
+  bool ok = true;
+  for (int i = (int)np - 1; i >= 0; --i) {
+    const uint64_t cs = pr[i] >> 32, fs = pr[i] & 0xFFFFFFFFull;
+    if (x >= ((RANS_L >> P) << 32) * fs) {
+      if (pos >= 12) {  // room for this word and the 8-byte state
+        pos -= 4;
+        for (int b = 0; b < 4; ++b) buf[pos + b] = (uint8_t)(x >> (8 * (3 - b)));
+      } else {
+        ok = false;
+      }
+      x >>= 32;
+    }
+    x = ((x / fs) << P) + (x % fs) + cs;
+  }
+  if (!ok) {
+    atomicOr(err, ERR_CAPACITY);
+    bits_out[c] = 0;
+    return;
+  }
+  const uint64_t words = ((cap_bytes & ~3ull) - pos) / 4;
+  pos -= 8;
+  for (int b = 0; b < 8; ++b) buf[pos + b] = (uint8_t)(x >> (8 * (7 - b)));
+  const uint64_t nbytes = 8 + 4 * words;
+  for (uint64_t i = 0; i < nbytes; ++i) buf[i] = buf[pos + i];  // front of the buffer (pos >= 0, ascending copy)
+  bits_out[c] = (uint32_t)(8 * nbytes);
+  if (out) {
+    uint8_t* dst = out + (offsets ? offsets[c] : (uint64_t)c * cap_bytes);
+    for (uint64_t i = 0; i < nbytes; ++i) dst[i] = buf[i];
+  }
 }
 
 // Minimal termination: shortest t with a multiple of 2^(64-t) in [low, low+rng).
@@ -363,17 +443,21 @@ int coder_reset(CoderState* st, int n, cudaStream_t s) {
   coder_reset_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n);
   return launch_status();
 }
-int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits,
+int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits, int rans,
                cudaStream_t s) {
   if (!n) return DLMZ_OK;
-  coder_load_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n, bytes, offsets, bits);
+  coder_load_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n, bytes, offsets, bits, rans);
   return launch_status();
 }
 int coder_finish(CoderState* st, int n, uint8_t* bytes, uint64_t cap_bytes, uint32_t* bits, uint8_t* out,
-                 const uint64_t* offsets, cudaStream_t s) {
+                 const uint64_t* offsets, int rans, const uint64_t* pairs, int pair_cap, int P, cudaStream_t s) {
   if (!n) return DLMZ_OK;
-  coder_finish_kernel<<<(n + 127) / 128, 128, 0, s>>>(st, n, bytes, cap_bytes, bits, out, offsets,
-                                                      device_error_word());
+  if (rans)
+    rans_finish_kernel<<<(n + 127) / 128, 128, 0, s>>>(st, n, pairs, pair_cap, P, bytes, cap_bytes, bits, out, offsets,
+                                                       device_error_word());
+  else
+    coder_finish_kernel<<<(n + 127) / 128, 128, 0, s>>>(st, n, bytes, cap_bytes, bits, out, offsets,
+                                                        device_error_word());
   return launch_status();
 }
 

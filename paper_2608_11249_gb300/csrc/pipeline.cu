@@ -258,7 +258,7 @@ struct BatchContext {
 
 // ---- per-batch step state ---------------------------------------------------------
 struct StepBufs {
-  DevBuf logits, W, Hq, top, mx, sel_count, sel_pos, committed, sum;
+  DevBuf logits, W, Hq, top, mx, sel_count, sel_pos, committed, sum, pairs;
   int ensure(size_t rows, int V, int nc, int kcap) {
     DLMZ_TRY(logits.ensure(rows * (size_t)V * 4));
     DLMZ_TRY(W.ensure(rows * 8));
@@ -273,7 +273,7 @@ struct StepBufs {
   }
   void release() {
     logits.release(); W.release(); Hq.release(); top.release(); mx.release();
-    sel_count.release(); sel_pos.release(); committed.release(); sum.release();
+    sel_count.release(); sel_pos.release(); committed.release(); sum.release(); pairs.release();
   }
 };
 
@@ -326,12 +326,19 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
   a.row0 = row0;
   a.rpc = rpc;
   a.kcap = kcap;
+  a.rans = pol.coder == DLMZ_CODER_RANS;
+  if (a.rans && !decode) {  // one (c, f) pair per position of every window
+    DLMZ_TRY(sb.pairs.ensure((size_t)nc * L * 8));
+    a.pairs = sb.pairs.as<uint64_t>();
+    a.pair_cap = L;
+  }
   return code_step(a, decode, nc, s);
 }
 
 static int validate_policy(const dlmz_k_policy* p) {
   if (!p) return DLMZ_EINVAL;
-  if (p->context > DLMZ_CONTEXT_RANDOM || (p->context == DLMZ_CONTEXT_NONE) != (p->context_c == 0) || p->reserved)
+  if (p->context > DLMZ_CONTEXT_RANDOM || (p->context == DLMZ_CONTEXT_NONE) != (p->context_c == 0) ||
+      p->coder > DLMZ_CODER_RANS)
     return DLMZ_EINVAL;
   if (p->kind == DLMZ_TOPK_CONF || p->kind == DLMZ_UNIFORM) return p->k >= 1 ? DLMZ_OK : DLMZ_EINVAL;
   if (p->kind == DLMZ_PROGRESSIVE)
@@ -367,7 +374,7 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
                                                              device_error_word());
     DLMZ_TRY(launch_status());
   }
-  if (decode) DLMZ_TRY(coder_load(cst, nc, in_bytes, in_off, in_bits, s));
+  if (decode) DLMZ_TRY(coder_load(cst, nc, in_bytes, in_off, in_bits, pol.coder == DLMZ_CODER_RANS, s));
   else DLMZ_TRY(coder_reset(cst, nc, s));
   // context positions of window w inside [a, b)
   auto ctx_in = [&](int w, int a, int b) -> int {
@@ -476,6 +483,7 @@ static int default_batch(const dlmz_model* m, uint32_t L, uint32_t n_chunks) {
 struct Header {
   uint32_t P, kind, vocab, chunk_len, batch_chunks, k, block, tau_q, k_min, k_max, n_chunks, crc;
   uint64_t fingerprint, n_symbols;
+  uint32_t coder = 0;                // 0: range coder, 1: rANS
   uint32_t ctx_kind = 0, ctx_c = 0;  // version 2: initial context (Sec. 3.4)
   uint64_t ctx_seed = 0;
   size_t size() const { return ctx_c ? 80 : 64; }
@@ -496,7 +504,7 @@ static uint64_t get64(const uint8_t* p) { uint64_t v = 0; for (int i = 0; i < 8;
 static void write_header(uint8_t* o, const Header& h) {
   memcpy(o, "DLMZ", 4);
   o[4] = h.ctx_c ? 2 : 1;
-  o[5] = 0;
+  o[5] = (uint8_t)h.coder;
   o[6] = (uint8_t)h.P;
   o[7] = (uint8_t)h.kind;
   put64(o + 8, h.fingerprint);
@@ -521,7 +529,8 @@ static void write_header(uint8_t* o, const Header& h) {
 // o holds the first min(n, 80) bytes of the file
 static int read_header(const uint8_t* o, size_t n, Header& h) {
   if (n < 64) return DLMZ_ECORRUPT;
-  if (memcmp(o, "DLMZ", 4) || (o[4] != 1 && o[4] != 2) || o[5] != 0) return DLMZ_ECORRUPT;
+  if (memcmp(o, "DLMZ", 4) || (o[4] != 1 && o[4] != 2) || o[5] > 1) return DLMZ_ECORRUPT;
+  h.coder = o[5];
   h.P = o[6];
   h.kind = o[7];
   h.fingerprint = get64(o + 8);
@@ -621,6 +630,7 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
     DLMZ_TRY(launch_status());
   }
   Header h{};
+  h.coder = pol->coder;
   h.ctx_kind = pol->context_c ? pol->context : 0;
   h.ctx_c = pol->context_c;
   h.ctx_seed = pol->context_seed;
@@ -642,7 +652,8 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
                            w.ctxsyms.as<uint8_t>(), s, bx));
     DLMZ_TRY(run_batch(m, w.sb, *pol, b.nc, b.L, w.symbols.as<int32_t>(), w.state.as<int32_t>(),
                        w.cst.as<CoderState>(), eb, cap, nullptr, nullptr, nullptr, false, bx, s));
-    DLMZ_TRY(coder_finish(w.cst.as<CoderState>(), b.nc, eb, cap, w.bits.as<uint32_t>() + b.c0, nullptr, nullptr, s));
+    DLMZ_TRY(coder_finish(w.cst.as<CoderState>(), b.nc, eb, cap, w.bits.as<uint32_t>() + b.c0, nullptr, nullptr,
+                          pol->coder == DLMZ_CODER_RANS, w.sb.pairs.as<uint64_t>(), b.L, P, s));
   }
   DLMZ_TRY(check_device(s));
   std::vector<uint32_t> bits(n_chunks), crcs(n_chunks);
@@ -710,6 +721,7 @@ static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes
   pol.tau_bits = (float)(h.tau_q / 65536.0);
   pol.k_min = h.k_min;
   pol.k_max = h.k_max;
+  pol.coder = h.coder;
   pol.context = h.ctx_kind;
   pol.context_c = h.ctx_c;
   pol.context_seed = h.ctx_seed;
@@ -941,7 +953,7 @@ int dlmz_select_smallest(const uint64_t* d_keys, uint32_t groups, uint32_t group
 }
 
 struct dlmz_coder {
-  int nc, L, V, P;
+  int nc, L, V, P, rans;
   uint64_t cap;
   DevBuf cst, bytes;
   StepBufs sb;
@@ -950,12 +962,13 @@ struct dlmz_coder {
   const uint32_t* in_bits = nullptr;
 };
 
-int dlmz_coder_create(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, dlmz_coder** out) {
+int dlmz_coder_create_ex(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, uint32_t coder, dlmz_coder** out) {
   if (!out) return DLMZ_EINVAL;
   *out = nullptr;
-  if (!n_chunks || !L || V < 2 || P > 24 || (1ull << P) <= V) return DLMZ_EINVAL;
+  if (!n_chunks || !L || V < 2 || P > 24 || (1ull << P) <= V || coder > DLMZ_CODER_RANS) return DLMZ_EINVAL;
   if (!device_error_word()) return DLMZ_ENOMEM;
   dlmz_coder* c = new dlmz_coder();
+  c->rans = coder == DLMZ_CODER_RANS;
   c->nc = (int)n_chunks;
   c->L = (int)L;
   c->V = (int)V;
@@ -967,6 +980,10 @@ int dlmz_coder_create(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, dlm
   }
   *out = c;
   return DLMZ_OK;
+}
+
+int dlmz_coder_create(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, dlmz_coder** out) {
+  return dlmz_coder_create_ex(n_chunks, L, V, P, DLMZ_CODER_RANGE, out);
 }
 
 void dlmz_coder_destroy(dlmz_coder* c) {
@@ -990,12 +1007,14 @@ int dlmz_coder_load_decoder(dlmz_coder* c, const uint8_t* d_bytes, const uint64_
   c->in_bytes = d_bytes;
   c->in_off = d_offsets;
   c->in_bits = d_bits;
-  return coder_load(c->cst.as<CoderState>(), c->nc, d_bytes, d_offsets, d_bits, reinterpret_cast<cudaStream_t>(stream));
+  return coder_load(c->cst.as<CoderState>(), c->nc, d_bytes, d_offsets, d_bits, c->rans,
+                    reinterpret_cast<cudaStream_t>(stream));
 }
 
 static int step_common(dlmz_coder* c, const dlmz_k_policy* pol, const float* d_logits, uint32_t row0, uint32_t rpc,
                        const int32_t* d_symbols, int32_t* d_state, int32_t* d_committed, bool decode, void* stream) {
   if (!c || !d_logits || !d_state || validate_policy(pol) != DLMZ_OK) return DLMZ_EINVAL;
+  if ((int)(pol->coder == DLMZ_CODER_RANS) != c->rans) return DLMZ_EINVAL;  // the coder's kind decides
   if (rpc == 0 || row0 + rpc > (uint32_t)c->L) return DLMZ_EINVAL;
   if (!decode && !d_symbols) return DLMZ_EINVAL;
   if (decode && !c->in_bytes) return DLMZ_EINVAL;
@@ -1018,7 +1037,7 @@ int dlmz_decode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_
 int dlmz_coder_finish(dlmz_coder* c, uint32_t* d_bits, uint8_t* d_bytes, const uint64_t* d_offsets, void* stream) {
   if (!c || !d_bits) return DLMZ_EINVAL;
   return coder_finish(c->cst.as<CoderState>(), c->nc, c->bytes.as<uint8_t>(), c->cap, d_bits, d_bytes, d_offsets,
-                      reinterpret_cast<cudaStream_t>(stream));
+                      c->rans, c->sb.pairs.as<uint64_t>(), c->L, c->P, reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

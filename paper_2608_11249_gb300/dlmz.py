@@ -22,6 +22,7 @@ OK, EINVAL, EBADINPUT, ECORRUPT, EMODEL, ENOMEM, ECUDA, ETIMEOUT, ECAPACITY = 0,
 FP32, BF16 = 0, 1
 TOPK_CONF, ENTROPY, UNIFORM, PROGRESSIVE = 0, 1, 2, 3
 CONTEXT_NONE, CONTEXT_CONTIGUOUS, CONTEXT_RANDOM = 0, 1, 2
+CODER_RANGE, CODER_RANS = 0, 1
 
 
 class DlmzError(RuntimeError):
@@ -39,7 +40,7 @@ class ModelConfig(Structure):
 class KPolicy(Structure):
     _fields_ = [("kind", c_uint32), ("k", c_uint32), ("block", c_uint32), ("tau_bits", c_float),
                 ("k_min", c_uint32), ("k_max", c_uint32), ("growth_q16", c_uint32), ("context", c_uint32),
-                ("context_c", c_uint32), ("reserved", c_uint32), ("context_seed", c_uint64)]
+                ("context_c", c_uint32), ("coder", c_uint32), ("context_seed", c_uint64)]
 
 
 class Profile(Structure):
@@ -75,6 +76,7 @@ _sig("dlmz_quantize", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P, _P, _P, _
 _sig("dlmz_select_smallest", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_select_smallest_noalloc", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_coder_create", c_int, c_uint32, c_uint32, c_uint32, c_uint32, POINTER(c_void_p))
+_sig("dlmz_coder_create_ex", c_int, c_uint32, c_uint32, c_uint32, c_uint32, c_uint32, POINTER(c_void_p))
 _sig("dlmz_coder_destroy", None, _P)
 _sig("dlmz_coder_reset_encoder", c_int, _P, _P)
 _sig("dlmz_coder_load_decoder", c_int, _P, _P, _P, _P, _P)
@@ -97,8 +99,8 @@ def strerror(code):
 
 
 def policy(kind=TOPK_CONF, k=1, block=0, tau_bits=0.0, k_min=1, k_max=0, growth_q16=65536,
-           context=CONTEXT_NONE, context_c=0, context_seed=0):
-    return KPolicy(kind, k, block, tau_bits, k_min, k_max, growth_q16, context, context_c, 0, context_seed)
+           context=CONTEXT_NONE, context_c=0, context_seed=0, coder=0):
+    return KPolicy(kind, k, block, tau_bits, k_min, k_max, growth_q16, context, context_c, coder, context_seed)
 
 
 class Model:
@@ -198,11 +200,11 @@ def check(stream=0):
 
 
 class Coder:
-    """Owns a dlmz_coder: one range-coder stream per window of a batch."""
+    """Owns a dlmz_coder: one coder stream (range coder or rANS) per window of a batch."""
 
-    def __init__(self, n_chunks, L, V, P):
+    def __init__(self, n_chunks, L, V, P, coder=CODER_RANGE):
         h = c_void_p()
-        _ok(lib.dlmz_coder_create(n_chunks, L, V, P, byref(h)), "dlmz_coder_create")
+        _ok(lib.dlmz_coder_create_ex(n_chunks, L, V, P, coder, byref(h)), "dlmz_coder_create_ex")
         self.h = h
 
     def close(self):

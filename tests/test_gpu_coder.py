@@ -17,14 +17,14 @@ from tests.gpu_helpers import dlmz, ptr, to_dev
 pytestmark = pytest.mark.gpu
 
 
-def _gpu_run(d, symbols, V, pol, opol, seed, L, ctx=None):
+def _gpu_run(d, symbols, V, pol, opol, seed, L, ctx=None, coder_kind=0):
     """Encode all windows on the GPU, then decode; return (bits, streams, decoded).
 
     ``ctx``: per-window context positions (the caller-side initial context, Sec. 3.4)."""
     import torch
     nc = symbols.shape[0]
     P = Q.precision_for_vocab(V)
-    coder = d.Coder(nc, L, V, P)
+    coder = d.Coder(nc, L, V, P, coder_kind)
     coder.reset_encoder()
     sym = to_dev(symbols.astype(np.int32))
     init = np.full((nc, L), V, dtype=np.int32)
@@ -44,7 +44,7 @@ def _gpu_run(d, symbols, V, pol, opol, seed, L, ctx=None):
                 lo = min(int(mk[t]) for mk in masked)
                 hi = max(int(mk[t + u - 1]) for mk in masked) + 1
                 lg = np.concatenate([sources.synthetic_logits(seed, c, step, L, V)[lo:hi] for c in range(nc)])
-                fn(to_dev(lg), lo, hi - lo, d.policy(opol.kind, u))
+                fn(to_dev(lg), lo, hi - lo, d.policy(opol.kind, u, coder=coder_kind))
                 t += u
                 step += 1
         elif opol.kind == S.TOPK_CONF:
@@ -84,7 +84,7 @@ def _gpu_run(d, symbols, V, pol, opol, seed, L, ctx=None):
     # decode from a packed copy of the streams
     offs = np.concatenate([[0], np.cumsum([(b + 7) // 8 for b in bits_h])[:-1]]).astype(np.uint64)
     packed = np.frombuffer(b"".join(streams) + b"\0" * 8, dtype=np.uint8)
-    dcoder = d.Coder(nc, L, V, P)
+    dcoder = d.Coder(nc, L, V, P, coder_kind)
     d_packed, d_offs, d_bits = to_dev(packed), to_dev(offs.view(np.int64)), to_dev(bits_h.astype(np.int32))
     dcoder.load_decoder(ptr(d_packed), ptr(d_offs), ptr(d_bits))
     state.copy_(to_dev(init))
@@ -151,3 +151,44 @@ def test_schedule_and_context_steps_bit_exact(dev, ci):
         (obits, obytes), _ = OP.encode_window(symbols[c], V, fn, opol, P, ctx=ctx[c])
         assert int(bits[c]) == obits and streams[c] == obytes, c
     assert np.array_equal(decoded, symbols)
+
+
+RANS_CASES = [
+    # V, L, nc, policy, context
+    (4, 6, 5, S.Policy(kind=S.TOPK_CONF, k=2, block=4), (X.NONE, 0, 0)),
+    (256, 512, 2, S.Policy(kind=S.TOPK_CONF, k=8, block=128), (X.NONE, 0, 0)),
+    (256, 64, 3, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=0), (X.NONE, 0, 0)),
+    (5000, 40, 2, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=64), (X.RANDOM, 5, 2)),
+    (126464, 24, 2, S.Policy(kind=S.UNIFORM, k=4), (X.NONE, 0, 0)),
+    (37, 50, 4, S.Policy(kind=S.PROGRESSIVE, k=1, growth_q16=3 << 15), (X.CONTIGUOUS, 3, 0)),
+]
+
+
+@pytest.mark.parametrize("ci", range(len(RANS_CASES)))
+def test_rans_steps_bit_exact_and_decode(dev, ci):
+    """The paper's rANS coder (Sec. 2.1) on identical logits: streams bit for bit, then decoded."""
+    d = dlmz()
+    V, L, nc, opol, (ck, cc, cs) = RANS_CASES[ci]
+    seed = 300 + ci
+    symbols = np.random.default_rng(seed).integers(0, V, (nc, L))
+    ctx = [X.positions(ck, cc, cs, L, c) for c in range(nc)]
+    pol = d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max, opol.growth_q16,
+                   coder=d.CODER_RANS)
+    bits, streams, decoded = _gpu_run(d, symbols, V, pol, opol, seed, L, ctx, d.CODER_RANS)
+    P = Q.precision_for_vocab(V)
+    for c in range(nc):
+        fn = lambda step, state, rows, c=c: sources.synthetic_logits(seed, c, step, L, V)[rows]
+        (obits, obytes), _ = OP.encode_window(symbols[c], V, fn, opol, P, ctx=ctx[c], coder=OP.RANS)
+        assert int(bits[c]) == obits and streams[c] == obytes, c
+    assert np.array_equal(decoded, symbols)
+
+
+def test_coder_kind_must_match(dev):
+    d = dlmz()
+    coder = d.Coder(2, 8, 256, 16, d.CODER_RANS)
+    lg = to_dev(np.zeros((16, 256), dtype=np.float32))
+    st = to_dev(np.full((2, 8), 256, dtype=np.int32))
+    sym = to_dev(np.zeros((2, 8), dtype=np.int32))
+    with pytest.raises(d.DlmzError) as e:
+        coder.encode_step(d.policy(d.TOPK_CONF, 1), ptr(lg), 0, 8, ptr(sym), ptr(st), 0)
+    assert e.value.code == d.EINVAL

@@ -94,12 +94,42 @@ def test_schedules_and_context_vs_oracle(dev, ci):
     assert abs(len(blob) - len(oblob)) <= 0.005 * len(oblob) + 8, (len(blob), len(oblob))
 
 
+RANS_RT = [
+    ((1, 32, 2, 2, 64, 256, "f32"), "bytes", 1500, 512, S.Policy(kind=S.TOPK_CONF, k=4, block=64), (OX.NONE, 0, 0), 0),
+    ((2, 256, 4, 4, 256, 256, "bf16"), "bytes", 1100, 256, S.Policy(kind=S.UNIFORM, k=32), (OX.RANDOM, 8, 5), 3),
+    ((1, 64, 4, 2, 128, 5000, "f32"), "tokens", 300, 100, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=8),
+     (OX.NONE, 0, 0), 0),
+]
+
+
+@pytest.mark.parametrize("ci", range(len(RANS_RT)))
+def test_rans_roundtrip_and_size_vs_oracle(dev, ci):
+    """Whole files with the rANS coder: round trip, header coder byte, size against the oracle's rANS file."""
+    d = dlmz()
+    spec, kind, n, L, opol, ctx, bc = RANS_RT[ci]
+    m = _model(d, spec, 80 + ci)
+    data = _data(kind, n, spec[5])
+    pol = d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max, opol.growth_q16,
+                   ctx[0], ctx[1], ctx[2], coder=d.CODER_RANS)
+    blob = m.compress(data, L, pol, bc)
+    assert m.decompress(blob) == data
+    h, streams = OC.read(blob)
+    assert h.coder == 1 and all(b % 32 == 0 and b >= 64 for b, _ in streams)
+    w = OM.Weights(OM.ModelConfig(*spec, seed=80 + ci))
+    oblob = OP.compress(w, data, L, opol, context=ctx, coder=OP.RANS)
+    assert abs(len(blob) - len(oblob)) <= 0.005 * len(oblob) + 8, (len(blob), len(oblob))
+    rblob = m.compress(data, L, d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max,
+                                         opol.growth_q16, ctx[0], ctx[1], ctx[2]), bc)
+    assert len(blob) - len(rblob) <= 13 * h.n_chunks + 8  # rANS: at most ~96 bits more per window than the range coder
+
+
 def test_bad_schedule_and_context_rejected(dev):
     d = dlmz()
     m = _model(d, (1, 32, 2, 2, 64, 256, "f32"), 1)
     for pol in (d.policy(d.UNIFORM, 0), d.policy(d.PROGRESSIVE, 1, growth_q16=0),
                 d.policy(d.PROGRESSIVE, 1, growth_q16=(64 << 16) + 1), d.policy(d.TOPK_CONF, 2, context=d.CONTEXT_RANDOM),
-                d.policy(d.TOPK_CONF, 2, context=7, context_c=1), d.policy(d.TOPK_CONF, 2, context_c=3)):
+                d.policy(d.TOPK_CONF, 2, context=7, context_c=1), d.policy(d.TOPK_CONF, 2, context_c=3),
+                d.policy(d.TOPK_CONF, 2, coder=2)):
         with pytest.raises(d.DlmzError) as e:
             m.compress(b"abcdef", 4, pol)
         assert e.value.code == d.EINVAL
