@@ -26,6 +26,7 @@ Diffusion LMs for Lossless Compression"):
 * ``coder``     -- range coder with minimal termination (statistical coding,
                    Sec. 2.1 and Sec. 4 "Implementation Details").
 * ``rans``      -- rANS coder (64-bit state, 32-bit words), the paper's coder.
+* ``ranking``   -- symbol ranking with varint output (the paper's ranking pipeline).
 * ``container`` -- compressed-file header (Sec. 3.3 last paragraph, Sec. 4).
 * ``pipeline``  -- the iterative pipeline S^(k+1) = f_theta(S^(k)) of
                    Sec. 3.2, compress and decompress.

@@ -8,7 +8,7 @@ Details") are stored so the decompressor replays every decision.  Layout
     off size field
       0   4  magic "DLMZ"
       4   1  version (1; 2 when the windows carry an initial context)
-      5   1  coder (0 = range coder, 1 = rANS)
+      5   1  coder (0 = range coder, 1 = rANS, 2 = symbol ranks as varints)
       6   1  P, CDF precision bits
       7   1  policy kind (0 = top-k confidence, 1 = entropy, 2 = uniform block,
              3 = progressive; for 3 the block field holds r in 16.16 fixed point)
@@ -145,7 +145,7 @@ def read(buf):
         raise ContainerError("bad magic")
     if f[1] not in (VERSION, VERSION_CONTEXT):
         raise ContainerError("unsupported version")
-    if f[2] not in (0, 1):
+    if f[2] not in (0, 1, 2):
         raise ContainerError("unknown coder")
     h = Header(*f[3:], coder=f[2])
     if h.chunk_len == 0 and h.n_symbols:

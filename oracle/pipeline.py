@@ -24,12 +24,14 @@ from . import context as X
 from . import model as M
 from . import quantizer as Q
 from . import rans
+from . import ranking
 from . import selector as S
 from .coder import Decoder, Encoder
 
-RANGE, RANS = 0, 1  # statistical coders: range coder, rANS (Sec. 2.1)
-_ENC = {RANGE: Encoder, RANS: rans.Encoder}
-_DEC = {RANGE: Decoder, RANS: rans.Decoder}
+# coders: range coder, rANS (statistical coding, Sec. 2.1), symbol ranks (varints)
+RANGE, RANS, RANKS = 0, 1, 2
+_ENC = {RANGE: Encoder, RANS: rans.Encoder, RANKS: ranking.Encoder}
+_DEC = {RANGE: Decoder, RANS: rans.Decoder, RANKS: ranking.Decoder}
 
 
 class BadInput(ValueError):
@@ -102,7 +104,10 @@ def encode_window(symbols, V, logits_fn, policy, P, trace=None, ctx=(), coder=RA
         assert sel, "a step must commit at least one position"
         for p in sel:
             i, s = row[p], int(symbols[p])
-            enc.encode(int(qz["cdf"][i, s]), int(qz["freq"][i, s]))
+            if coder == RANKS:
+                enc.encode_rank(qz["freq"][i], s)
+            else:
+                enc.encode(int(qz["cdf"][i, s]), int(qz["freq"][i, s]))
         state[sel] = symbols[sel]
         if trace is not None:
             trace.append(list(sel))
