@@ -125,4 +125,4 @@ def test_pipeline_round_trips_with_rans(w4, pol):
     h, _ = C.read(blob)
     assert h.coder == PL.RANS and blob[5] == 1
     with pytest.raises(C.ContainerError):
-        C.read(blob[:5] + b"\x02" + blob[6:])
+        C.read(blob[:5] + b"\x03" + blob[6:])
