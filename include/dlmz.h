@@ -91,6 +91,8 @@ DLMZ_API int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg);
 
 #define DLMZ_CODER_RANGE 0u /* range coder, minimal termination: ideal length + at most ~1 bit per window */
 #define DLMZ_CODER_RANS 1u  /* rANS, 64-bit state, 32-bit words: ideal length + at most 96 bits per window */
+#define DLMZ_CODER_RANKS 2u /* symbol ranking: each symbol's rank (frequency descending, ties by index) as an
+                               LEB128 varint -- the paper's ranking pipeline before its back-end compressor */
 
 #define DLMZ_CONTEXT_NONE 0u       /* every position starts masked (c = 0) */
 #define DLMZ_CONTEXT_CONTIGUOUS 1u /* the first c symbols of each window stay visible */
@@ -108,7 +110,8 @@ typedef struct {
   uint32_t context;      /* DLMZ_CONTEXT_*: initial context of every window (compress only; the
                             decompressor reads it from the file) */
   uint32_t context_c;    /* c, symbols per window left visible (0 exactly when context is NONE) */
-  uint32_t coder;        /* DLMZ_CODER_RANGE (default) or DLMZ_CODER_RANS (the paper's rANS, Sec. 2.1) */
+  uint32_t coder;        /* DLMZ_CODER_RANGE (default), DLMZ_CODER_RANS (the paper's rANS, Sec. 2.1) or
+                            DLMZ_CODER_RANKS (symbol ranking, varint ranks) */
   uint64_t context_seed; /* RANDOM: seed of the positions */
 } dlmz_k_policy;
 

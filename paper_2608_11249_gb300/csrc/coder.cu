@@ -18,6 +18,10 @@
 // when x >= 2^(63-P) f.  Last in, first out: the steps buffer a window's
 // (c, f) pairs and the finish kernel codes them in reverse; the stream is the
 // final state (8 bytes big-endian) then the words in reverse emission order.
+// Symbol ranks (the paper's ranking pipeline): each coded symbol becomes
+// #{v : f_v > f_s} + #{v < s : f_v = f_s} (integer frequencies of the step's
+// table), written as an LEB128 varint; the decoder finds the frequency level
+// holding rank r by binary search (block counts), then the symbol by index.
 #include "kernels.cuh"
 #include "coder.cuh"
 #include "exp_table.inc"
@@ -215,6 +219,10 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
     const float m = a.mx[row];
     const uint64_t Wr = a.W[row];
     const int top = a.top[row];
+    auto qv = [&](float x) -> int {
+      return isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f))
+                         : 8191;
+    };
     uint64_t sseg = 0;
     for (int v = v0; v < v1; ++v) {
       const float x = lr[v];
@@ -224,6 +232,8 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
     uint64_t total;
     const uint64_t pre = block_excl_scan(sseg, wsum, &total);
     const uint64_t D = (1ull << P) - total;
+    // f_v of this row (the same integer table the coders use)
+#define FREQ(v_) (1 + (uint64_t)(T[qv(lr[v_]) & 255] >> (qv(lr[v_]) >> 8)) * R / Wr + ((v_) == top ? D : 0))
     const uint64_t lo = pre + (v0 > top ? D : 0);
     const uint64_t hi = lo + sseg + (top >= v0 && top < v1 ? D : 0);
     if (!DECODE) {
@@ -243,9 +253,27 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
         }
       }
       __syncthreads();
+      uint64_t rank = 0;
+      if (a.coder == 2) {  // rank of sym: frequencies above f_s, then equal ones with a smaller index
+        uint64_t cnt = 0;
+        for (int v = v0; v < v1; ++v) {
+          const uint64_t f = FREQ(v);
+          cnt += f > s_fs || (f == s_fs && v < sym);
+        }
+        block_excl_scan(cnt, wsum, &rank);
+      }
       if (threadIdx.x == 0) {
         CoderState t = st;
-        if (a.rans) {  // buffered; coded in reverse when the window is finished
+        if (a.coder == 2) {
+          uint64_t r = rank;
+          do {
+            const uint8_t b = (uint8_t)((r & 0x7F) | (r >= 0x80 ? 0x80 : 0));
+            if (t.n_units < a.cap_bytes) ebuf[t.n_units] = b;
+            else atomicOr(a.err, ERR_CAPACITY);
+            t.n_units++;
+            r >>= 7;
+          } while (r);
+        } else if (a.coder == 1) {  // buffered; coded in reverse when the window is finished
           if (t.n_units < (uint32_t)a.pair_cap) a.pairs[(size_t)c * a.pair_cap + t.n_units] = (s_cs << 32) | s_fs;
           else atomicOr(a.err, ERR_CAPACITY);
           t.n_units++;
@@ -258,7 +286,25 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       __syncthreads();
     } else {
       if (threadIdx.x == 0) {
-        if (a.rans) {
+        if (a.coder == 2) {  // next varint of the window's rank stream
+          uint64_t r = 0, pos = st.n_units;
+          int sh = 0;
+          bool done = false;
+          while (!done) {
+            const uint8_t b = pos < dn ? dbuf[pos] : 0x80;
+            ++pos;
+            if (sh < 63) r |= (uint64_t)(b & 0x7F) << sh;
+            sh += 7;
+            done = !(b & 0x80) || sh > 35;
+            if (pos > dn) done = true;
+          }
+          if (pos > dn || sh > 35 || r >= (uint64_t)V) {
+            atomicOr(a.err, ERR_CORRUPT);
+            r = 0;
+          }
+          st.n_units = (uint32_t)pos;
+          s_slot = r;
+        } else if (a.coder == 1) {
           s_slot = st.low & ((1ull << P) - 1);  // x mod 2^P
         } else {
           const uint64_t r = st.rng >> P;
@@ -272,7 +318,39 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       }
       __syncthreads();
       const uint64_t slot = s_slot;
-      if (slot >= lo && slot < hi) {
+      if (a.coder == 2) {  // slot holds the rank r: find the frequency level, then the symbol by index
+        uint64_t flo = 1, fhi = (1ull << P) + 1, tot;  // count(f >= flo) > r >= count(f >= fhi)
+        while (fhi - flo > 1) {
+          const uint64_t mid = (flo + fhi) / 2;
+          uint64_t cnt = 0;
+          for (int v = v0; v < v1; ++v) cnt += FREQ(v) >= mid;
+          block_excl_scan(cnt, wsum, &tot);
+          if (tot > slot) flo = mid;
+          else fhi = mid;
+        }
+        uint64_t above = 0, eq = 0;
+        for (int v = v0; v < v1; ++v) {
+          const uint64_t f = FREQ(v);
+          above += f > flo;
+          eq += f == flo;
+        }
+        block_excl_scan(above, wsum, &tot);
+        const uint64_t t = slot - tot;  // index of the symbol among those with f == flo
+        const uint64_t pre = block_excl_scan(eq, wsum, &tot);
+        if (t >= pre && t < pre + eq) {
+          uint64_t k = pre;
+          for (int v = v0; v < v1; ++v) {
+            if (FREQ(v) == flo) {
+              if (k == t) {
+                s_sym = v;
+                s_fs = flo;
+                break;
+              }
+              ++k;
+            }
+          }
+        }
+      } else if (slot >= lo && slot < hi) {
         uint64_t cum = lo;
         for (int v = v0; v < v1; ++v) {
           const float x = lr[v];
@@ -290,7 +368,9 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       __syncthreads();
       if (threadIdx.x == 0) {
         CoderState t = st;
-        if (a.rans) {
+        if (a.coder == 2) {
+          // the rank stream advanced when it was read
+        } else if (a.coder == 1) {
           t.low = s_fs * (t.low >> P) + slot - s_cs;
           if (t.low < RANS_L) {
             t.low = (t.low << 32) | word_at(dbuf, dn, 8 + 4ull * t.n_units);
@@ -311,6 +391,7 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       __syncthreads();
     }
   }
+#undef FREQ
   if (threadIdx.x == 0) {
     a.state_c[c] = st;
     if (a.committed) a.committed[c] = n;
@@ -335,14 +416,16 @@ __global__ void coder_reset_kernel(CoderState* st, int n) {
 }
 
 __global__ void coder_load_kernel(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets,
-                                  const uint32_t* bits, int rans) {
+                                  const uint32_t* bits, int coder) {
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= n) return;
   const uint8_t* b = bytes + (offsets ? offsets[c] : 0);
   const uint64_t nb = (bits[c] + 7) / 8;
   uint64_t v = 0;
-  if (rans) {  // the final state of the encoder leads the stream
+  if (coder == 1) {  // the final state of the encoder leads the stream
     v = (word_at(b, nb, 0) << 32) | word_at(b, nb, 4);
+    st[c].n_units = 0;
+  } else if (coder == 2) {  // ranks: read from byte 0
     st[c].n_units = 0;
   } else {
     for (int i = 0; i < 4; ++i) v = (v << 16) | unit_at(b, nb, i);
@@ -443,16 +526,38 @@ int coder_reset(CoderState* st, int n, cudaStream_t s) {
   coder_reset_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n);
   return launch_status();
 }
-int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits, int rans,
+int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits, int coder,
                cudaStream_t s) {
   if (!n) return DLMZ_OK;
-  coder_load_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n, bytes, offsets, bits, rans);
+  coder_load_kernel<<<(n + 255) / 256, 256, 0, s>>>(st, n, bytes, offsets, bits, coder);
   return launch_status();
 }
+
+// Ranks: the varint stream is complete as written; report its length and copy it out.
+__global__ void ranks_finish_kernel(const CoderState* st, int n, const uint8_t* bytes, uint64_t cap_bytes,
+                                    uint32_t* bits_out, uint8_t* out, const uint64_t* offsets, int* err) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n) return;
+  const uint64_t nbytes = st[c].n_units;
+  if (nbytes > cap_bytes) {
+    atomicOr(err, ERR_CAPACITY);
+    bits_out[c] = 0;
+    return;
+  }
+  bits_out[c] = (uint32_t)(8 * nbytes);
+  if (out) {
+    const uint8_t* buf = bytes + (size_t)c * cap_bytes;
+    uint8_t* dst = out + (offsets ? offsets[c] : (uint64_t)c * cap_bytes);
+    for (uint64_t i = 0; i < nbytes; ++i) dst[i] = buf[i];
+  }
+}
 int coder_finish(CoderState* st, int n, uint8_t* bytes, uint64_t cap_bytes, uint32_t* bits, uint8_t* out,
-                 const uint64_t* offsets, int rans, const uint64_t* pairs, int pair_cap, int P, cudaStream_t s) {
+                 const uint64_t* offsets, int coder, const uint64_t* pairs, int pair_cap, int P, cudaStream_t s) {
   if (!n) return DLMZ_OK;
-  if (rans)
+  if (coder == 2)
+    ranks_finish_kernel<<<(n + 127) / 128, 128, 0, s>>>(st, n, bytes, cap_bytes, bits, out, offsets,
+                                                        device_error_word());
+  else if (coder == 1)
     rans_finish_kernel<<<(n + 127) / 128, 128, 0, s>>>(st, n, pairs, pair_cap, P, bytes, cap_bytes, bits, out, offsets,
                                                        device_error_word());
   else

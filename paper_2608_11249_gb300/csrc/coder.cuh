@@ -9,6 +9,7 @@ namespace dlmz {
 // emitted 16-bit units; decoder: `low` holds val = code - low, `n_units` the
 // next unit to read.  rANS -- encoder: `n_units` counts the buffered (c, f)
 // pairs; decoder: `low` is the state x, `n_units` the next 32-bit word.
+// Ranks -- `n_units` is the byte position in the window's varint stream.
 struct CoderState {
   uint64_t low;
   uint64_t rng;
@@ -34,7 +35,7 @@ struct CodeArgs {
   int32_t* committed;        // optional [n_chunks]
   int* err;
   int V, P, L, row0, rpc, kcap;
-  int rans;                  // 0: range coder, 1: rANS
+  int coder;                 // 0: range coder, 1: rANS, 2: symbol ranks (varints)
   uint64_t* pairs;           // rANS encoder: (c << 32 | f) per coded symbol [n_chunks x pair_cap]
   int pair_cap;
 };
@@ -45,12 +46,12 @@ int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0
                 cudaStream_t s);
 int code_step(const CodeArgs& a, bool decode, int n_chunks, cudaStream_t s);
 int coder_reset(CoderState* st, int n, cudaStream_t s);
-int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits, int rans,
+int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits, int coder,
                cudaStream_t s);
 // Terminates every stream (range coder) or codes every window's buffered pairs
 // in reverse (rANS: pairs, pair_cap, P), then bit lengths / copies as documented
 // at dlmz_coder_finish.
 int coder_finish(CoderState* st, int n, uint8_t* bytes, uint64_t cap_bytes, uint32_t* bits, uint8_t* out,
-                 const uint64_t* offsets, int rans, const uint64_t* pairs, int pair_cap, int P, cudaStream_t s);
+                 const uint64_t* offsets, int coder, const uint64_t* pairs, int pair_cap, int P, cudaStream_t s);
 
 }  // namespace dlmz

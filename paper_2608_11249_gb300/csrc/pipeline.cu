@@ -326,8 +326,8 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
   a.row0 = row0;
   a.rpc = rpc;
   a.kcap = kcap;
-  a.rans = pol.coder == DLMZ_CODER_RANS;
-  if (a.rans && !decode) {  // one (c, f) pair per position of every window
+  a.coder = (int)pol.coder;
+  if (pol.coder == DLMZ_CODER_RANS && !decode) {  // one (c, f) pair per position of every window
     DLMZ_TRY(sb.pairs.ensure((size_t)nc * L * 8));
     a.pairs = sb.pairs.as<uint64_t>();
     a.pair_cap = L;
@@ -338,7 +338,7 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
 static int validate_policy(const dlmz_k_policy* p) {
   if (!p) return DLMZ_EINVAL;
   if (p->context > DLMZ_CONTEXT_RANDOM || (p->context == DLMZ_CONTEXT_NONE) != (p->context_c == 0) ||
-      p->coder > DLMZ_CODER_RANS)
+      p->coder > DLMZ_CODER_RANKS)
     return DLMZ_EINVAL;
   if (p->kind == DLMZ_TOPK_CONF || p->kind == DLMZ_UNIFORM) return p->k >= 1 ? DLMZ_OK : DLMZ_EINVAL;
   if (p->kind == DLMZ_PROGRESSIVE)
@@ -374,7 +374,7 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
                                                              device_error_word());
     DLMZ_TRY(launch_status());
   }
-  if (decode) DLMZ_TRY(coder_load(cst, nc, in_bytes, in_off, in_bits, pol.coder == DLMZ_CODER_RANS, s));
+  if (decode) DLMZ_TRY(coder_load(cst, nc, in_bytes, in_off, in_bits, (int)pol.coder, s));
   else DLMZ_TRY(coder_reset(cst, nc, s));
   // context positions of window w inside [a, b)
   auto ctx_in = [&](int w, int a, int b) -> int {
@@ -483,7 +483,7 @@ static int default_batch(const dlmz_model* m, uint32_t L, uint32_t n_chunks) {
 struct Header {
   uint32_t P, kind, vocab, chunk_len, batch_chunks, k, block, tau_q, k_min, k_max, n_chunks, crc;
   uint64_t fingerprint, n_symbols;
-  uint32_t coder = 0;                // 0: range coder, 1: rANS
+  uint32_t coder = 0;                // 0: range coder, 1: rANS, 2: symbol ranks
   uint32_t ctx_kind = 0, ctx_c = 0;  // version 2: initial context (Sec. 3.4)
   uint64_t ctx_seed = 0;
   size_t size() const { return ctx_c ? 80 : 64; }
@@ -529,7 +529,7 @@ static void write_header(uint8_t* o, const Header& h) {
 // o holds the first min(n, 80) bytes of the file
 static int read_header(const uint8_t* o, size_t n, Header& h) {
   if (n < 64) return DLMZ_ECORRUPT;
-  if (memcmp(o, "DLMZ", 4) || (o[4] != 1 && o[4] != 2) || o[5] > 1) return DLMZ_ECORRUPT;
+  if (memcmp(o, "DLMZ", 4) || (o[4] != 1 && o[4] != 2) || o[5] > 2) return DLMZ_ECORRUPT;
   h.coder = o[5];
   h.P = o[6];
   h.kind = o[7];
@@ -653,7 +653,7 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
     DLMZ_TRY(run_batch(m, w.sb, *pol, b.nc, b.L, w.symbols.as<int32_t>(), w.state.as<int32_t>(),
                        w.cst.as<CoderState>(), eb, cap, nullptr, nullptr, nullptr, false, bx, s));
     DLMZ_TRY(coder_finish(w.cst.as<CoderState>(), b.nc, eb, cap, w.bits.as<uint32_t>() + b.c0, nullptr, nullptr,
-                          pol->coder == DLMZ_CODER_RANS, w.sb.pairs.as<uint64_t>(), b.L, P, s));
+                          (int)pol->coder, w.sb.pairs.as<uint64_t>(), b.L, P, s));
   }
   DLMZ_TRY(check_device(s));
   std::vector<uint32_t> bits(n_chunks), crcs(n_chunks);
@@ -953,7 +953,7 @@ int dlmz_select_smallest(const uint64_t* d_keys, uint32_t groups, uint32_t group
 }
 
 struct dlmz_coder {
-  int nc, L, V, P, rans;
+  int nc, L, V, P, coder;
   uint64_t cap;
   DevBuf cst, bytes;
   StepBufs sb;
@@ -965,10 +965,10 @@ struct dlmz_coder {
 int dlmz_coder_create_ex(uint32_t n_chunks, uint32_t L, uint32_t V, uint32_t P, uint32_t coder, dlmz_coder** out) {
   if (!out) return DLMZ_EINVAL;
   *out = nullptr;
-  if (!n_chunks || !L || V < 2 || P > 24 || (1ull << P) <= V || coder > DLMZ_CODER_RANS) return DLMZ_EINVAL;
+  if (!n_chunks || !L || V < 2 || P > 24 || (1ull << P) <= V || coder > DLMZ_CODER_RANKS) return DLMZ_EINVAL;
   if (!device_error_word()) return DLMZ_ENOMEM;
   dlmz_coder* c = new dlmz_coder();
-  c->rans = coder == DLMZ_CODER_RANS;
+  c->coder = (int)coder;
   c->nc = (int)n_chunks;
   c->L = (int)L;
   c->V = (int)V;
@@ -1007,14 +1007,14 @@ int dlmz_coder_load_decoder(dlmz_coder* c, const uint8_t* d_bytes, const uint64_
   c->in_bytes = d_bytes;
   c->in_off = d_offsets;
   c->in_bits = d_bits;
-  return coder_load(c->cst.as<CoderState>(), c->nc, d_bytes, d_offsets, d_bits, c->rans,
+  return coder_load(c->cst.as<CoderState>(), c->nc, d_bytes, d_offsets, d_bits, c->coder,
                     reinterpret_cast<cudaStream_t>(stream));
 }
 
 static int step_common(dlmz_coder* c, const dlmz_k_policy* pol, const float* d_logits, uint32_t row0, uint32_t rpc,
                        const int32_t* d_symbols, int32_t* d_state, int32_t* d_committed, bool decode, void* stream) {
   if (!c || !d_logits || !d_state || validate_policy(pol) != DLMZ_OK) return DLMZ_EINVAL;
-  if ((int)(pol->coder == DLMZ_CODER_RANS) != c->rans) return DLMZ_EINVAL;  // the coder's kind decides
+  if ((int)pol->coder != c->coder) return DLMZ_EINVAL;  // the coder's kind decides
   if (rpc == 0 || row0 + rpc > (uint32_t)c->L) return DLMZ_EINVAL;
   if (!decode && !d_symbols) return DLMZ_EINVAL;
   if (decode && !c->in_bytes) return DLMZ_EINVAL;
@@ -1037,7 +1037,7 @@ int dlmz_decode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_
 int dlmz_coder_finish(dlmz_coder* c, uint32_t* d_bits, uint8_t* d_bytes, const uint64_t* d_offsets, void* stream) {
   if (!c || !d_bits) return DLMZ_EINVAL;
   return coder_finish(c->cst.as<CoderState>(), c->nc, c->bytes.as<uint8_t>(), c->cap, d_bits, d_bytes, d_offsets,
-                      c->rans, c->sb.pairs.as<uint64_t>(), c->L, c->P, reinterpret_cast<cudaStream_t>(stream));
+                      c->coder, c->sb.pairs.as<uint64_t>(), c->L, c->P, reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

@@ -22,7 +22,7 @@ OK, EINVAL, EBADINPUT, ECORRUPT, EMODEL, ENOMEM, ECUDA, ETIMEOUT, ECAPACITY = 0,
 FP32, BF16 = 0, 1
 TOPK_CONF, ENTROPY, UNIFORM, PROGRESSIVE = 0, 1, 2, 3
 CONTEXT_NONE, CONTEXT_CONTIGUOUS, CONTEXT_RANDOM = 0, 1, 2
-CODER_RANGE, CODER_RANS = 0, 1
+CODER_RANGE, CODER_RANS, CODER_RANKS = 0, 1, 2
 
 
 class DlmzError(RuntimeError):

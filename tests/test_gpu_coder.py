@@ -192,3 +192,32 @@ def test_coder_kind_must_match(dev):
     with pytest.raises(d.DlmzError) as e:
         coder.encode_step(d.policy(d.TOPK_CONF, 1), ptr(lg), 0, 8, ptr(sym), ptr(st), 0)
     assert e.value.code == d.EINVAL
+
+
+RANK_CASES = [
+    # V, L, nc, policy, context
+    (4, 6, 5, S.Policy(kind=S.TOPK_CONF, k=2, block=4), (X.NONE, 0, 0)),
+    (256, 100, 3, S.Policy(kind=S.TOPK_CONF, k=4, block=64), (X.NONE, 0, 0)),
+    (256, 64, 3, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=0), (X.RANDOM, 4, 1)),
+    (5000, 33, 2, S.Policy(kind=S.UNIFORM, k=5), (X.NONE, 0, 0)),
+    (37, 50, 2, S.Policy(kind=S.PROGRESSIVE, k=2, growth_q16=3 << 15), (X.CONTIGUOUS, 2, 0)),
+]
+
+
+@pytest.mark.parametrize("ci", range(len(RANK_CASES)))
+def test_rank_steps_bit_exact_and_decode(dev, ci):
+    """Symbol ranking (varint ranks) on identical logits: rank streams byte for byte, then decoded."""
+    d = dlmz()
+    V, L, nc, opol, (ck, cc, cs) = RANK_CASES[ci]
+    seed = 400 + ci
+    symbols = np.random.default_rng(seed).integers(0, V, (nc, L))
+    ctx = [X.positions(ck, cc, cs, L, c) for c in range(nc)]
+    pol = d.policy(opol.kind, opol.k, opol.block, opol.tau_bits, opol.k_min, opol.k_max, opol.growth_q16,
+                   coder=d.CODER_RANKS)
+    bits, streams, decoded = _gpu_run(d, symbols, V, pol, opol, seed, L, ctx, d.CODER_RANKS)
+    P = Q.precision_for_vocab(V)
+    for c in range(nc):
+        fn = lambda step, state, rows, c=c: sources.synthetic_logits(seed, c, step, L, V)[rows]
+        (obits, obytes), _ = OP.encode_window(symbols[c], V, fn, opol, P, ctx=ctx[c], coder=OP.RANKS)
+        assert int(bits[c]) == obits and streams[c] == obytes, c
+    assert np.array_equal(decoded, symbols)

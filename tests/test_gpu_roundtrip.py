@@ -123,13 +123,39 @@ def test_rans_roundtrip_and_size_vs_oracle(dev, ci):
     assert len(blob) - len(rblob) <= 13 * h.n_chunks + 8  # rANS: at most ~96 bits more per window than the range coder
 
 
+def test_ranks_roundtrip_and_size_vs_oracle(dev):
+    """Whole files with symbol ranks: round trip, coder byte, size against the oracle's rank file."""
+    d = dlmz()
+    spec = (1, 32, 2, 2, 64, 256, "f32")
+    m = _model(d, spec, 90)
+    data = _data("bytes", 1200, 256)
+    opol = S.Policy(kind=S.TOPK_CONF, k=4, block=64)
+    pol = d.policy(opol.kind, opol.k, opol.block, coder=d.CODER_RANKS)
+    blob = m.compress(data, 256, pol)
+    assert m.decompress(blob) == data
+    h, streams = OC.read(blob)
+    assert h.coder == 2 and all(b % 8 == 0 for b, _ in streams)
+    w = OM.Weights(OM.ModelConfig(*spec, seed=90))
+    oblob = OP.compress(w, data, 256, opol, coder=OP.RANKS)
+    assert abs(len(blob) - len(oblob)) <= 0.005 * len(oblob) + 8, (len(blob), len(oblob))
+    for i in (80, len(blob) // 2, len(blob) - 1):  # edited rank bytes: rejected, never a crash
+        bad = blob[:i] + bytes([blob[i] ^ 0x40]) + blob[i + 1:]
+        try:
+            out = m.decompress(bad)
+        except d.DlmzError as e:
+            assert e.code == d.ECORRUPT
+        else:
+            assert out == data
+    d.check()
+
+
 def test_bad_schedule_and_context_rejected(dev):
     d = dlmz()
     m = _model(d, (1, 32, 2, 2, 64, 256, "f32"), 1)
     for pol in (d.policy(d.UNIFORM, 0), d.policy(d.PROGRESSIVE, 1, growth_q16=0),
                 d.policy(d.PROGRESSIVE, 1, growth_q16=(64 << 16) + 1), d.policy(d.TOPK_CONF, 2, context=d.CONTEXT_RANDOM),
                 d.policy(d.TOPK_CONF, 2, context=7, context_c=1), d.policy(d.TOPK_CONF, 2, context_c=3),
-                d.policy(d.TOPK_CONF, 2, coder=2)):
+                d.policy(d.TOPK_CONF, 2, coder=3)):
         with pytest.raises(d.DlmzError) as e:
             m.compress(b"abcdef", 4, pol)
         assert e.value.code == d.EINVAL
