@@ -29,6 +29,13 @@ METRIC = "input bytes/sec compress+decompress on 1 GB300; bits/byte; % of roofli
 MODEL = dict(n_layers=8, d=512, n_heads=8, n_kv_heads=8, ffn=2048, vocab=256, seed=0)
 CHUNK, BATCH, BLOCK, K = 512, 1024, 128, 8
 INPUT_BYTES = 4 << 20
+# DRAM read + write bytes per tcgen05 GEMM launch, averaged over the 33 GEMM
+# launches of one forward of this workload (8 x QKV, O, gate/up, down + LM
+# head), from ncu dram__bytes_read.sum + dram__bytes_write.sum at full size
+# (profiles/gemm_dram_traffic_byte_workload.md).  Equal to the algorithmic
+# bytes within 2%: no operand is re-read from DRAM.  Re-measure when the GEMM
+# kernel changes.
+GEMM_DRAM_BYTES_PER_LAUNCH = 3.089e9
 WORKLOAD = ("small byte-level masked DLM, bf16, 8 layers d=512 8 heads FFN 2048 V=256; 4 MiB order-2 "
             "Markov/Zipf(1.1) bytes; windows of 512 B, 1024 windows per batch, block 128, top-k 8 by "
             "confidence, 16-bit CDFs")
@@ -293,7 +300,8 @@ def run(args):
         "roofline": {"bound": "tensor", "kernel": "tcgen05 GEMM (all projections + LM head)",
                      "achieved": achieved, "peak": tf_sus, "unit": "TFLOP/s", "frac": achieved / tf_sus,
                      "peak_source": "%s bf16_tflops_sustained (kernel timed inside a long step)" % src,
-                     "traffic": None, "launches": int(g_n), "avg_launch_ms": g_ms / g_n if g_n else None},
+                     "traffic": GEMM_DRAM_BYTES_PER_LAUNCH, "traffic_unit": "bytes per launch (mean, ncu)",
+                     "launches": int(g_n), "avg_launch_ms": g_ms / g_n if g_n else None},
         "roofline_attention": {"bound": "tensor", "achieved": a_fl / (a_ms / 1000.0) / 1e12 if a_ms else 0.0,
                                "peak": tf_sus, "unit": "TFLOP/s",
                                "frac": (a_fl / (a_ms / 1000.0) / 1e12 / tf_sus) if a_ms else 0.0},
