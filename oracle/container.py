@@ -23,10 +23,12 @@ Details") are stored so the decompressor replays every decision.  Layout
      60   4  checksum: CRC-32 (IEEE) of the little-endian CRC-32s of the
              windows' input bytes, window by window
    version 2 only (initial context, Sec. 3.4: the visible symbols are stored):
-     64   4  context kind (1 = contiguous, 2 = random)
+     64   4  context kind (1 = contiguous, 2 = random, 3 = attention-based)
      68   4  c, context symbols per window
      72   8  seed of the random positions
-     80   -  the context symbols, window by window (min(c, window length) each,
+     80   -  kind 3 only: the context positions, window by window (min(c, window
+             length) each, ascending, u32)
+      -   -  the context symbols, window by window (min(c, window length) each,
              ascending position; 1 byte each when V <= 256, else u32)
       -   -  n_chunks LEB128 varints: bit length of each chunk's stream
       -   -  streams, chunk by chunk, ceil(bits / 8) bytes each
@@ -92,6 +94,7 @@ class Header:
     ctx_c: int = 0
     ctx_seed: int = 0
     ctx_data: bytes = b""
+    ctx_pos: bytes = b""
 
 
 def varint(n):
@@ -127,7 +130,7 @@ def write(h, streams):
         MAGIC, ver, h.coder, h.P, h.kind, h.fingerprint, h.vocab, h.chunk_len, h.batch_chunks, h.k,
         h.block, h.tau_q, h.k_min, h.k_max, h.n_symbols, h.n_chunks, h.crc32))
     if ver == VERSION_CONTEXT:
-        out += EXT.pack(h.ctx_kind, h.ctx_c, h.ctx_seed) + h.ctx_data
+        out += EXT.pack(h.ctx_kind, h.ctx_c, h.ctx_seed) + h.ctx_pos + h.ctx_data
     for bits, _ in streams:
         out += varint(bits)
     for bits, data in streams:
@@ -159,11 +162,17 @@ def read(buf):
             raise ContainerError("truncated header")
         h.ctx_kind, h.ctx_c, h.ctx_seed = EXT.unpack_from(buf, pos)
         pos += EXT.size
-        if h.ctx_kind not in (1, 2) or h.ctx_c == 0:
+        if h.ctx_kind not in (1, 2, 3) or h.ctx_c == 0:
             raise ContainerError("bad context")
         sb = 1 if h.vocab <= 256 else 4
         full, tail = divmod(h.n_symbols, h.chunk_len)
-        nb = sb * (full * min(h.ctx_c, h.chunk_len) + min(h.ctx_c, tail))
+        count = full * min(h.ctx_c, h.chunk_len) + min(h.ctx_c, tail)
+        if h.ctx_kind == 3:
+            if pos + 4 * count > len(buf):
+                raise ContainerError("truncated context")
+            h.ctx_pos = bytes(buf[pos:pos + 4 * count])
+            pos += 4 * count
+        nb = sb * count
         if pos + nb > len(buf):
             raise ContainerError("truncated context")
         h.ctx_data = bytes(buf[pos:pos + nb])

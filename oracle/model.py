@@ -142,9 +142,13 @@ def silu(x):
     return x / (1.0 + np.exp(-x))
 
 
-def attention(q, k, v, n_heads, n_kv_heads, head_dim):
-    """Bidirectional multi-head / grouped-query attention over one window."""
+def attention(q, k, v, n_heads, n_kv_heads, head_dim, probs=None):
+    """Bidirectional multi-head / grouped-query attention over one window.
+
+    ``probs`` (a list): receives the head-averaged attention probabilities [L, L].
+    """
     L = q.shape[0]
+    pavg = np.zeros((L, L)) if probs is not None else None
     group = n_heads // n_kv_heads
     out = np.empty((L, n_heads * head_dim))
     scale = 1.0 / np.sqrt(head_dim)
@@ -158,11 +162,18 @@ def attention(q, k, v, n_heads, n_kv_heads, head_dim):
         p = np.exp(s)
         p /= p.sum(axis=1, keepdims=True)
         out[:, h * head_dim:(h + 1) * head_dim] = p @ vg
+        if pavg is not None:
+            pavg += p / n_heads
+    if probs is not None:
+        probs.append(pavg)
     return out
 
 
-def hidden(wts, state):
-    """Final normed hidden states [L, d] (the LM head input) for one window."""
+def hidden(wts, state, probs=None):
+    """Final normed hidden states [L, d] (the LM head input) for one window.
+
+    ``probs`` (a list): receives each layer's head-averaged attention [L, L].
+    """
     cfg = wts.cfg
     rnd = lambda a: W.storage_round(a, cfg.dtype)
     r32 = W.round_f32
@@ -176,7 +187,7 @@ def hidden(wts, state):
         q = rnd(rope(q, cfg.n_heads, hd, cfg.rope_theta))
         k = rnd(rope(k, cfg.n_kv_heads, hd, cfg.rope_theta))
         v = rnd(v)
-        o = rnd(attention(q, k, v, cfg.n_heads, cfg.n_kv_heads, hd))
+        o = rnd(attention(q, k, v, cfg.n_heads, cfg.n_kv_heads, hd, probs))
         x = r32(x + o @ wts.layer(l, WO).T)
         h = rnd(rmsnorm(x, wts.g_ffn[l], cfg.norm_eps))
         a = rnd(silu(h @ wts.layer(l, WGATE).T) * (h @ wts.layer(l, WUP).T))

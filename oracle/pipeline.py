@@ -164,12 +164,16 @@ def compress(wts, data, chunk_len, policy, batch_chunks=1, context=(X.NONE, 0, 0
     nchunks = (n + chunk_len - 1) // chunk_len
     fn = model_logits_fn(wts)
     ckind, cc, cseed = context
-    if ckind not in (X.NONE, X.CONTIGUOUS, X.RANDOM) or cc < 0 or (ckind == X.NONE) != (cc == 0):
+    if ckind not in (X.NONE, X.CONTIGUOUS, X.RANDOM, X.ATTENTION) or cc < 0 or (ckind == X.NONE) != (cc == 0):
         raise BadInput("bad context")
-    streams, ctx_sym = [], []
+    streams, ctx_sym, ctx_pos = [], [], []
     for c in range(nchunks):
         win = sym[c * chunk_len:(c + 1) * chunk_len]
-        ctx = X.positions(ckind, cc, cseed, win.size, c)
+        if ckind == X.ATTENTION:
+            ctx = X.attention_positions(wts, win, cc)
+            ctx_pos.append(ctx)
+        else:
+            ctx = X.positions(ckind, cc, cseed, win.size, c)
         ctx_sym.append(win[ctx])
         if coder not in _ENC:
             raise BadInput("unknown coder")
@@ -182,7 +186,8 @@ def compress(wts, data, chunk_len, policy, batch_chunks=1, context=(X.NONE, 0, 0
                  n_symbols=n, n_chunks=nchunks,
                  crc32=C.window_checksum(bytes(data), chunk_len * (1 if V <= 256 else 4)),
                  coder=coder, ctx_kind=ckind, ctx_c=cc, ctx_seed=cseed,
-                 ctx_data=bytes_from_symbols(np.concatenate(ctx_sym) if ctx_sym else [], V))
+                 ctx_data=bytes_from_symbols(np.concatenate(ctx_sym) if ctx_sym else [], V),
+                 ctx_pos=np.concatenate(ctx_pos).astype("<u4").tobytes() if ctx_pos else b"")
     return C.write(h, streams)
 
 
@@ -204,10 +209,16 @@ def decompress(wts, blob):
     validate_policy(policy)
     fn = model_logits_fn(wts)
     ctx_all = symbols_from_bytes(h.ctx_data, cfg.vocab)
+    pos_all = np.frombuffer(h.ctx_pos, dtype="<u4").astype(np.int64)
     out, used = [], 0
     for c, st in enumerate(streams):
         n = min(h.chunk_len, h.n_symbols - c * h.chunk_len)
-        ctx = X.positions(h.ctx_kind, h.ctx_c, h.ctx_seed, n, c)
+        if h.ctx_kind == X.ATTENTION:
+            ctx = pos_all[used:used + min(h.ctx_c, n)]
+            if ctx.size and (ctx.max() >= n or np.any(np.diff(ctx) <= 0)):
+                raise C.ContainerError("bad context positions")
+        else:
+            ctx = X.positions(h.ctx_kind, h.ctx_c, h.ctx_seed, n, c)
         out.append(decode_window(st, n, cfg.vocab, fn, policy, h.P, ctx, ctx_all[used:used + ctx.size], h.coder))
         used += ctx.size
     sym = np.concatenate(out) if out else np.zeros(0, dtype=np.int64)
