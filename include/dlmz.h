@@ -98,6 +98,9 @@ DLMZ_API int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg);
 #define DLMZ_CONTEXT_CONTIGUOUS 1u /* the first c symbols of each window stay visible */
 #define DLMZ_CONTEXT_RANDOM 2u     /* c positions per window drawn from context_seed (SplitMix64,
                                       partial Fisher-Yates); symbols stored raw in the file */
+#define DLMZ_CONTEXT_ATTENTION 3u  /* attention-based (Sec. 3.4, policy 4): the c positions that masked tokens
+                                      attend to most (two complementary masked forwards, Attention Rollout);
+                                      positions and symbols stored in the file */
 
 typedef struct {
   uint32_t kind;
@@ -162,6 +165,16 @@ DLMZ_API int dlmz_decompress_device(const dlmz_model* m, const uint8_t* d_in, si
 DLMZ_API int dlmz_forward_logits(const dlmz_model* m, const int32_t* d_state, uint32_t n_chunks,
                         uint32_t L, uint32_t row0, uint32_t rows_per_chunk, float* d_logits,
                         void* stream);
+/* Attention-based context scores (Sec. 3.4, policy 4) of n_chunks windows of L
+ * symbols d_symbols [n_chunks x L] (int32, each < V): two forwards, one with
+ * the even and one with the odd positions masked; every layer's attention
+ * averaged over heads, A_l, and rolled out (Attention Rollout: R = Ã_N ... Ã_1,
+ * Ã_l = A_l / 2 + I / 2); d_scores [n_chunks x L] (float32) receives, for each
+ * position j, sum over the masked i of R[i, j] from the pass in which j is
+ * visible.  Compression keeps the c highest (ties: lower position).  Uses
+ * n_layers * n_chunks * L^2 * 4 bytes of device scratch.  Errors: EINVAL. */
+DLMZ_API int dlmz_context_scores(const dlmz_model* m, const int32_t* d_symbols, uint32_t n_chunks, uint32_t L,
+                                 float* d_scores, void* stream);
 
 /* Dense contraction of the forward (Definition 3's projections and LM head):
  * d_D [M x N] float32 = d_A [M x K] bf16 . d_B [N x K]^T bf16, all row-major

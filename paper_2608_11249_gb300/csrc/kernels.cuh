@@ -69,6 +69,11 @@ int swiglu(const float* gu, int T_tokens, int F, int gu_block, T* out, cudaStrea
 template <typename T>
 int attention_simt(const T* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                    int head_dim, int d, T* out, cudaStream_t s);
+// Head-averaged attention probabilities of every window [n_chunks][L][L] from the
+// RoPE'd Q and K of one layer (attention-based context, Sec. 3.4).
+template <typename T>
+int attention_maps(const T* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads, int head_dim, int d,
+                   float* maps, cudaStream_t s);
 bool attention_tc_supported(int L, int hd);
 int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int L, int n_heads, int n_kv_heads,
                       int head_dim, int d, bf16* out, cudaStream_t s);

@@ -133,9 +133,11 @@ static int gemm(const T* A, const T* B, int M, int N, int K, int epi, const Gemm
   return gemm_simt<T>(A, K, B, K, M, N, K, epi, ep, s);
 }
 
+// maps (optional): every layer's head-averaged attention [n_layers][nc][L][L]; without
+// logits the LM head is skipped.
 template <typename T>
 static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int row0, int rpc, float* logits,
-                        cudaStream_t s) {
+                        cudaStream_t s, float* maps = nullptr) {
   const dlmz_model_config& c = m->cfg;
   const int d = c.d, F = c.ffn, V = c.vocab, hd = m->hd, nq = m->nqkv;
   const int Tt = nc * L, R = nc * rpc;
@@ -210,6 +212,9 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
         ep.vt_rows = attention_vt_rows(hd);
       }
       DLMZ_TRY(gemm_bf16_tc(y, d, reinterpret_cast<const bf16*>(m->wqkv[l]), d, Tt, nq, d, EPI_ROPE_BF16, ep, s));
+      if (maps)
+        DLMZ_TRY(attention_maps<bf16>(reinterpret_cast<const bf16*>(qkv), nq, nc, L, c.n_heads, c.n_kv_heads, hd, d,
+                                      maps + (size_t)l * Tt * L, s));
       if (tc_attn)
         DLMZ_TRY(attention_bf16_tc(reinterpret_cast<const bf16*>(qkv), nq, w.vt.p, nc, L, c.n_heads,
                                    c.n_kv_heads, hd, d, reinterpret_cast<bf16*>(attn), s));
@@ -244,6 +249,7 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
       DLMZ_TRY(gemm<T>(h, reinterpret_cast<const T*>(m->wqkv[l]), Tt, nq, d, sizeof(T) == 2 ? EPI_BF16 : EPI_F32, ep,
                        s));
       DLMZ_TRY(rope_inplace<T>(qkv, Tt, nq, c.n_heads + c.n_kv_heads, hd, L, cs, s));
+      if (maps) DLMZ_TRY(attention_maps<T>(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, maps + (size_t)l * Tt * L, s));
       if constexpr (sizeof(T) == 2) {
         if (hd == 64 || hd == 128)
           DLMZ_TRY(attention_bf16_mma(qkv, nq, nc, L, c.n_heads, c.n_kv_heads, hd, d, attn, s));
@@ -262,10 +268,17 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
       DLMZ_TRY(gemm<T>(act, reinterpret_cast<const T*>(m->wdown[l]), Tt, d, F, EPI_RESID_F32, ep, s));
     }
   }
+  if (!logits) return DLMZ_OK;
   T* hc = w.hc.as<T>();
   DLMZ_TRY(rmsnorm<T>(x, R, d, m->gains, c.norm_eps, hc, L, row0, rpc, s));
   ep = epi(logits, V);
   return gemm<T>(hc, reinterpret_cast<const T*>(m->head), R, V, d, EPI_F32, ep, s);
+}
+
+int model_attention_maps(dlmz_model* m, const int32_t* state, int nc, int L, float* maps, cudaStream_t s) {
+  if (nc <= 0 || L <= 0 || !maps) return DLMZ_EINVAL;
+  if (m->bf16) return forward_impl<bf16>(m, state, nc, L, 0, 1, nullptr, s, maps);
+  return forward_impl<float>(m, state, nc, L, 0, 1, nullptr, s, maps);
 }
 
 int model_forward(dlmz_model* m, const int32_t* state, int nc, int L, int row0, int rpc, float* logits,

@@ -63,6 +63,13 @@ namespace dlmz {
 // [row0, row0+rpc) of every window.
 int model_forward(dlmz_model* m, const int32_t* state, int n_chunks, int L, int row0, int rpc, float* logits,
                   cudaStream_t s);
+// Every layer's head-averaged attention probabilities [n_layers][n_chunks][L][L]
+// for the windows' states (no LM head).
+int model_attention_maps(dlmz_model* m, const int32_t* state, int n_chunks, int L, float* maps, cudaStream_t s);
+// Attention-based context scores [n_chunks][L] of the windows' symbols (Sec. 3.4):
+// two masked passes, Attention Rollout; maps and state are scratch.
+int context_attention_scores(dlmz_model* m, const int32_t* symbols, int n_chunks, int L, float* scores, DevBuf& maps,
+                             DevBuf& state, cudaStream_t s);
 // Frees the pipeline workspace attached to the model (pipeline.cu).
 void pipeline_release(dlmz_model* m);
 // Bytes of forward workspace per token (for batch sizing).

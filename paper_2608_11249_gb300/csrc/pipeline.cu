@@ -337,7 +337,7 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
 
 static int validate_policy(const dlmz_k_policy* p) {
   if (!p) return DLMZ_EINVAL;
-  if (p->context > DLMZ_CONTEXT_RANDOM || (p->context == DLMZ_CONTEXT_NONE) != (p->context_c == 0) ||
+  if (p->context > DLMZ_CONTEXT_ATTENTION || (p->context == DLMZ_CONTEXT_NONE) != (p->context_c == 0) ||
       p->coder > DLMZ_CODER_RANKS)
     return DLMZ_EINVAL;
   if (p->kind == DLMZ_TOPK_CONF || p->kind == DLMZ_UNIFORM) return p->k >= 1 ? DLMZ_OK : DLMZ_EINVAL;
@@ -455,9 +455,11 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
 struct PipeWs {
   StepBufs sb;
   DevBuf symbols, state, cst, staging, bits, crcs, offsets, hin, hout, ctxpos, ctxsyms;
+  DevBuf ctxscore, ctxkeys, ctxsel, ctxmaps, ctxstate;  // attention-based context
   void release() {
     sb.release(); symbols.release(); state.release(); cst.release(); staging.release(); bits.release();
     crcs.release(); offsets.release(); hin.release(); hout.release(); ctxpos.release(); ctxsyms.release();
+    ctxscore.release(); ctxkeys.release(); ctxsel.release(); ctxmaps.release(); ctxstate.release();
   }
 };
 
@@ -487,13 +489,16 @@ struct Header {
   uint32_t ctx_kind = 0, ctx_c = 0;  // version 2: initial context (Sec. 3.4)
   uint64_t ctx_seed = 0;
   size_t size() const { return ctx_c ? 80 : 64; }
-  // bytes of the stored context symbols (after the header)
-  uint64_t ctx_bytes() const {
+  // context symbols over all windows
+  uint64_t ctx_count() const {
     if (!ctx_c || !chunk_len) return 0;
     const uint64_t full = n_symbols / chunk_len, tail = n_symbols % chunk_len;
     const uint64_t per = ctx_c < chunk_len ? ctx_c : chunk_len;
-    return (full * per + (ctx_c < tail ? ctx_c : tail)) * (vocab > 256 ? 4 : 1);
+    return full * per + (ctx_c < tail ? ctx_c : tail);
   }
+  // bytes of the stored context positions (attention-based context only) and symbols, after the header
+  uint64_t ctx_pos_bytes() const { return ctx_kind == DLMZ_CONTEXT_ATTENTION ? 4 * ctx_count() : 0; }
+  uint64_t ctx_bytes() const { return ctx_pos_bytes() + ctx_count() * (vocab > 256 ? 4 : 1); }
 };
 
 static void put32(uint8_t* p, uint32_t v) { for (int i = 0; i < 4; ++i) p[i] = (uint8_t)(v >> (8 * i)); }
@@ -553,7 +558,7 @@ static int read_header(const uint8_t* o, size_t n, Header& h) {
     h.ctx_kind = get32(o + 64);
     h.ctx_c = get32(o + 68);
     h.ctx_seed = get64(o + 72);
-    if ((h.ctx_kind != DLMZ_CONTEXT_CONTIGUOUS && h.ctx_kind != DLMZ_CONTEXT_RANDOM) || h.ctx_c == 0)
+    if (h.ctx_kind < DLMZ_CONTEXT_CONTIGUOUS || h.ctx_kind > DLMZ_CONTEXT_ATTENTION || h.ctx_c == 0)
       return DLMZ_ECORRUPT;
   }
   return DLMZ_OK;
@@ -561,16 +566,22 @@ static int read_header(const uint8_t* o, size_t n, Header& h) {
 
 // The batch's context: positions (host + device) and where its symbols are in the file.
 static int batch_context(const dlmz_k_policy& pol, int c0, int nc, int Lb, int sb, DevBuf& dpos, uint64_t sym_off,
-                         const uint8_t* file, uint8_t* out, cudaStream_t s, BatchContext& bx) {
+                         const uint8_t* file, uint8_t* out, cudaStream_t s, BatchContext& bx,
+                         const int32_t* attn_pos = nullptr) {
   bx = BatchContext{};
   bx.ce = context_count(pol, Lb);
   bx.sb = sb;
   if (bx.ce == 0) return DLMZ_OK;
   bx.file_syms = file ? file + sym_off * sb : nullptr;
   bx.out_syms = out ? out + sym_off * sb : nullptr;
-  if (pol.context == DLMZ_CONTEXT_RANDOM) {
+  if (pol.context == DLMZ_CONTEXT_RANDOM || pol.context == DLMZ_CONTEXT_ATTENTION) {
     bx.pos.resize((size_t)nc * bx.ce);
-    for (int w = 0; w < nc; ++w) context_positions(pol, Lb, (uint64_t)(c0 + w), bx.pos.data() + (size_t)w * bx.ce);
+    if (pol.context == DLMZ_CONTEXT_RANDOM) {
+      for (int w = 0; w < nc; ++w) context_positions(pol, Lb, (uint64_t)(c0 + w), bx.pos.data() + (size_t)w * bx.ce);
+    } else {  // attention-based: given by the caller (chosen on the device, or read from the file)
+      if (!attn_pos) return DLMZ_EINVAL;
+      std::copy(attn_pos, attn_pos + bx.pos.size(), bx.pos.begin());
+    }
     DLMZ_TRY(dpos.ensure(bx.pos.size() * 4));
     DLMZ_CUDA_TRY(cudaMemcpyAsync(dpos.p, bx.pos.data(), bx.pos.size() * 4, cudaMemcpyHostToDevice, s));
     bx.d_pos = dpos.as<int32_t>();
@@ -596,6 +607,41 @@ static std::vector<BatchPlan> plan_batches(uint64_t n_sym, uint32_t L, int bc) {
   for (uint64_t c = 0; c < nfull; c += bc) v.push_back({(int)c, (int)(nfull - c < (uint64_t)bc ? nfull - c : bc), (int)L});
   if (n_sym % L) v.push_back({(int)nfull, 1, (int)(n_sym % L)});
   return v;
+}
+
+// larger score -> smaller key (scores are >= 0), equal scores -> equal keys (the lower position wins)
+__global__ void score_keys_kernel(const float* scores, int64_t n, uint64_t* keys) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    keys[i] = (uint64_t)(~(__float_as_uint(fmaxf(scores[i], 0.f)) | 0x80000000u));
+}
+
+// Attention-based context of windows [0, nc) of length Lb: the ce highest-scoring
+// positions of each, ascending, to host `pos` [nc x ce].  Scored in sub-batches so
+// the attention maps stay near 2 GB.
+static int attention_context(dlmz_model* m, const int32_t* symbols, int nc, int Lb, int ce, PipeWs& w,
+                             std::vector<int32_t>& pos, cudaStream_t s) {
+  pos.assign((size_t)nc * ce, 0);
+  if (ce == 0 || nc == 0) return DLMZ_OK;
+  const size_t per = (size_t)m->cfg.n_layers * Lb * Lb * 4;
+  int sub = (int)std::max<size_t>(1, ((size_t)2 << 30) / per);
+  if (sub > nc) sub = nc;
+  DLMZ_TRY(w.ctxscore.ensure((size_t)nc * Lb * 4));
+  DLMZ_TRY(w.ctxkeys.ensure((size_t)nc * Lb * 8));
+  DLMZ_TRY(w.ctxsel.ensure((size_t)nc * ce * 4 + (size_t)nc * 4));
+  for (int c0 = 0; c0 < nc; c0 += sub) {
+    const int n = std::min(sub, nc - c0);
+    DLMZ_TRY(context_attention_scores(m, symbols + (size_t)c0 * Lb, n, Lb, w.ctxscore.as<float>() + (size_t)c0 * Lb,
+                                      w.ctxmaps, w.ctxstate, s));
+  }
+  const int64_t n = (int64_t)nc * Lb;
+  score_keys_kernel<<<grid_for(n), 256, 0, s>>>(w.ctxscore.as<float>(), n, w.ctxkeys.as<uint64_t>());
+  DLMZ_TRY(launch_status());
+  int32_t* sel = w.ctxsel.as<int32_t>();
+  DLMZ_TRY(select_rows<uint64_t>(nullptr, nc, Lb, -1, 0, Lb, w.ctxkeys.as<uint64_t>(), 0, ce, 0, 0, 0, ce,
+                                 sel + (size_t)nc * ce, sel, s));
+  DLMZ_CUDA_TRY(cudaMemcpyAsync(pos.data(), sel, pos.size() * 4, cudaMemcpyDeviceToHost, s));
+  DLMZ_CUDA_TRY(cudaStreamSynchronize(s));
+  return DLMZ_OK;
 }
 
 static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, uint32_t L, const dlmz_k_policy* pol,
@@ -637,10 +683,11 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
   h.chunk_len = L;
   h.n_symbols = n_sym;
   h.vocab = V;
-  const uint64_t ctx_bytes = h.ctx_bytes();
+  const uint64_t ctx_bytes = h.ctx_bytes(), ctx_pos_bytes = h.ctx_pos_bytes();
   const int sbytes = tok ? 4 : 1;
   DLMZ_TRY(w.ctxsyms.ensure(ctx_bytes + 16));
   const uint64_t ce_full = (uint64_t)context_count(*pol, (int)L);
+  std::vector<uint8_t> all_pos(ctx_pos_bytes);  // attention-based context: positions of every window, u32 LE
   for (const BatchPlan& b : plan_batches(n_sym, L, bc)) {
     const int64_t nsym_b = (int64_t)b.nc * b.L;
     symbols_in_kernel<<<grid_for(nsym_b), 256, 0, s>>>(d_in, (int64_t)b.c0 * L, nsym_b, tok, (int)V,
@@ -648,8 +695,13 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
     DLMZ_TRY(launch_status());
     uint8_t* eb = w.staging.as<uint8_t>() + (size_t)b.c0 * cap;
     BatchContext bx;
+    std::vector<int32_t> apos;
+    if (pol->context == DLMZ_CONTEXT_ATTENTION) {
+      DLMZ_TRY(attention_context(m, w.symbols.as<int32_t>(), b.nc, b.L, context_count(*pol, b.L), w, apos, s));
+      for (size_t i = 0; i < apos.size(); ++i) put32(all_pos.data() + 4 * ((uint64_t)b.c0 * ce_full + i), (uint32_t)apos[i]);
+    }
     DLMZ_TRY(batch_context(*pol, b.c0, b.nc, b.L, sbytes, w.ctxpos, (uint64_t)b.c0 * ce_full, nullptr,
-                           w.ctxsyms.as<uint8_t>(), s, bx));
+                           w.ctxsyms.as<uint8_t>() + ctx_pos_bytes, s, bx, apos.data()));
     DLMZ_TRY(run_batch(m, w.sb, *pol, b.nc, b.L, w.symbols.as<int32_t>(), w.state.as<int32_t>(),
                        w.cst.as<CoderState>(), eb, cap, nullptr, nullptr, nullptr, false, bx, s));
     DLMZ_TRY(coder_finish(w.cst.as<CoderState>(), b.nc, eb, cap, w.bits.as<uint32_t>() + b.c0, nullptr, nullptr,
@@ -688,8 +740,11 @@ static int compress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes, 
   if (pos > out_cap) return DLMZ_ECAPACITY;
   if (!d_out) return DLMZ_EINVAL;
   DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out, head.data(), head.size(), cudaMemcpyHostToDevice, s));
-  if (ctx_bytes)
-    DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out + head.size(), w.ctxsyms.p, ctx_bytes, cudaMemcpyDeviceToDevice, s));
+  if (ctx_pos_bytes)
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out + head.size(), all_pos.data(), ctx_pos_bytes, cudaMemcpyHostToDevice, s));
+  if (ctx_bytes > ctx_pos_bytes)
+    DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out + head.size() + ctx_pos_bytes, w.ctxsyms.as<uint8_t>() + ctx_pos_bytes,
+                                  ctx_bytes - ctx_pos_bytes, cudaMemcpyDeviceToDevice, s));
   if (!lens.empty())
     DLMZ_CUDA_TRY(cudaMemcpyAsync(d_out + head.size() + ctx_bytes, lens.data(), lens.size(), cudaMemcpyHostToDevice, s));
   if (n_chunks) {
@@ -775,10 +830,23 @@ static int decompress_device(dlmz_model* m, const uint8_t* d_in, size_t in_bytes
   DLMZ_TRY(w.state.ensure(bl * 4));
   DLMZ_TRY(w.cst.ensure((size_t)bc * sizeof(CoderState)));
   const uint64_t ce_full = (uint64_t)context_count(pol, (int)L);
+  const uint64_t ctx_pos_bytes = h.ctx_pos_bytes();
+  std::vector<uint8_t> all_pos(ctx_pos_bytes);
+  if (ctx_pos_bytes) DLMZ_CUDA_TRY(cudaMemcpy(all_pos.data(), d_in + hsize, ctx_pos_bytes, cudaMemcpyDeviceToHost));
   for (const BatchPlan& b : plan_batches(h.n_symbols, L, bc)) {
     BatchContext bx;
-    DLMZ_TRY(batch_context(pol, b.c0, b.nc, b.L, tok ? 4 : 1, w.ctxpos, (uint64_t)b.c0 * ce_full, d_in + hsize,
-                           nullptr, s, bx));
+    std::vector<int32_t> apos;
+    if (ctx_pos_bytes) {  // positions of the batch's windows: ascending, inside the window
+      const int ce = context_count(pol, b.L);
+      apos.resize((size_t)b.nc * ce);
+      for (size_t i = 0; i < apos.size(); ++i) {
+        const uint32_t p = get32(all_pos.data() + 4 * ((uint64_t)b.c0 * ce_full + i));
+        if (p >= (uint32_t)b.L || (i % ce && (int32_t)p <= apos[i - 1])) return DLMZ_ECORRUPT;
+        apos[i] = (int32_t)p;
+      }
+    }
+    DLMZ_TRY(batch_context(pol, b.c0, b.nc, b.L, tok ? 4 : 1, w.ctxpos, (uint64_t)b.c0 * ce_full,
+                           d_in + hsize + ctx_pos_bytes, nullptr, s, bx, apos.data()));
     DLMZ_TRY(run_batch(m, w.sb, pol, b.nc, b.L, nullptr, w.state.as<int32_t>(), w.cst.as<CoderState>(), nullptr, 0,
                        d_in, w.offsets.as<uint64_t>() + b.c0, w.bits.as<uint32_t>() + b.c0, true, bx, s));
     const int64_t nsym_b = (int64_t)b.nc * b.L;
@@ -919,6 +987,15 @@ int dlmz_forward_logits(const dlmz_model* m, const int32_t* d_state, uint32_t n_
   if (!device_error_word()) return DLMZ_ENOMEM;
   return model_forward(const_cast<dlmz_model*>(m), d_state, (int)n_chunks, (int)L, (int)row0, (int)rows_per_chunk,
                        d_logits, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_context_scores(const dlmz_model* mc, const int32_t* d_symbols, uint32_t n_chunks, uint32_t L,
+                        float* d_scores, void* stream) {
+  dlmz_model* m = const_cast<dlmz_model*>(mc);
+  if (!m || !d_symbols || !d_scores || !L || n_chunks > 0x7fffffffu) return DLMZ_EINVAL;
+  PipeWs& w = pipe_of(m);
+  return context_attention_scores(m, d_symbols, (int)n_chunks, (int)L, d_scores, w.ctxmaps, w.ctxstate,
+                                  reinterpret_cast<cudaStream_t>(stream));
 }
 
 int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32_t M, uint32_t N, uint32_t K, void* stream) {

@@ -21,7 +21,7 @@ lib = ctypes.CDLL(_LIB_PATH)
 OK, EINVAL, EBADINPUT, ECORRUPT, EMODEL, ENOMEM, ECUDA, ETIMEOUT, ECAPACITY = 0, -1, -2, -3, -4, -5, -6, -7, -8
 FP32, BF16 = 0, 1
 TOPK_CONF, ENTROPY, UNIFORM, PROGRESSIVE = 0, 1, 2, 3
-CONTEXT_NONE, CONTEXT_CONTIGUOUS, CONTEXT_RANDOM = 0, 1, 2
+CONTEXT_NONE, CONTEXT_CONTIGUOUS, CONTEXT_RANDOM, CONTEXT_ATTENTION = 0, 1, 2, 3
 CODER_RANGE, CODER_RANS, CODER_RANKS = 0, 1, 2
 
 
@@ -71,6 +71,7 @@ _sig("dlmz_compress_device", c_int, _P, _P, c_size_t, c_uint32, POINTER(KPolicy)
      POINTER(c_size_t), _P)
 _sig("dlmz_decompress_device", c_int, _P, _P, c_size_t, _P, c_size_t, POINTER(c_size_t), _P)
 _sig("dlmz_forward_logits", c_int, _P, _P, c_uint32, c_uint32, c_uint32, c_uint32, _P, _P)
+_sig("dlmz_context_scores", c_int, _P, _P, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_gemm_bf16", c_int, _P, _P, _P, c_uint32, c_uint32, c_uint32, _P)
 _sig("dlmz_quantize", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P, _P, _P, _P, _P)
 _sig("dlmz_select_smallest", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
@@ -167,6 +168,9 @@ class Model:
     def forward_logits(self, d_state, n_chunks, L, row0, rows_per_chunk, d_logits, stream=0):
         _ok(lib.dlmz_forward_logits(self.h, d_state, n_chunks, L, row0, rows_per_chunk, d_logits, stream),
             "dlmz_forward_logits")
+
+    def context_scores(self, d_symbols, n_chunks, L, d_scores, stream=0):
+        _ok(lib.dlmz_context_scores(self.h, d_symbols, n_chunks, L, d_scores, stream), "dlmz_context_scores")
 
 
 def gemm_bf16(d_A, d_B, d_D, M, N, K, stream=0):
