@@ -2,20 +2,18 @@
 // every position attends to every position of its window, no mask).
 //
 // Persistent CTAs (two per SM) walk work items (128 queries, head, window); 6 warps:
-//   warp 0      TMA: Q once; per key tile of 128: K (2-stage ring, requested
-//               one tile ahead of V) and V^T (keys contiguous, written so by
-//               the QKV epilogue; single buffer).
-//   warp 1      allocates 256 TMEM columns (S: 128, O: head_dim) and issues
-//               S_j = Q K_j^T and O += P_j V_j with tcgen05.mma from one thread.
+//   warp 0      TMA: Q once per item; per key tile of 128: K and V^T (keys
+//               contiguous, written so by the QKV epilogue), each through a
+//               2-stage ring, K requested one tile ahead of V.
+//   warp 1      allocates 256 TMEM columns (S: 128, P: 64, O: head_dim) and
+//               issues S_j = Q K_j^T (A and B in shared memory) and
+//               O += P_j V_j (A = P_j in TMEM) with tcgen05.mma from one thread.
 //   warps 2-5   softmax, one thread per query row (its TMEM lane): the row of
 //               S_j in one 128-column TMEM load, its max, P_j = 2^(S_j - m) by
-//               ex2.approx.f16x2 written to shared memory as f16 (the A operand
-//               of P V); the running max is raised (and O rescaled in TMEM)
-//               only when it grows by more than 8 (log2 units), so P <= 2^8;
-//               finally O / l -> bf16.
-// V^T (f16) carries an extra row of ones after the head dimensions (and 15
-// zero rows), so O's column head_dim accumulates the row sum l of P on the
-// tensor core, rescaled together with O.
+//               ex2.approx.f16x2, stored back to TMEM as f16 pairs (the A
+//               operand of P V), and the row sum l of those f16 values; the
+//               running max is raised (and O and l rescaled) only when it grows
+//               by more than 8 (log2 units), so P <= 2^8; finally O / l -> bf16.
 // GQA: query head h reads KV head h / (n_heads / n_kv_heads).  Requires the
 // window length to be a multiple of 128.  All waits are bounded.
 #include "kernels.cuh"
@@ -28,36 +26,57 @@ constexpr int BQ = 128, BK = 128;
 constexpr int THREADS = 192;
 constexpr int TMEM_COLS = 256;
 constexpr float RESCALE_THRESHOLD = 8.0f;
-constexpr int VT_EXTRA = 16;  // ones row + zero rows appended to V^T
 
 template <int HD>
 struct Smem {
-  static constexpr int HDP = HD + VT_EXTRA;
-  static constexpr int Q = 0;                        // HD/64 blocks of [128 x 64] bf16
-  static constexpr int KT = BK * HD * 2;             // one key tile: HD/64 blocks of [128 x 64]
+  static_assert(HD == 64, "one 128-byte swizzle row per Q / K row");
+  static constexpr int Q = 0;                        // [128 x 64] bf16
+  static constexpr int KT = BK * HD * 2;             // one key tile [128 x 64] bf16
   static constexpr int K = Q + BQ * HD * 2;          // 2 key tiles
-  static constexpr int VT = K + 2 * KT;              // 2 blocks of [HDP x 64] f16 (keys 0-63, 64-127)
-  static constexpr int P = VT + HDP * BK * 2;        // 2 blocks of [128 x 64] f16
-  static constexpr int BARS = P + BQ * BK * 2;
-  static constexpr int TOTAL = BARS + 128 + 1024;    // + barriers + alignment slack
+  static constexpr int VTT = HD * BK * 2;            // one V^T tile: 2 blocks of [HD x 64] f16 (keys 0-63, 64-127)
+  static constexpr int VT = K + 2 * KT;              // 2 V^T tiles
+  static constexpr int BARS = VT + 2 * VTT;
+  static constexpr int TOTAL = BARS + 256 + 1024;    // + barriers + alignment slack
 };
+
+// Row sum of 128 f16 values held as 64 pairs: two levels of f16x2 adds (partial
+// sums of at most 4 values <= 2^8 each), then f32.
+__device__ __forceinline__ float row_sum_f16x2(const uint32_t* p) {
+  uint32_t t[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    uint32_t a, b;
+    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(a) : "r"(p[i]), "r"(p[i + 16]));
+    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(b) : "r"(p[i + 32]), "r"(p[i + 48]));
+    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(t[i]) : "r"(a), "r"(b));
+  }
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const __half2 h = *reinterpret_cast<const __half2*>(&t[i]);
+    const float2 f = __half22float2(h);
+    acc[i & 3] += f.x + f.y;
+  }
+  return (acc[0] + acc[1]) + (acc[2] + acc[3]);
+}
 
 template <int HD>
 __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 registers per thread
     fa_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt, int n_chunks,
                  int L, int nh, int nkv, int d, bf16* __restrict__ out, float scale_log2, int* err) {
   using S = Smem<HD>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
-  const uint32_t base = smem_u32(sm);
-  const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT, sP = base + S::P;
+  const uint32_t base = (smem_u32(smem_raw) + 1023) & ~1023u;
+  const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT;
   const uint32_t bar = base + S::BARS;
-  const uint32_t q_full = bar, v_full = bar + 24, v_empty = bar + 32, s_full = bar + 40, p_ready = bar + 48,
-                 o_done = bar + 56, s_free = bar + 96, q_empty = bar + 104, o_free = bar + 112;
-  auto k_full = [&](int st) { return st ? bar + 72 : bar + 8; };   // per key stage
-  auto k_empty = [&](int st) { return st ? bar + 80 : bar + 16; };
+  const uint32_t q_full = bar, q_empty = bar + 8, s_full = bar + 80, s_free = bar + 88, p_ready = bar + 96,
+                 o_done = bar + 104, o_free = bar + 112;
+  auto k_full = [&](int st) { return bar + 16 + 8 * st; };   // per key stage
+  auto k_empty = [&](int st) { return bar + 32 + 8 * st; };
+  auto v_full = [&](int st) { return bar + 48 + 8 * st; };   // per V^T stage
+  auto v_empty = [&](int st) { return bar + 64 + 8 * st; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nt = L / BK, nqt = L / BQ;
   // work items (query tile, head, window), query tile fastest; this CTA takes
@@ -80,12 +99,12 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
     for (int st = 0; st < 2; ++st) {
       mbar_init(k_full(st), 1);
       mbar_init(k_empty(st), 1);
+      mbar_init(v_full(st), 1);
+      mbar_init(v_empty(st), 1);
     }
-    mbar_init(v_full, 1);
-    mbar_init(v_empty, 1);
     mbar_init(s_full, 1);
-    mbar_init(p_ready, 4 * 32);
     mbar_init(s_free, 4 * 32);
+    mbar_init(p_ready, 4 * 32);
     mbar_init(o_done, 1);
     mbar_init(o_free, 4 * 32);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -95,16 +114,14 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
   __syncthreads();
   t5::fence_after();
   const uint32_t tmem = tmem_slot;
-  const uint32_t tS = tmem, tO = tmem + BK;
-  constexpr int HDP = S::HDP;
+  const uint32_t tS = tmem, tP = tmem + BK, tO = tmem + BK + BK / 2;
 
   if (warp == 0) {
     if (lane == 0) {
-      uint32_t kpend = 0, kpar0 = 0, kpar1 = 0, vp = 0;
-      bool v_pend = false, q_pend = false;
+      uint32_t kpend = 0, vpend = 0, kpar = 0, vpar = 0;  // per stage (bit): copy issued, its phase
+      bool q_pend = false;
       uint32_t qp = 0;
-      // per global tile J: (item's Q when J starts an item), K_J, then V_{J-1};
-      // K runs one tile ahead of V through its 2-stage ring
+      // per global tile J: (item's Q when J starts an item), K_J, then V_{J-1}
       for (int J = 0; J <= total && !abort_flag; ++J) {
         if (J < total) {
           const int it = J / nt, j = J % nt;
@@ -126,34 +143,37 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
           for (int kb = 0; kb < HD / 64; ++kb)
             t5::tma_load_2d(sK + st * S::KT + kb * BK * 128, &tmQK, d + g * HD + kb * 64, w * L + j * BK, k_full(st));
           kpend |= 1u << st;
-          if (st) kpar1 = ph;
-          else kpar0 = ph;
+          kpar = (kpar & ~(1u << st)) | (ph << st);
         }
         if (J >= 1) {
           const int Jv = J - 1, it = Jv / nt, j = Jv % nt;
           int w, h, q0;
           item_of(it, w, h, q0);
           const int g = h / (nh / nkv);
-          if (!mbar_wait_bounded(v_empty, (Jv & 1) ^ 1, &abort_flag, err)) break;
-          mbar_arrive_expect_tx(v_full, BK * HDP * 2);
+          const int st = Jv & 1;
+          const uint32_t ph = (Jv >> 1) & 1;
+          if (!mbar_wait_bounded(v_empty(st), ph ^ 1, &abort_flag, err)) break;
+          mbar_arrive_expect_tx(v_full(st), BK * HD * 2);
           for (int kk = 0; kk < 2; ++kk)
-            t5::tma_load_2d(sVt + kk * HDP * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HDP, v_full);
-          v_pend = true;
-          vp = Jv & 1;
+            t5::tma_load_2d(sVt + st * S::VTT + kk * HD * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HD,
+                            v_full(st));
+          vpend |= 1u << st;
+          vpar = (vpar & ~(1u << st)) | (ph << st);
         }
       }
       if (abort_flag) {  // let our own copies land before the CTA can exit
         volatile int never = 0;
         if (q_pend) mbar_wait_bounded(q_full, qp, &never, err, 100000000ull);
-        if (kpend & 1u) mbar_wait_bounded(k_full(0), kpar0, &never, err, 100000000ull);
-        if (kpend & 2u) mbar_wait_bounded(k_full(1), kpar1, &never, err, 100000000ull);
-        if (v_pend) mbar_wait_bounded(v_full, vp, &never, err, 100000000ull);
+        for (int st = 0; st < 2; ++st) {
+          if (kpend & (1u << st)) mbar_wait_bounded(k_full(st), (kpar >> st) & 1, &never, err, 100000000ull);
+          if (vpend & (1u << st)) mbar_wait_bounded(v_full(st), (vpar >> st) & 1, &never, err, 100000000ull);
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
-      constexpr uint32_t ID_O = t5::idesc_f16(BQ, HDP);
+      constexpr uint32_t ID_O = t5::idesc_f16(BQ, HD);
       bool issued = false;
       // S_J = Q K_J^T; the first tile of an item waits for that item's Q, the
       // last one releases Q to the next item's load
@@ -175,7 +195,7 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       };
       bool ok = total == 0 || issue_s(0);
       for (int J = 0; ok && J < total; ++J) {
-        const int it = J / nt, j = J % nt;
+        const int it = J / nt, j = J % nt, st = J & 1;
         // S_{J+1} goes as soon as the softmax has S_J in registers, so it runs under P_J's exponentials
         // (across items too: the next item's first QK^T overlaps this item's last softmax and epilogue)
         if (J + 1 < total) {
@@ -183,22 +203,21 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
           if (!issue_s(J + 1)) break;
         }
         if (!mbar_wait_bounded(p_ready, J & 1, &abort_flag, err)) break;
-        if (!mbar_wait_bounded(v_full, J & 1, &abort_flag, err)) break;
+        if (!mbar_wait_bounded(v_full(st), (J >> 1) & 1, &abort_flag, err)) break;
         // the first PV of an item overwrites O: the softmax warps must have read the previous item's O
         if (j == 0 && it > 0 && !mbar_wait_bounded(o_free, (it - 1) & 1, &abort_flag, err)) break;
         t5::fence_after();
+        // 8 steps of 16 keys: P_j columns 8k..8k+7, V^T block k / 4 at byte offset 32 (k % 4)
 #pragma unroll
-        for (int kk = 0; kk < 2; ++kk)
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            t5::mma_bf16(tO, t5::sw128_desc(sP + kk * BQ * 128 + 32 * k), t5::sw128_desc(sVt + kk * HDP * 128 + 32 * k),
-                         ID_O, (j | kk | k) != 0);
-        t5::commit(v_empty);
+        for (int k = 0; k < BK / 16; ++k)
+          t5::mma_tmem_a(tO, tP + 8 * k, t5::sw128_desc(sVt + st * S::VTT + (k >> 2) * HD * 128 + 32 * (k & 3)),
+                         ID_O, (j | k) != 0);
+        t5::commit(v_empty(st));
         t5::commit(o_done);
       }
       if (abort_flag && issued) {
         volatile int never = 0;
-        const uint32_t drain = bar + 88;
+        const uint32_t drain = bar + 120;
         mbar_init(drain, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         t5::commit(drain);
@@ -209,7 +228,7 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
     const int q = warp & 3;
     const int r = q * 32 + lane;  // query row within the tile (= TMEM lane)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    float m = -INFINITY;
+    float m = -INFINITY, l = 0.0f;
     for (int J = 0; J < total; ++J) {
       const int j = J % nt;
       // waits are made warp-uniform: tcgen05.ld/st below are warp-collective
@@ -227,25 +246,27 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       // the running max first (P needs only m); P_J is computed in registers while PV_{J-1} may still run
       float f = 1.0f;
       bool need = false;
-      if (j == 0) {  // P buffer and O were released by this item's predecessor's epilogue
+      if (j == 0) {  // P and O were released by this item's predecessor's epilogue
         m = mx;
+        l = 0.0f;
       } else if (mx > m + RESCALE_THRESHOLD) {
         need = true;
         f = t5::ex2(m - mx);
         m = mx;
       }
-      // P = 2^(s * scale - m) as f16 pairs (in place of S)
+      // P = 2^(s * scale - m) as f16 pairs (in place of S): pair c holds keys 2c, 2c + 1
 #pragma unroll
       for (int c = 0; c < BK / 2; ++c)
         sr[c] = t5::ex2_f16x2(t5::pack_f16x2(fmaf(__uint_as_float(sr[2 * c]), scale_log2, -m),
                                              fmaf(__uint_as_float(sr[2 * c + 1]), scale_log2, -m)));
+      l = l * f + row_sum_f16x2(sr);
       if (j > 0) {
-        // PV_{J-1} done: P buffer free, O stable
+        // PV_{J-1} done: P's columns free, O stable
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (J - 1) & 1, &abort_flag, err))) break;
         t5::fence_after();
         if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
 #pragma unroll 1
-          for (int c = 0; c < HDP / 16; ++c) {
+          for (int c = 0; c < HD / 16; ++c) {
             uint32_t o[16];
             t5::tmem_ld16(tO + lane_off + c * 16, o);
 #pragma unroll
@@ -254,28 +275,19 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
           }
         }
       }
-      // 16-byte chunks of 8 keys, 128B-swizzled rows
-#pragma unroll
-      for (int cc = 0; cc < BK / 8; ++cc) {
-        const uint32_t a = sP + (cc >> 3) * BQ * 128 + r * 128 + (((cc & 7) ^ (r & 7)) << 4);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(sr[4 * cc]), "r"(sr[4 * cc + 1]),
-                     "r"(sr[4 * cc + 2]), "r"(sr[4 * cc + 3])
-                     : "memory");
-      }
-      t5::fence_proxy_async();
+      t5::tmem_st64(tP + lane_off, sr);
       t5::fence_before();
       mbar_arrive(p_ready);
       if (j == nt - 1) {  // this item's epilogue: O / l -> bf16
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, J & 1, &abort_flag, err))) break;
         t5::fence_after();
-        uint32_t o[HD], lsum[16];
+        uint32_t o[HD];
         t5::tmem_ld64(tO + lane_off, o);
-        t5::tmem_ld16(tO + lane_off + HD, lsum);
         t5::fence_before();
         mbar_arrive(o_free);  // O is in registers: the next item's first PV may overwrite it
         int w, h, q0;
         item_of(J / nt, w, h, q0);
-        const float inv = 1.0f / __uint_as_float(lsum[0]);
+        const float inv = 1.0f / l;
         bf16* dst = out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
         uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
@@ -304,26 +316,7 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
 
 bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 && hd == 64; }
 
-int attention_vt_rows(int hd) { return hd + fat::VT_EXTRA; }
-
-__global__ void vt_init_kernel(__half* vt, int blocks, int hd, int L) {
-  const int rows = hd + fat::VT_EXTRA;
-  const int64_t n = (int64_t)blocks * fat::VT_EXTRA * L;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t b = i / ((int64_t)fat::VT_EXTRA * L), rem = i % ((int64_t)fat::VT_EXTRA * L);
-    const int e = (int)(rem / L), p = (int)(rem % L);
-    vt[(b * rows + hd + e) * L + p] = __float2half(e == 0 ? 1.0f : 0.0f);
-  }
-}
-
-int attention_vt_init(void* vt, int blocks, int hd, int L, cudaStream_t s) {
-  const int64_t n = (int64_t)blocks * fat::VT_EXTRA * L;
-  if (n == 0) return DLMZ_OK;
-  int64_t g = (n + 255) / 256;
-  if (g > 65535) g = 65535;
-  vt_init_kernel<<<(unsigned)g, 256, 0, s>>>(reinterpret_cast<__half*>(vt), blocks, hd, L);
-  return launch_status();
-}
+int attention_vt_rows(int hd) { return hd; }
 
 int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int L, int nh, int nkv, int hd, int d,
                       bf16* out, cudaStream_t s) {
@@ -333,7 +326,7 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
     return DLMZ_EINVAL;
   CUtensorMap mqk, mvt;
   DLMZ_TRY(t5::make_map_bf16(&mqk, qkv, (uint64_t)n_chunks * L, ld, ld, 128, 64));
-  DLMZ_TRY(t5::make_map_f16(&mvt, vt, (uint64_t)n_chunks * nkv * (hd + fat::VT_EXTRA), L, L, hd + fat::VT_EXTRA, 64));
+  DLMZ_TRY(t5::make_map_f16(&mvt, vt, (uint64_t)n_chunks * nkv * hd, L, L, hd, 64));
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
   constexpr int SM = fat::Smem<64>::TOTAL;
   static bool attr = false;

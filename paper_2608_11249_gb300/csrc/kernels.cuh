@@ -77,10 +77,8 @@ int attention_maps(const T* qkv, int ld, int n_chunks, int L, int n_heads, int n
 bool attention_tc_supported(int L, int hd);
 int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int L, int n_heads, int n_kv_heads,
                       int head_dim, int d, bf16* out, cudaStream_t s);
-// Rows per (window, kv head) of the attention kernel's V^T buffer (head_dim + extra rows).
+// Rows per (window, kv head) of the attention kernel's V^T buffer.
 int attention_vt_rows(int head_dim);
-// Writes the extra rows of every (window, kv head) block of V^T: row head_dim = 1, the rest 0.
-int attention_vt_init(void* vt, int blocks, int head_dim, int L, cudaStream_t s);
 int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                        int head_dim, int d, bf16* out, cudaStream_t s);
 

@@ -154,12 +154,6 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
   if (tc_attn) {
     const int vrows = attention_vt_rows(hd), blocks = nc * (int)c.n_kv_heads;
     DLMZ_TRY(w.vt.ensure((size_t)blocks * vrows * L * 2));
-    if (w.vt_ptr != w.vt.p || w.vt_L != L || w.vt_blocks != blocks) {
-      DLMZ_TRY(attention_vt_init(w.vt.p, blocks, hd, L, s));
-      w.vt_ptr = w.vt.p;
-      w.vt_L = L;
-      w.vt_blocks = blocks;
-    }
   }
   if (w.rope_L < L) {  // (cos, sin) of pos * theta^(-2i/hd), from double precision
     const int half = hd / 2;

@@ -36,8 +36,6 @@ struct DevBuf {
 struct ForwardWorkspace {
   DevBuf x, h, qkv, attn, act, gu, hc, rope, vt, ssq;
   int rope_L = 0;
-  const void* vt_ptr = nullptr;  // layout for which V^T's constant rows were written
-  int vt_L = 0, vt_blocks = 0;
 };
 
 }  // namespace dlmz
