@@ -2,9 +2,10 @@
 // every position attends to every position of its window, no mask).
 //
 // Persistent CTAs (two per SM) walk work items (128 queries, head, window); 6 warps:
-//   warp 0      TMA: Q once per item; per key tile of 128: K and V^T (keys
-//               contiguous, written so by the QKV epilogue), each through a
-//               2-stage ring, K requested one tile ahead of V.
+//   warp 0      TMA: Q once per item (2-stage ring, so the next item's Q is
+//               in flight during this item); per key tile of 128: K and V^T
+//               (keys contiguous, written so by the QKV epilogue), each
+//               through a 2-stage ring, K requested one tile ahead of V.
 //   warp 1      allocates 256 TMEM columns (S: 128, P: 64, O: head_dim) and
 //               issues S_j = Q K_j^T (A and B in shared memory) and
 //               O += P_j V_j (A = P_j in TMEM) with tcgen05.mma from one thread.
@@ -30,34 +31,47 @@ constexpr float RESCALE_THRESHOLD = 8.0f;
 template <int HD>
 struct Smem {
   static_assert(HD == 64, "one 128-byte swizzle row per Q / K row");
-  static constexpr int Q = 0;                        // [128 x 64] bf16
+  static constexpr int QT = BQ * HD * 2;             // one query tile [128 x 64] bf16
+  static constexpr int Q = 0;                        // 2 query tiles
   static constexpr int KT = BK * HD * 2;             // one key tile [128 x 64] bf16
-  static constexpr int K = Q + BQ * HD * 2;          // 2 key tiles
+  static constexpr int K = Q + 2 * QT;               // 2 key tiles
   static constexpr int VTT = HD * BK * 2;            // one V^T tile: 2 blocks of [HD x 64] f16 (keys 0-63, 64-127)
   static constexpr int VT = K + 2 * KT;              // 2 V^T tiles
   static constexpr int BARS = VT + 2 * VTT;
   static constexpr int TOTAL = BARS + 256 + 1024;    // + barriers + alignment slack
 };
 
-// Row sum of 128 f16 values held as 64 pairs: two levels of f16x2 adds (partial
-// sums of at most 4 values <= 2^8 each), then f32.
+__device__ __forceinline__ uint32_t hadd2(uint32_t a, uint32_t b) {
+  uint32_t y;
+  asm("add.rn.f16x2 %0, %1, %2;" : "=r"(y) : "r"(a), "r"(b));
+  return y;
+}
+// Row sum of 128 f16 values held as 64 pairs: a pairwise f16x2 tree (every
+// partial sum <= 128 * 2^8 stays finite in f16), the last two lanes in f32.
 __device__ __forceinline__ float row_sum_f16x2(const uint32_t* p) {
-  uint32_t t[16];
+  uint32_t t[32];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    uint32_t a, b;
-    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(a) : "r"(p[i]), "r"(p[i + 16]));
-    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(b) : "r"(p[i + 32]), "r"(p[i + 48]));
-    asm("add.rn.f16x2 %0, %1, %2;" : "=r"(t[i]) : "r"(a), "r"(b));
-  }
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int i = 0; i < 32; ++i) t[i] = hadd2(p[i], p[i + 32]);
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const __half2 h = *reinterpret_cast<const __half2*>(&t[i]);
-    const float2 f = __half22float2(h);
-    acc[i & 3] += f.x + f.y;
-  }
-  return (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  for (int w = 16; w >= 1; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) t[i] = hadd2(t[i], t[i + w]);
+  const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&t[0]));
+  return f.x + f.y;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float y;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+  return y;
+}
+// (x0, x1) * (a0, a1) + (b0, b1) in one packed f32x2 FMA; each lane rounds as fmaf.
+__device__ __forceinline__ void fma2(float& y0, float& y1, float x0, float x1, float a0, float a1, float b0, float b1) {
+  uint64_t x, a, b, y;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(x) : "f"(x0), "f"(x1));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(a) : "f"(a0), "f"(a1));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(b) : "f"(b0), "f"(b1));
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(y) : "l"(x), "l"(a), "l"(b));
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(y0), "=f"(y1) : "l"(y));
 }
 
 template <int HD>
@@ -71,8 +85,9 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
   const uint32_t base = (smem_u32(smem_raw) + 1023) & ~1023u;
   const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT;
   const uint32_t bar = base + S::BARS;
-  const uint32_t q_full = bar, q_empty = bar + 8, s_full = bar + 80, s_free = bar + 88, p_ready = bar + 96,
-                 o_done = bar + 104, o_free = bar + 112;
+  const uint32_t s_full = bar + 80, s_free = bar + 88, p_ready = bar + 96, o_done = bar + 104, o_free = bar + 112;
+  auto q_full = [&](int st) { return bar + 128 + 8 * st; };  // per query stage
+  auto q_empty = [&](int st) { return bar + 144 + 8 * st; };
   auto k_full = [&](int st) { return bar + 16 + 8 * st; };   // per key stage
   auto k_empty = [&](int st) { return bar + 32 + 8 * st; };
   auto v_full = [&](int st) { return bar + 48 + 8 * st; };   // per V^T stage
@@ -94,9 +109,9 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
-    mbar_init(q_full, 1);
-    mbar_init(q_empty, 1);
     for (int st = 0; st < 2; ++st) {
+      mbar_init(q_full(st), 1);
+      mbar_init(q_empty(st), 1);
       mbar_init(k_full(st), 1);
       mbar_init(k_empty(st), 1);
       mbar_init(v_full(st), 1);
@@ -119,8 +134,7 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
   if (warp == 0) {
     if (lane == 0) {
       uint32_t kpend = 0, vpend = 0, kpar = 0, vpar = 0;  // per stage (bit): copy issued, its phase
-      bool q_pend = false;
-      uint32_t qp = 0;
+      uint32_t qpend = 0, qpar = 0;
       // per global tile J: (item's Q when J starts an item), K_J, then V_{J-1}
       for (int J = 0; J <= total && !abort_flag; ++J) {
         if (J < total) {
@@ -128,13 +142,15 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
           int w, h, q0;
           item_of(it, w, h, q0);
           const int g = h / (nh / nkv);
-          if (j == 0) {  // the previous item's last QK^T has read Q
-            if (it > 0 && !mbar_wait_bounded(q_empty, (it - 1) & 1, &abort_flag, err)) break;
-            mbar_arrive_expect_tx(q_full, BQ * HD * 2);
+          if (j == 0) {  // item it - 2's last QK^T has read this Q stage
+            const int qs = it & 1;
+            const uint32_t qph = (it >> 1) & 1;
+            if (!mbar_wait_bounded(q_empty(qs), qph ^ 1, &abort_flag, err)) break;
+            mbar_arrive_expect_tx(q_full(qs), BQ * HD * 2);
             for (int kb = 0; kb < HD / 64; ++kb)
-              t5::tma_load_2d(sQ + kb * BQ * 128, &tmQK, h * HD + kb * 64, w * L + q0, q_full);
-            q_pend = true;
-            qp = it & 1;
+              t5::tma_load_2d(sQ + qs * S::QT + kb * BQ * 128, &tmQK, h * HD + kb * 64, w * L + q0, q_full(qs));
+            qpend |= 1u << qs;
+            qpar = (qpar & ~(1u << qs)) | (qph << qs);
           }
           const int st = J & 1;
           const uint32_t ph = (J >> 1) & 1;
@@ -163,8 +179,8 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       }
       if (abort_flag) {  // let our own copies land before the CTA can exit
         volatile int never = 0;
-        if (q_pend) mbar_wait_bounded(q_full, qp, &never, err, 100000000ull);
         for (int st = 0; st < 2; ++st) {
+          if (qpend & (1u << st)) mbar_wait_bounded(q_full(st), (qpar >> st) & 1, &never, err, 100000000ull);
           if (kpend & (1u << st)) mbar_wait_bounded(k_full(st), (kpar >> st) & 1, &never, err, 100000000ull);
           if (vpend & (1u << st)) mbar_wait_bounded(v_full(st), (vpar >> st) & 1, &never, err, 100000000ull);
         }
@@ -178,18 +194,18 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       // S_J = Q K_J^T; the first tile of an item waits for that item's Q, the
       // last one releases Q to the next item's load
       auto issue_s = [&](int J) -> bool {
-        const int st = J & 1;
-        if (J % nt == 0 && !mbar_wait_bounded(q_full, (J / nt) & 1, &abort_flag, err)) return false;
+        const int st = J & 1, it = J / nt, qs = it & 1;
+        if (J % nt == 0 && !mbar_wait_bounded(q_full(qs), (it >> 1) & 1, &abort_flag, err)) return false;
         if (!mbar_wait_bounded(k_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
         t5::fence_after();
         for (int kb = 0; kb < HD / 64; ++kb)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            t5::mma_bf16(tS, t5::sw128_desc(sQ + kb * BQ * 128 + 32 * k),
+            t5::mma_bf16(tS, t5::sw128_desc(sQ + qs * S::QT + kb * BQ * 128 + 32 * k),
                          t5::sw128_desc(sK + st * S::KT + kb * BK * 128 + 32 * k), ID_S, (kb | k) != 0);
         t5::commit(s_full);
         t5::commit(k_empty(st));
-        if (J % nt == nt - 1) t5::commit(q_empty);
+        if (J % nt == nt - 1) t5::commit(q_empty(qs));
         issued = true;
         return true;
       };
@@ -240,7 +256,8 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       mbar_arrive(s_free);  // S_J is in registers: the MMA warp may overwrite it with S_{J+1}
       float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};  // 4 independent chains
 #pragma unroll
-      for (int i = 0; i < BK; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sr[i]));
+      for (int i = 0; i < BK / 2; ++i)
+        m4[i & 3] = max3(m4[i & 3], __uint_as_float(sr[2 * i]), __uint_as_float(sr[2 * i + 1]));
       float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       mx *= scale_log2;
       // the running max first (P needs only m); P_J is computed in registers while PV_{J-1} may still run
@@ -256,9 +273,11 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       }
       // P = 2^(s * scale - m) as f16 pairs (in place of S): pair c holds keys 2c, 2c + 1
 #pragma unroll
-      for (int c = 0; c < BK / 2; ++c)
-        sr[c] = t5::ex2_f16x2(t5::pack_f16x2(fmaf(__uint_as_float(sr[2 * c]), scale_log2, -m),
-                                             fmaf(__uint_as_float(sr[2 * c + 1]), scale_log2, -m)));
+      for (int c = 0; c < BK / 2; ++c) {
+        float x0, x1;
+        fma2(x0, x1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), scale_log2, scale_log2, -m, -m);
+        sr[c] = t5::ex2_f16x2(t5::pack_f16x2(x0, x1));
+      }
       l = l * f + row_sum_f16x2(sr);
       if (j > 0) {
         // PV_{J-1} done: P's columns free, O stable
