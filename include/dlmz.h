@@ -184,6 +184,24 @@ DLMZ_API int dlmz_context_scores(const dlmz_model* m, const int32_t* d_symbols, 
 DLMZ_API int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32_t M, uint32_t N, uint32_t K,
                             void* stream);
 
+/* Bidirectional grouped-query attention of one layer (Definition 3: every
+ * position attends to every position of its window; no mask), on its own:
+ * for window w, query head h and its KV head g = h / (n_heads / n_kv_heads),
+ *   out[w L + i, h hd + e] = sum_j softmax_j(q_i . k_j / sqrt(hd)) v_j[e].
+ * d_qkv: bf16 [n_chunks L x ld] device rows (window-major, L rows per window),
+ *   columns [Q heads | K heads | V heads]: query head h at h*hd, key head g at
+ *   n_heads*hd + g*hd, value head g at (n_heads + n_kv_heads)*hd + g*hd;
+ *   ld >= (n_heads + 2 n_kv_heads) hd and a multiple of 8.
+ * d_out: bf16 [n_chunks L x n_heads hd] device.  Both 16-byte aligned; the
+ *   caller owns both.
+ * head_dim one of 8, 16, 32, 64, 128; n_chunks <= 65535.  Runs on the tcgen05
+ * tensor cores when L % 128 == 0 and head_dim == 64 (V is converted to f16
+ * there, so |v| < 65504), else on CUDA cores; P is rounded to f16 (tensor
+ * cores) or kept in float32 (CUDA cores) before P V.  DLMZ_EINVAL on bad
+ * sizes or alignment, DLMZ_ENOMEM if the V^T scratch cannot be allocated. */
+DLMZ_API int dlmz_attention_bf16(const void* d_qkv, uint32_t ld, uint32_t n_chunks, uint32_t L, uint32_t n_heads,
+                                 uint32_t n_kv_heads, uint32_t head_dim, void* d_out, void* stream);
+
 /* Integer quantiser (one rule shared by encoder and decoder): per row of
  * float32 logits [rows x V], with P CDF bits (V < 2^P, P <= 24):
  *   m = max, top = lowest argmax; q_v = rint(min(fl(fl(m - l_v) * C), 8191)),

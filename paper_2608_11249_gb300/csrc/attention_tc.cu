@@ -337,6 +337,37 @@ bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 &&
 
 int attention_vt_rows(int hd) { return hd; }
 
+// V^T (f16, [window][kv head][hd][L]) from the V columns of [Q | K | V] rows,
+// through a 32 x 32 shared-memory tile so reads and writes are both coalesced.
+__global__ void vt_from_rows_kernel(const bf16* __restrict__ qkv, int ld, int v_col, int L, int nkv, int hd, int wg0,
+                                    __half* __restrict__ vt) {
+  __shared__ float t[32][33];
+  const int wg = wg0 + (int)blockIdx.z, w = wg / nkv, g = wg % nkv;
+  const int p0 = blockIdx.x * 32, d0 = blockIdx.y * 32;
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int p = p0 + i, dim = d0 + threadIdx.x;
+    t[i][threadIdx.x] =
+        p < L && dim < hd ? __bfloat162float(qkv[(size_t)(w * L + p) * ld + v_col + g * hd + dim]) : 0.0f;
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int dim = d0 + i, p = p0 + threadIdx.x;
+    if (p < L && dim < hd) vt[((size_t)wg * hd + dim) * L + p] = __float2half(t[threadIdx.x][i]);
+  }
+}
+
+int attention_vt_from_rows(const bf16* qkv, int ld, int v_col, int n_chunks, int L, int nkv, int hd, void* vt,
+                           cudaStream_t s) {
+  const int blocks = n_chunks * nkv;
+  for (int wg0 = 0; wg0 < blocks; wg0 += 65535) {
+    const int nz = blocks - wg0 < 65535 ? blocks - wg0 : 65535;
+    vt_from_rows_kernel<<<dim3((L + 31) / 32, (hd + 31) / 32, nz), dim3(32, 8), 0, s>>>(
+        qkv, ld, v_col, L, nkv, hd, wg0, reinterpret_cast<__half*>(vt));
+    DLMZ_TRY(launch_status());
+  }
+  return DLMZ_OK;
+}
+
 int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int L, int nh, int nkv, int hd, int d,
                       bf16* out, cudaStream_t s) {
   if (n_chunks == 0) return DLMZ_OK;

@@ -79,6 +79,9 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
                       int head_dim, int d, bf16* out, cudaStream_t s);
 // Rows per (window, kv head) of the attention kernel's V^T buffer.
 int attention_vt_rows(int head_dim);
+// Writes that buffer (f16) from the V columns [v_col, v_col + n_kv_heads * head_dim) of bf16 rows.
+int attention_vt_from_rows(const bf16* qkv, int ld, int v_col, int n_chunks, int L, int n_kv_heads, int head_dim,
+                           void* vt, cudaStream_t s);
 int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int n_heads, int n_kv_heads,
                        int head_dim, int d, bf16* out, cudaStream_t s);
 

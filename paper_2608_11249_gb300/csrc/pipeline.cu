@@ -1012,6 +1012,32 @@ int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32_t M, uin
   return gemm_simt<bf16>(A, (int)K, B, (int)K, (int)M, (int)N, (int)K, EPI_F32, ep, s);
 }
 
+int dlmz_attention_bf16(const void* d_qkv, uint32_t ld, uint32_t n_chunks, uint32_t L, uint32_t n_heads,
+                        uint32_t n_kv_heads, uint32_t head_dim, void* d_out, void* stream) {
+  if (!d_qkv || !d_out || !n_heads || !n_kv_heads || n_heads % n_kv_heads || !head_dim || head_dim % 8 ||
+      head_dim > 128)
+    return DLMZ_EINVAL;
+  const uint64_t d = (uint64_t)n_heads * head_dim, width = d + 2ull * n_kv_heads * head_dim;
+  if (ld < width || ld % 8 || ((reinterpret_cast<uintptr_t>(d_qkv) | reinterpret_cast<uintptr_t>(d_out)) & 15))
+    return DLMZ_EINVAL;
+  if (n_chunks > 65535 || (uint64_t)n_chunks * L * ld >= (1ull << 31) || (uint64_t)n_chunks * L * d >= (1ull << 31))
+    return DLMZ_EINVAL;
+  if (!n_chunks || !L) return DLMZ_OK;
+  if (!device_error_word()) return DLMZ_ENOMEM;
+  const bf16* qkv = reinterpret_cast<const bf16*>(d_qkv);
+  bf16* out = reinterpret_cast<bf16*>(d_out);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int nc = (int)n_chunks, l = (int)L, nh = (int)n_heads, nkv = (int)n_kv_heads, hd = (int)head_dim;
+  if (attention_tc_supported(l, hd)) {
+    static DevBuf vt;  // V^T scratch of the tensor-core kernel
+    DLMZ_TRY(vt.ensure((size_t)nc * nkv * attention_vt_rows(hd) * l * 2));
+    DLMZ_TRY(attention_vt_from_rows(qkv, (int)ld, (int)(d + (uint64_t)nkv * hd), nc, l, nkv, hd, vt.p, s));
+    return attention_bf16_tc(qkv, (int)ld, vt.p, nc, l, nh, nkv, hd, (int)d, out, s);
+  }
+  if (hd == 64 || hd == 128) return attention_bf16_mma(qkv, (int)ld, nc, l, nh, nkv, hd, (int)d, out, s);
+  return attention_simt<bf16>(qkv, (int)ld, nc, l, nh, nkv, hd, (int)d, out, s);
+}
+
 int dlmz_quantize(const float* d_logits, uint32_t rows, uint32_t V, uint32_t P, uint32_t* d_cdf, uint64_t* d_W,
                   uint64_t* d_A, int32_t* d_Hq, int32_t* d_top, void* stream) {
   if (!d_logits || !d_W || !d_Hq || V < 2 || P > 24 || (1ull << P) <= V) return DLMZ_EINVAL;

@@ -73,6 +73,7 @@ _sig("dlmz_decompress_device", c_int, _P, _P, c_size_t, _P, c_size_t, POINTER(c_
 _sig("dlmz_forward_logits", c_int, _P, _P, c_uint32, c_uint32, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_context_scores", c_int, _P, _P, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_gemm_bf16", c_int, _P, _P, _P, c_uint32, c_uint32, c_uint32, _P)
+_sig("dlmz_attention_bf16", c_int, _P, c_uint32, c_uint32, c_uint32, c_uint32, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_quantize", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P, _P, _P, _P, _P)
 _sig("dlmz_select_smallest", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
 _sig("dlmz_select_smallest_noalloc", c_int, _P, c_uint32, c_uint32, c_uint32, _P, _P)
@@ -175,6 +176,11 @@ class Model:
 
 def gemm_bf16(d_A, d_B, d_D, M, N, K, stream=0):
     _ok(lib.dlmz_gemm_bf16(d_A, d_B, d_D, M, N, K, stream), "dlmz_gemm_bf16")
+
+
+def attention_bf16(d_qkv, ld, n_chunks, L, n_heads, n_kv_heads, head_dim, d_out, stream=0):
+    _ok(lib.dlmz_attention_bf16(d_qkv, ld, n_chunks, L, n_heads, n_kv_heads, head_dim, d_out, stream),
+        "dlmz_attention_bf16")
 
 
 def quantize(d_logits, rows, V, P, d_cdf, d_W, d_A, d_Hq, d_top, stream=0):
