@@ -35,6 +35,7 @@ constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int B_HALF = BN / 2 * BK * 2;  // the 128 B rows one CTA of a pair loads for both
 constexpr int BM_ALIGN_VT = 128;  // transposed V needs whole windows per 128-row tile
 constexpr int THREADS = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
@@ -76,6 +77,32 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+// Clusters of two CTAs: rank, cluster-wide barrier, a TMA load delivered to the
+// same shared-memory offset (and barrier offset) of every CTA in `mask`, and a
+// commit that arrives on the barrier at `bar`'s offset in every CTA in `mask`.
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
+                                               uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%2, "
+      "%3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(mask)
       : "memory");
 }
 
@@ -177,6 +204,7 @@ __device__ __forceinline__ float row_ssq(const GemmEpilogue& ep, int m, int M) {
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, int lane, int m0, int M, int n0,
                                               const GemmEpilogue& ep, uint8_t* stg, float row_ss) {
+  if (m0 >= M) return;  // the second tile of a pair past the last row block: nothing to write
   const uint32_t tbase = tacc + ((uint32_t)(q * 32) << 16);
   const int row0 = m0 + q * 32;
   constexpr int NCH = (EPI == EPI_SWIGLU_BF16 ? BN / 64 : BN / 32) / 2;  // chunks per column half
@@ -341,7 +369,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
-      mbar_init(empty0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 2);  // released by the products of both CTAs of the pair
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
@@ -361,32 +389,53 @@ __global__ void __launch_bounds__(THREADS, 1)
   fence_before();
   __syncthreads();
   fence_after();
+  cluster_sync();  // the peer's barriers are initialised before anything is multicast into them
   const uint32_t tmem = tmem_slot;
 
   const int num_k = K / BK;
   const int n_tiles = N / BN;
   const int m_tiles = (M + BM - 1) / BM;
-  const int total = m_tiles * n_tiles;
+  // the two CTAs of a cluster take row blocks 2i and 2i+1 of one column block and
+  // share its B tile: each loads 128 of the 256 rows and multicasts them to both
+  const uint32_t rank = cluster_rank();
+  const int n_clusters = (int)gridDim.x >> 1, cid = (int)blockIdx.x >> 1;
+  const int total = ((m_tiles + 1) >> 1) * n_tiles;  // tile pairs
+  auto tile_of = [&](int t, int& m0, int& n0) {
+    m0 = ((t / n_tiles) * 2 + (int)rank) * BM;
+    n0 = (t % n_tiles) * BN;
+  };
 
   if (warp == 0) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / its last phase
-      for (int tile = blockIdx.x; tile < total && !abort_flag; tile += gridDim.x) {
-        const int m0 = (tile / n_tiles) * BM;
-        const int n0 = (tile % n_tiles) * BN;
+      for (int tile = cid; tile < total && !abort_flag; tile += n_clusters) {
+        int m0, n0;
+        tile_of(tile, m0, n0);
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, &abort_flag, err)) break;
-          mbar_arrive_expect_tx(full0 + 8 * stage, STAGE_BYTES);
-          tma_load_2d(smem_u32(sA + stage * A_BYTES), &tmA, kb * BK, m0, full0 + 8 * stage);
-          tma_load_2d(smem_u32(sB + stage * B_BYTES), &tmB, kb * BK, n0, full0 + 8 * stage);
+          mbar_arrive_expect_tx(full0 + 8 * stage, STAGE_BYTES);  // A + both halves of B
+          // a tile past the last row block (odd row-block count) loads rows 0.. instead: in bounds,
+          // same byte count, and its accumulator is never written out
+          tma_load_2d(smem_u32(sA + stage * A_BYTES), &tmA, kb * BK, m0 < M ? m0 : 0, full0 + 8 * stage);
+          tma_load_2d_mc(smem_u32(sB + stage * B_BYTES + rank * B_HALF), &tmB, kb * BK, n0 + (int)rank * (BN / 2),
+                         full0 + 8 * stage, 0x3);
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
           }
+        }
+      }
+      // both products have released every stage this CTA filled: no arrive from the
+      // peer can land after this CTA exits
+      for (int s = 0; s < STAGES && !abort_flag; ++s) {
+        if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, &abort_flag, err)) break;
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1;
         }
       }
       if (abort_flag) {  // drain our own copies before the CTA may exit
@@ -403,7 +452,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool issued_any = false;
-      for (int tile = blockIdx.x; tile < total && !abort_flag; tile += gridDim.x) {
+      for (int tile = cid; tile < total && !abort_flag; tile += n_clusters) {
         if (!mbar_wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1, &abort_flag, err)) break;
         fence_after();
         const uint32_t d_tmem = tmem + acc * BN;
@@ -420,7 +469,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           for (int k = 0; k < BK / 16; ++k)
             mma_bf16(d_tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (kb | k) != 0);
           issued_any = true;
-          mma_commit(empty0 + 8 * stage);
+          mma_commit_mc(empty0 + 8 * stage, 0x3);  // the stage is free once both CTAs' products read it
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
@@ -447,16 +496,23 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t acc_phase = 0;
     constexpr bool kScale = EPI == EPI_ROPE_BF16 || EPI == EPI_SWIGLU_BF16;
     float ss_next = 0.f;
-    if (kScale && blockIdx.x < total) ss_next = row_ssq(ep, (blockIdx.x / n_tiles) * BM + q * 32 + lane, M);
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+    if (kScale && cid < total) {
+      int m1, n1;
+      tile_of(cid, m1, n1);
+      ss_next = row_ssq(ep, m1 + q * 32 + lane, M);
+    }
+    for (int tile = cid; tile < total; tile += n_clusters) {
       const float ss_cur = ss_next;
-      if (kScale && tile + (int)gridDim.x < total)  // next tile's row, loaded while this tile drains
-        ss_next = row_ssq(ep, ((tile + gridDim.x) / n_tiles) * BM + q * 32 + lane, M);
+      if (kScale && tile + n_clusters < total) {  // next tile's row, loaded while this tile drains
+        int m1, n1;
+        tile_of(tile + n_clusters, m1, n1);
+        ss_next = row_ssq(ep, m1 + q * 32 + lane, M);
+      }
       // warp-uniform outcome: the epilogue's tcgen05.ld is warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait_bounded(tfull0 + 8 * acc, acc_phase, &abort_flag, err))) break;
       fence_after();
-      const int m0 = (tile / n_tiles) * BM;
-      const int n0 = (tile % n_tiles) * BN;
+      int m0, n0;
+      tile_of(tile, m0, n0);
       epilogue_tile<EPI>(tmem + acc * BN, q, half, lane, m0, M, n0, ep, stg, ss_cur);
       fence_before();
       mbar_arrive(tempty0 + 8 * acc);
@@ -468,6 +524,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
   fence_before();
   __syncthreads();
+  cluster_sync();
   if (warp == 1) {
     fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
@@ -532,12 +589,34 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
     DLMZ_CUDA_TRY(cudaFuncSetAttribute(gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
     attr = true;
   }
-  const int tiles = ((M + BM - 1) / BM) * (N / BN);
-  const int grid = tiles < num_sms() ? tiles : num_sms();
+  // clusters of two CTAs (one per SM), as many as fit at once, each walking tile pairs
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute cl[1];
+  cl[0].id = cudaLaunchAttributeClusterDimension;
+  cl[0].val.clusterDim.x = 2;
+  cl[0].val.clusterDim.y = 1;
+  cl[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = s;
+  cfg.attrs = cl;
+  cfg.numAttrs = 1;
+  static int max_clusters = 0;
+  if (!max_clusters) {
+    cfg.gridDim = dim3(2 * (num_sms() / 2));
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, gemm_kernel<EPI>, &cfg) != cudaSuccess || max_clusters < 1) {
+      (void)cudaGetLastError();
+      max_clusters = num_sms() / 2;
+    }
+    // one CTA per SM (shared memory and all 512 TMEM columns): never more clusters than SM pairs
+    if (max_clusters > num_sms() / 2) max_clusters = num_sms() / 2;
+  }
+  const int pairs = ((M + BM - 1) / BM + 1) / 2 * (N / BN);
+  cfg.gridDim = dim3(2 * (pairs < max_clusters ? pairs : max_clusters));
   const double out_b = EPI == EPI_F32 ? 4.0 * M * N : EPI == EPI_RESID_F32 ? 8.0 * M * N
                      : EPI == EPI_SWIGLU_BF16 ? 1.0 * M * N : 2.0 * M * N;
   ProfScope prof(PROF_GEMM_TC, s, 2.0 * M * N * K, 2.0 * M * K + 2.0 * N * K + out_b);
-  gemm_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(a, b, M, N, K, ep, device_error_word());
+  DLMZ_CUDA_TRY(cudaLaunchKernelEx(&cfg, gemm_kernel<EPI>, a, b, M, N, K, ep, device_error_word()));
   return launch_status();
 }
 
@@ -552,7 +631,7 @@ int gemm_bf16_tc(const __nv_bfloat16* A, int lda, const __nv_bfloat16* B, int ld
   if ((lda | ldb) & 7) return DLMZ_EINVAL;
   CUtensorMap ma, mb;
   DLMZ_TRY(t5::make_map_bf16(&ma, A, M, K, lda, tc::BM, tc::BK));
-  DLMZ_TRY(t5::make_map_bf16(&mb, B, N, K, ldb, tc::BN, tc::BK));
+  DLMZ_TRY(t5::make_map_bf16(&mb, B, N, K, ldb, tc::BN / 2, tc::BK));  // one CTA of a pair loads half a tile
   switch (epi) {
     case EPI_BF16: return tc::launch<EPI_BF16>(ma, mb, M, N, K, ep, s);
     case EPI_F32: return tc::launch<EPI_F32>(ma, mb, M, N, K, ep, s);
