@@ -35,7 +35,7 @@ INPUT_BYTES = 4 << 20
 # (profiles/gemm_dram_traffic_byte_workload.md).  Equal to the algorithmic
 # bytes within 2%: no operand is re-read from DRAM.  Re-measure when the GEMM
 # kernel changes.
-GEMM_DRAM_BYTES_PER_LAUNCH = 3.089e9
+GEMM_DRAM_BYTES_PER_LAUNCH = 3.088e9
 WORKLOAD = ("small byte-level masked DLM, bf16, 8 layers d=512 8 heads FFN 2048 V=256; 4 MiB order-2 "
             "Markov/Zipf(1.1) bytes; windows of 512 B, 1024 windows per batch, block 128, top-k 8 by "
             "confidence, 16-bit CDFs")
