@@ -14,7 +14,9 @@
 //               ex2.approx.f16x2, stored back to TMEM as f16 pairs (the A
 //               operand of P V), and the row sum l of those f16 values; the
 //               running max is raised (and O and l rescaled) only when it grows
-//               by more than 8 (log2 units), so P <= 2^8; finally O / l -> bf16.
+//               by more than 8 (log2 units), so P <= 2^8; finally O / l -> bf16,
+//               deferred into the next item's first tile so the next S is
+//               taken (and the MMA warp goes on) before the last P V is waited for.
 // GQA: query head h reads KV head h / (n_heads / n_kv_heads).  Requires the
 // window length to be a multiple of 128.  All waits are bounded.
 #include "kernels.cuh"
@@ -72,6 +74,24 @@ __device__ __forceinline__ void fma2(float& y0, float& y1, float x0, float x1, f
   asm("mov.b64 %0, {%1, %2};" : "=l"(b) : "f"(b0), "f"(b1));
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(y) : "l"(x), "l"(a), "l"(b));
   asm("mov.b64 {%0, %1}, %2;" : "=f"(y0), "=f"(y1) : "l"(y));
+}
+
+// One query row of an item's output: O / l -> bf16, HD values from 16-byte stores.
+template <int HD>
+__device__ __forceinline__ void write_row(bf16* __restrict__ dst, const uint32_t (&o)[HD], float l) {
+  const float inv = 1.0f / l;
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int t = 0; t < HD / 8; ++t) {
+    uint32_t u[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      __nv_bfloat162 p2 = __floats2bfloat162_rn(__uint_as_float(o[8 * t + 2 * e]) * inv,
+                                                __uint_as_float(o[8 * t + 2 * e + 1]) * inv);
+      u[e] = *reinterpret_cast<uint32_t*>(&p2);
+    }
+    d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
+  }
 }
 
 template <int HD>
@@ -244,7 +264,17 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
     const int q = warp & 3;
     const int r = q * 32 + lane;  // query row within the tile (= TMEM lane)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    auto row_of = [&](int it) {  // this thread's output row of item `it`
+      int w, h, q0;
+      item_of(it, w, h, q0);
+      return out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
+    };
     float m = -INFINITY, l = 0.0f;
+    // An item's epilogue is deferred into the next item's first tile: that tile's S is loaded
+    // (so the MMA warp can go on) and exponentiated first; O is read where the P store has to
+    // wait for the last P V anyway, and written out after P_J is handed over.
+    bool pend = false;
+    float l_pend = 0.0f;
     for (int J = 0; J < total; ++J) {
       const int j = J % nt;
       // waits are made warp-uniform: tcgen05.ld/st below are warp-collective
@@ -263,7 +293,7 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
       // the running max first (P needs only m); P_J is computed in registers while PV_{J-1} may still run
       float f = 1.0f;
       bool need = false;
-      if (j == 0) {  // P and O were released by this item's predecessor's epilogue
+      if (j == 0) {  // a new item: fresh running max and row sum
         m = mx;
         l = 0.0f;
       } else if (mx > m + RESCALE_THRESHOLD) {
@@ -279,47 +309,49 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
         sr[c] = t5::ex2_f16x2(t5::pack_f16x2(x0, x1));
       }
       l = l * f + row_sum_f16x2(sr);
-      if (j > 0) {
-        // PV_{J-1} done: P's columns free, O stable
+      bool p_stored = false;
+      if (j > 0 || pend) {
+        // PV_{J-1} done: P's columns free, O stable (at an item's first tile: the previous item's O is final)
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (J - 1) & 1, &abort_flag, err))) break;
         t5::fence_after();
-        if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
+        if (j == 0) {
+          uint32_t o[HD];
+          t5::tmem_ld64(tO + lane_off, o);
+          t5::tmem_st64(tP + lane_off, sr);
+          t5::fence_before();
+          mbar_arrive(o_free);  // O is in registers: this item's first PV may overwrite it
+          mbar_arrive(p_ready);
+          p_stored = true;
+          write_row<HD>(row_of(J / nt - 1), o, l_pend);  // the previous item's output, off the MMA warp's path
+          pend = false;
+        } else if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
 #pragma unroll 1
           for (int c = 0; c < HD / 16; ++c) {
-            uint32_t o[16];
-            t5::tmem_ld16(tO + lane_off + c * 16, o);
+            uint32_t oc[16];
+            t5::tmem_ld16(tO + lane_off + c * 16, oc);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
-            t5::tmem_st16(tO + lane_off + c * 16, o);
+            for (int i = 0; i < 16; ++i) oc[i] = __float_as_uint(__uint_as_float(oc[i]) * f);
+            t5::tmem_st16(tO + lane_off + c * 16, oc);
           }
         }
       }
-      t5::tmem_st64(tP + lane_off, sr);
-      t5::fence_before();
-      mbar_arrive(p_ready);
-      if (j == nt - 1) {  // this item's epilogue: O / l -> bf16
-        if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, J & 1, &abort_flag, err))) break;
+      if (!p_stored) {
+        t5::tmem_st64(tP + lane_off, sr);
+        t5::fence_before();
+        mbar_arrive(p_ready);
+      }
+      if (j == nt - 1) {
+        pend = true;
+        l_pend = l;
+      }
+    }
+    if (pend && !abort_flag) {  // the last item's epilogue
+      if (__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (total - 1) & 1, &abort_flag, err))) {
         t5::fence_after();
         uint32_t o[HD];
         t5::tmem_ld64(tO + lane_off, o);
         t5::fence_before();
-        mbar_arrive(o_free);  // O is in registers: the next item's first PV may overwrite it
-        int w, h, q0;
-        item_of(J / nt, w, h, q0);
-        const float inv = 1.0f / l;
-        bf16* dst = out + ((size_t)w * L + q0 + r) * d + (size_t)h * HD;
-        uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-        for (int t = 0; t < HD / 8; ++t) {
-          uint32_t u[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 p2 = __floats2bfloat162_rn(__uint_as_float(o[8 * t + 2 * e]) * inv,
-                                                      __uint_as_float(o[8 * t + 2 * e + 1]) * inv);
-            u[e] = *reinterpret_cast<uint32_t*>(&p2);
-          }
-          d4[t] = make_uint4(u[0], u[1], u[2], u[3]);
-        }
+        write_row<HD>(row_of((total - 1) / nt), o, l_pend);
       }
     }
   }
