@@ -197,8 +197,11 @@ DLMZ_API int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32
  * head_dim one of 8, 16, 32, 64, 128; n_chunks <= 65535.  Runs on the tcgen05
  * tensor cores when L % 128 == 0 and head_dim == 64 (V is converted to f16
  * there, so |v| < 65504), else on CUDA cores; P is rounded to f16 (tensor
- * cores) or kept in float32 (CUDA cores) before P V.  DLMZ_EINVAL on bad
- * sizes or alignment, DLMZ_ENOMEM if the V^T scratch cannot be allocated. */
+ * cores) or kept in float32 (CUDA cores) before P V.  The tensor-core path
+ * converts V into a library-owned V^T scratch buffer (grown with cudaMalloc
+ * as needed, kept until exit): calls that overlap on the GPU race on it;
+ * sequential calls are independent.  DLMZ_EINVAL on bad sizes or alignment,
+ * DLMZ_ENOMEM if the V^T scratch cannot be allocated. */
 DLMZ_API int dlmz_attention_bf16(const void* d_qkv, uint32_t ld, uint32_t n_chunks, uint32_t L, uint32_t n_heads,
                                  uint32_t n_kv_heads, uint32_t head_dim, void* d_out, void* stream);
 

@@ -8,14 +8,21 @@
 // stream), the gate/up projection (SwiGLU in the epilogue) and the LM head
 // (float32 logits).
 //
-// Design (one CTA per SM, persistent over output tiles of 128 x 256):
+// Design (one CTA per SM, persistent over output tiles of 128 x 256, in
+// clusters of two: the CTAs of a cluster take row blocks 2i and 2i+1 of one
+// column block, and each loads 128 of the 256 rows of the shared B slice and
+// multicasts them to both, so each B byte leaves L2 once per pair):
 //   warp 0      TMA producer: 128B-swizzled A/B K-slices (64 elements) into a
-//               4-stage shared-memory ring, completion on mbarriers.
+//               4-stage shared-memory ring, completion on mbarriers (a slot is
+//               refilled once the products of both CTAs have read it).
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
 //               issues tcgen05.mma (M=128, N=256, K=16) from one thread;
-//               tcgen05.commit frees a ring slot / publishes an accumulator.
-//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns per warp (each
-//               thread owns one output row), fused op, vectorised stores.
+//               tcgen05.commit frees a ring slot (in both CTAs) / publishes an
+//               accumulator.
+//   warps 2-9   epilogue, two warps per TMEM lane quadrant (one column half
+//               each): tcgen05.ld 32 lanes x 32 columns (each thread owns one
+//               output row), fused op, staged through shared memory so global
+//               accesses are row-contiguous.
 // Two accumulators let the epilogue of tile i overlap the MMAs of tile i+1.
 // Every mbarrier wait is bounded; on timeout the CTA sets the error word,
 // waits (bounded) for its own outstanding copies and MMAs, frees TMEM and
