@@ -168,3 +168,100 @@ def test_bf16_model_rounds_storage():
     a = M.forward(w, np.array([1, 2, 11, 3]))
     b = M.forward(_weights(), np.array([1, 2, 11, 3]))
     assert np.max(np.abs(a - b)) < 2e-2  # bf16 storage vs float32 storage of the same draws
+
+
+def _torch_block_forward(cfg, t, state):
+    """Definition 3's LLaDA-style block restated with PyTorch float64 CPU library calls.
+
+    Written from the block definition (pre-norm RMSNorm, rotary embedding as a
+    complex rotation of the pairs (i, i + hd/2), grouped-query attention via
+    scaled_dot_product_attention without a mask, SwiGLU = silu(gate) * up,
+    residual adds, final RMSNorm, untied head), not from oracle/model.py.  A
+    tensor the model stores is rounded to float32 (torch's own conversion).
+    """
+    import torch
+    import torch.nn.functional as F
+
+    f64 = torch.float64
+    st = lambda a: a.to(torch.float32).to(f64)
+    T = {k: torch.from_numpy(np.asarray(v, dtype=np.float64)) for k, v in t.items()}
+    hd, L = cfg.d // cfg.n_heads, len(state)
+    idx = torch.as_tensor(np.asarray(state), dtype=torch.long)
+
+    def norm(x):
+        return x * torch.rsqrt((x * x).mean(-1, keepdim=True) + cfg.norm_eps)
+
+    half = hd // 2
+    inv = float(cfg.rope_theta) ** (-torch.arange(half, dtype=f64) * 2.0 / hd)
+    rot = torch.polar(torch.ones(L, half, dtype=f64), torch.arange(L, dtype=f64)[:, None] * inv[None, :])
+
+    def rope(u, nh):
+        u = u.view(L, nh, hd)
+        z = torch.complex(u[..., :half], u[..., half:]) * rot[:, None, :]
+        return torch.cat([z.real, z.imag], -1).reshape(L, nh * hd)
+
+    x = st(T[M.TID_EMBED][idx])
+    g = cfg.n_heads // cfg.n_kv_heads
+    for l in range(cfg.n_layers):
+        P = lambda which: T[M.layer_tid(l, which)]
+        h = st(norm(x))
+        q = st(rope(F.linear(h, P(M.WQ)), cfg.n_heads)).view(L, cfg.n_heads, hd).transpose(0, 1)
+        k = st(rope(F.linear(h, P(M.WK)), cfg.n_kv_heads)).view(L, cfg.n_kv_heads, hd).transpose(0, 1)
+        v = st(F.linear(h, P(M.WV))).view(L, cfg.n_kv_heads, hd).transpose(0, 1)
+        o = F.scaled_dot_product_attention(q, k.repeat_interleave(g, 0), v.repeat_interleave(g, 0), is_causal=False)
+        x = st(x + F.linear(st(o.transpose(0, 1).reshape(L, cfg.d)), P(M.WO)))
+        h = st(norm(x))
+        a = st(F.silu(F.linear(h, P(M.WGATE))) * F.linear(h, P(M.WUP)))
+        x = st(x + F.linear(a, P(M.WDOWN)))
+    return st(F.linear(st(norm(x)), T[M.TID_HEAD])).numpy()
+
+
+def test_forward_matches_independent_torch_block():
+    # nonzero gate and up weights large enough that SiLU is far from x/2 (with
+    # N(0, 0.02) weights silu(g) u ~ g u / 2 is nearly symmetric in g and u, so a
+    # gate/up swap would hide); GQA, RoPE and two layers exercise the whole block
+    pytest.importorskip("torch")
+    cfg = M.ModelConfig(n_layers=2, d=32, n_heads=4, n_kv_heads=2, ffn=48, vocab=11, dtype="f32", seed=3)
+    rng = np.random.default_rng(21)
+    t = {tid: W.round_f32(rng.normal(scale=0.4 if tid >= 2 else 1.0, size=shp))
+         for tid, shp in M.tensor_shapes(cfg).items()}
+    w = M.Weights(cfg, tensors=t)
+    s = np.array([3, 11, 0, 7, 11, 2, 10, 5, 11])
+    ours = M.forward(w, s)
+    ref = _torch_block_forward(cfg, t, s)
+    assert np.max(np.abs(ours - ref)) <= 1e-4 * max(1.0, np.max(np.abs(ref)))
+    # the SwiGLU is asymmetric at this scale: exchanging the gate and up weights moves the logits
+    t2 = dict(t)
+    for l in range(cfg.n_layers):
+        t2[M.layer_tid(l, M.WGATE)], t2[M.layer_tid(l, M.WUP)] = t[M.layer_tid(l, M.WUP)], t[M.layer_tid(l, M.WGATE)]
+    assert np.max(np.abs(_torch_block_forward(cfg, t2, s) - ref)) > 1e-1
+
+
+def test_ffn_closed_form_single_layer():
+    # one layer with Wv = 0 (attention adds nothing): the block output is
+    # x + (silu(h Wg^T) * (h Wu^T)) Wd^T with h = RMSNorm(x), x = E[s], written out per element
+    cfg = M.ModelConfig(n_layers=1, d=8, n_heads=2, n_kv_heads=2, ffn=6, vocab=5, dtype="f32")
+    rng = np.random.default_rng(22)
+    w = M.Weights(cfg)
+    wg = W.round_f32(rng.normal(scale=0.8, size=(6, 8)))
+    wu = W.round_f32(rng.normal(scale=0.8, size=(6, 8)))
+    wd = W.round_f32(rng.normal(scale=0.8, size=(8, 6)))
+    w.t[M.layer_tid(0, M.WV)] = np.zeros((8, 8))
+    w.t[M.layer_tid(0, M.WGATE)] = wg
+    w.t[M.layer_tid(0, M.WUP)] = wu
+    w.t[M.layer_tid(0, M.WDOWN)] = wd
+    s = np.array([4, 0, 5, 2])
+    want = np.empty((len(s), 8))
+    for r, sym in enumerate(s):
+        x = [float(e) for e in w.embed[sym]]
+        ms = sum(e * e for e in x) / 8
+        h = [e / (ms + cfg.norm_eps) ** 0.5 for e in x]
+        a = []
+        for f in range(6):
+            gf = sum(h[i] * wg[f, i] for i in range(8))
+            uf = sum(h[i] * wu[f, i] for i in range(8))
+            a.append(gf / (1.0 + np.exp(-gf)) * uf)
+        xo = [x[o] + sum(a[f] * wd[o, f] for f in range(6)) for o in range(8)]
+        ms = sum(e * e for e in xo) / 8
+        want[r] = [e / (ms + cfg.norm_eps) ** 0.5 for e in xo]
+    assert np.allclose(M.hidden(w, s), want, atol=1e-5)
