@@ -222,11 +222,9 @@ int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int nh, int
     fa::flash_kernel<64><<<grid, 128, SM, s>>>(qkv, ld, L, nh, nkv, d, out, scale_log2);
   } else if (hd == 128) {
     constexpr int SM = 5 * 64 * 128 * 2;
-    static bool attr = false;
-    if (!attr) {
-      DLMZ_CUDA_TRY(cudaFuncSetAttribute(fa::flash_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM));
-      attr = true;
-    }
+    static PerDeviceOnce attr;
+    DLMZ_TRY(attr.run(
+        [] { return cudaFuncSetAttribute(fa::flash_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
     fa::flash_kernel<128><<<grid, 128, SM, s>>>(qkv, ld, L, nh, nkv, d, out, scale_log2);
   } else {
     return DLMZ_EINVAL;

@@ -12,7 +12,7 @@
 
 namespace dlmz {
 
-// Device-side error word (one per process/device, zeroed by dlmz_check).
+// Device-side error word (one per device, zeroed by dlmz_check).
 // Bits: 1 = wait timed out, 2 = corrupt stream, 4 = non-finite logits,
 // 8 = stream capacity exceeded.
 enum : int { ERR_TIMEOUT = 1, ERR_CORRUPT = 2, ERR_NONFINITE = 4, ERR_CAPACITY = 8 };
@@ -66,15 +66,48 @@ inline int launch_status() {
   return DLMZ_OK;
 }
 
-inline int num_sms() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 1;
+// ---- per-device caches ------------------------------------------------------
+// Kernel attributes, occupancy limits, SM counts and scratch buffers belong to
+// one device, so every cache of the library is indexed by the ordinal of the
+// current device (at most kMaxDevices devices per process).
+constexpr int kMaxDevices = 64;
+
+// Ordinal of the current device, or -1 when it cannot be used as an index.
+inline int device_ordinal() {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return -1;
+  return d;
+}
+
+// Runs a set-up step (returning cudaError_t) once per device: the first call
+// on each device runs it, later calls on that device return DLMZ_OK at once.
+struct PerDeviceOnce {
+  bool done[kMaxDevices] = {};
+  template <class F>
+  int run(F f) {
+    const int d = device_ordinal();
+    if (d < 0) return DLMZ_ECUDA;
+    if (done[d]) return DLMZ_OK;
+    const cudaError_t e = f();
+    if (e != cudaSuccess) {
+      fprintf(stderr, "dlmz: per-device set-up failed: %s\n", cudaGetErrorString(e));
+      return DLMZ_ECUDA;
+    }
+    done[d] = true;
+    return DLMZ_OK;
   }
-  return n;
+};
+
+inline int num_sms() {
+  static int n[kMaxDevices] = {};
+  const int dev = device_ordinal();
+  if (dev < 0) return 1;
+  if (!n[dev]) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    n[dev] = v > 0 ? v : 1;
+  }
+  return n[dev];
 }
 
 // ---- device helpers -------------------------------------------------------

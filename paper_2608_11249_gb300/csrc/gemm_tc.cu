@@ -8,17 +8,15 @@
 // stream), the gate/up projection (SwiGLU in the epilogue) and the LM head
 // (float32 logits).
 //
-// Design (one CTA per SM, persistent over output tiles of 128 x 256, in
-// clusters of two: the CTAs of a cluster take row blocks 2i and 2i+1 of one
-// column block, and each loads 128 of the 256 rows of the shared B slice and
-// multicasts them to both, so each B byte leaves L2 once per pair):
+// Design (one CTA per SM, persistent over output tiles of 128 x 256 taken in
+// grouped order: a group of G row blocks is swept column block by column
+// block, so the G A-slices stay in L2 while B streams through it once per
+// group; G is sized from K so the group's A fits in a fraction of L2):
 //   warp 0      TMA producer: 128B-swizzled A/B K-slices (64 elements) into a
-//               4-stage shared-memory ring, completion on mbarriers (a slot is
-//               refilled once the products of both CTAs have read it).
+//               4-stage shared-memory ring, completion on mbarriers.
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
 //               issues tcgen05.mma (M=128, N=256, K=16) from one thread;
-//               tcgen05.commit frees a ring slot (in both CTAs) / publishes an
-//               accumulator.
+//               tcgen05.commit frees a ring slot / publishes an accumulator.
 //   warps 2-9   epilogue, two warps per TMEM lane quadrant (one column half
 //               each): tcgen05.ld 32 lanes x 32 columns (each thread owns one
 //               output row), fused op, staged through shared memory so global
@@ -42,99 +40,17 @@ constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int B_HALF = BN / 2 * BK * 2;  // the 128 B rows one CTA of a pair loads for both
 constexpr int BM_ALIGN_VT = 128;  // transposed V needs whole windows per 128-row tile
 constexpr int THREADS = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
 constexpr int STG_BYTES = 8 * 32 * 128;  // epilogue staging, 8 warps x 32 x 32 float32
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256 + STG_BYTES;
 
-// Instruction descriptor (kind::f16): D f32, A/B bf16, both K-major, M=128, N=256.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                           ((uint32_t)(BM >> 4) << 24);
+constexpr uint32_t IDESC = t5::idesc_bf16(BM, BN);  // D f32, A/B bf16, both K-major
 
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (SBO), descriptor version 1.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFF) >> 4);
-  d |= (uint64_t)1 << 16;             // LBO (unused for swizzled K-major)
-  d |= (uint64_t)(1024 >> 4) << 32;   // SBO
-  d |= (uint64_t)1 << 46;             // version
-  d |= (uint64_t)2 << 61;             // SWIZZLE_128B
-  return d;
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
-                                            uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
-      "%3}], [%4];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
-      : "memory");
-}
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(IDESC), "r"(accumulate));
-}
-
-__device__ __forceinline__ void mma_commit(uint32_t bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-      : "memory");
-}
-
-// Clusters of two CTAs: rank, cluster-wide barrier, a TMA load delivered to the
-// same shared-memory offset (and barrier offset) of every CTA in `mask`, and a
-// commit that arrives on the barrier at `bar`'s offset in every CTA in `mask`.
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-}
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
-                                               uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%2, "
-      "%3}], [%4], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(mask)
-      : "memory");
-}
-__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
-      "h"(mask)
-      : "memory");
-}
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%"
-      "15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-__device__ __forceinline__ void fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
+using t5::fence_after;
+using t5::fence_before;
+using t5::tmem_ld32;
 
 // Epilogue staging: each epilogue warp owns a 32 x 32 float32 buffer; 16-byte
 // chunks are XOR-swizzled by row so both the row-per-thread writes and the
@@ -211,7 +127,6 @@ __device__ __forceinline__ float row_ssq(const GemmEpilogue& ep, int m, int M) {
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, int lane, int m0, int M, int n0,
                                               const GemmEpilogue& ep, uint8_t* stg, float row_ss) {
-  if (m0 >= M) return;  // the second tile of a pair past the last row block: nothing to write
   const uint32_t tbase = tacc + ((uint32_t)(q * 32) << 16);
   const int row0 = m0 + q * 32;
   constexpr int NCH = (EPI == EPI_SWIGLU_BF16 ? BN / 64 : BN / 32) / 2;  // chunks per column half
@@ -350,10 +265,21 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
   }
 }
 
+// Tile t of the grouped order: groups of `group` row blocks, column blocks in
+// order inside a group, row blocks fastest (the last group may be shorter).
+__device__ __forceinline__ void grouped_tile(int t, int m_tiles, int n_tiles, int group, int& m0, int& n0) {
+  const int per_group = group * n_tiles;
+  const int g = t / per_group, r = t % per_group;
+  const int gm0 = g * group;
+  const int gs = m_tiles - gm0 < group ? m_tiles - gm0 : group;
+  m0 = (gm0 + r % gs) * BM;
+  n0 = (r / gs) * BN;
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                int M, int N, int K, GemmEpilogue ep, int* err) {
+                int M, int N, int K, int group, GemmEpilogue ep, int* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -376,7 +302,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
-      mbar_init(empty0 + 8 * s, 2);  // released by the products of both CTAs of the pair
+      mbar_init(empty0 + 8 * s, 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
@@ -396,53 +322,34 @@ __global__ void __launch_bounds__(THREADS, 1)
   fence_before();
   __syncthreads();
   fence_after();
-  cluster_sync();  // the peer's barriers are initialised before anything is multicast into them
   const uint32_t tmem = tmem_slot;
 
   const int num_k = K / BK;
   const int n_tiles = N / BN;
   const int m_tiles = (M + BM - 1) / BM;
-  // the two CTAs of a cluster take row blocks 2i and 2i+1 of one column block and
-  // share its B tile: each loads 128 of the 256 rows and multicasts them to both
-  const uint32_t rank = cluster_rank();
-  const int n_clusters = (int)gridDim.x >> 1, cid = (int)blockIdx.x >> 1;
-  const int total = ((m_tiles + 1) >> 1) * n_tiles;  // tile pairs
-  auto tile_of = [&](int t, int& m0, int& n0) {
-    m0 = ((t / n_tiles) * 2 + (int)rank) * BM;
-    n0 = (t % n_tiles) * BN;
-  };
+  const int total = m_tiles * n_tiles;
+  const int cid = (int)blockIdx.x, n_ctas = (int)gridDim.x;
+  auto tile_of = [&](int t, int& m0, int& n0) { grouped_tile(t, m_tiles, n_tiles, group, m0, n0); };
 
   if (warp == 0) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / its last phase
-      for (int tile = cid; tile < total && !abort_flag; tile += n_clusters) {
+      for (int tile = cid; tile < total && !abort_flag; tile += n_ctas) {
         int m0, n0;
         tile_of(tile, m0, n0);
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, &abort_flag, err)) break;
-          mbar_arrive_expect_tx(full0 + 8 * stage, STAGE_BYTES);  // A + both halves of B
-          // a tile past the last row block (odd row-block count) loads rows 0.. instead: in bounds,
-          // same byte count, and its accumulator is never written out
-          tma_load_2d(smem_u32(sA + stage * A_BYTES), &tmA, kb * BK, m0 < M ? m0 : 0, full0 + 8 * stage);
-          tma_load_2d_mc(smem_u32(sB + stage * B_BYTES + rank * B_HALF), &tmB, kb * BK, n0 + (int)rank * (BN / 2),
-                         full0 + 8 * stage, 0x3);
+          mbar_arrive_expect_tx(full0 + 8 * stage, STAGE_BYTES);  // rows past M read as zero, full byte count
+          t5::tma_load_2d(smem_u32(sA + stage * A_BYTES), &tmA, kb * BK, m0, full0 + 8 * stage);
+          t5::tma_load_2d(smem_u32(sB + stage * B_BYTES), &tmB, kb * BK, n0, full0 + 8 * stage);
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
           }
-        }
-      }
-      // both products have released every stage this CTA filled: no arrive from the
-      // peer can land after this CTA exits
-      for (int s = 0; s < STAGES && !abort_flag; ++s) {
-        if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, &abort_flag, err)) break;
-        if (++stage == STAGES) {
-          stage = 0;
-          phase ^= 1;
         }
       }
       if (abort_flag) {  // drain our own copies before the CTA may exit
@@ -459,7 +366,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool issued_any = false;
-      for (int tile = cid; tile < total && !abort_flag; tile += n_clusters) {
+      for (int tile = cid; tile < total && !abort_flag; tile += n_ctas) {
         if (!mbar_wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1, &abort_flag, err)) break;
         fence_after();
         const uint32_t d_tmem = tmem + acc * BN;
@@ -474,16 +381,16 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            mma_bf16(d_tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (kb | k) != 0);
+            t5::mma_bf16(d_tmem, t5::sw128_desc(a0 + 32 * k), t5::sw128_desc(b0 + 32 * k), IDESC, (kb | k) != 0);
           issued_any = true;
-          mma_commit_mc(empty0 + 8 * stage, 0x3);  // the stage is free once both CTAs' products read it
+          t5::commit(empty0 + 8 * stage);  // the stage is free once the products have read it
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
           }
         }
         if (!ok) break;
-        mma_commit(tfull0 + 8 * acc);
+        t5::commit(tfull0 + 8 * acc);
         if (++acc == 2) {
           acc = 0;
           acc_phase ^= 1;
@@ -491,7 +398,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (abort_flag && issued_any) {  // wait for our MMAs before TMEM is freed
         volatile int never = 0;
-        mma_commit(drain);
+        t5::commit(drain);
         mbar_wait_bounded(drain, 0, &never, err, 100000000ull);
       }
     }
@@ -508,11 +415,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       tile_of(cid, m1, n1);
       ss_next = row_ssq(ep, m1 + q * 32 + lane, M);
     }
-    for (int tile = cid; tile < total; tile += n_clusters) {
+    for (int tile = cid; tile < total; tile += n_ctas) {
       const float ss_cur = ss_next;
-      if (kScale && tile + n_clusters < total) {  // next tile's row, loaded while this tile drains
+      if (kScale && tile + n_ctas < total) {  // next tile's row, loaded while this tile drains
         int m1, n1;
-        tile_of(tile + n_clusters, m1, n1);
+        tile_of(tile + n_ctas, m1, n1);
         ss_next = row_ssq(ep, m1 + q * 32 + lane, M);
       }
       // warp-uniform outcome: the epilogue's tcgen05.ld is warp-collective
@@ -531,7 +438,6 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
   fence_before();
   __syncthreads();
-  cluster_sync();
   if (warp == 1) {
     fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
@@ -588,42 +494,32 @@ int t5::make_map_f16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t
 
 namespace tc {
 
+// Row blocks per group of the tile order: the group's A slices (BM x K bf16
+// each) take at most ~48 MB of the 129 MB L2, and at least one block.
+static int group_for(int m_tiles, int K) {
+  const long a_tile = (long)BM * K * 2;
+  long g = (48l << 20) / a_tile;
+  if (g < 1) g = 1;
+  if (g > m_tiles) g = m_tiles;
+  return (int)g;
+}
+
 template <int EPI>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const GemmEpilogue& ep,
                   cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    DLMZ_CUDA_TRY(cudaFuncSetAttribute(gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
-    attr = true;
-  }
-  // clusters of two CTAs (one per SM), as many as fit at once, each walking tile pairs
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute cl[1];
-  cl[0].id = cudaLaunchAttributeClusterDimension;
-  cl[0].val.clusterDim.x = 2;
-  cl[0].val.clusterDim.y = 1;
-  cl[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(THREADS);
-  cfg.dynamicSmemBytes = SMEM_BYTES;
-  cfg.stream = s;
-  cfg.attrs = cl;
-  cfg.numAttrs = 1;
-  static int max_clusters = 0;
-  if (!max_clusters) {
-    cfg.gridDim = dim3(2 * (num_sms() / 2));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, gemm_kernel<EPI>, &cfg) != cudaSuccess || max_clusters < 1) {
-      (void)cudaGetLastError();
-      max_clusters = num_sms() / 2;
-    }
-    // one CTA per SM (shared memory and all 512 TMEM columns): never more clusters than SM pairs
-    if (max_clusters > num_sms() / 2) max_clusters = num_sms() / 2;
-  }
-  const int pairs = ((M + BM - 1) / BM + 1) / 2 * (N / BN);
-  cfg.gridDim = dim3(2 * (pairs < max_clusters ? pairs : max_clusters));
+  static PerDeviceOnce attr;
+  DLMZ_TRY(attr.run([] {
+    return cudaFuncSetAttribute(gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  }));
+  // persistent: one CTA per SM (shared memory and all 512 TMEM columns) walks the tiles
+  const int m_tiles = (M + BM - 1) / BM;
+  const long tiles = (long)m_tiles * (N / BN);
+  if (tiles > 0x7fffffffl) return DLMZ_EINVAL;
+  const int grid = tiles < num_sms() ? (int)tiles : num_sms();
   const double out_b = EPI == EPI_F32 ? 4.0 * M * N : EPI == EPI_RESID_F32 ? 8.0 * M * N
                      : EPI == EPI_SWIGLU_BF16 ? 1.0 * M * N : 2.0 * M * N;
   ProfScope prof(PROF_GEMM_TC, s, 2.0 * M * N * K, 2.0 * M * K + 2.0 * N * K + out_b);
-  DLMZ_CUDA_TRY(cudaLaunchKernelEx(&cfg, gemm_kernel<EPI>, a, b, M, N, K, ep, device_error_word()));
+  gemm_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(a, b, M, N, K, group_for(m_tiles, K), ep, device_error_word());
   return launch_status();
 }
 
@@ -638,7 +534,7 @@ int gemm_bf16_tc(const __nv_bfloat16* A, int lda, const __nv_bfloat16* B, int ld
   if ((lda | ldb) & 7) return DLMZ_EINVAL;
   CUtensorMap ma, mb;
   DLMZ_TRY(t5::make_map_bf16(&ma, A, M, K, lda, tc::BM, tc::BK));
-  DLMZ_TRY(t5::make_map_bf16(&mb, B, N, K, ldb, tc::BN / 2, tc::BK));  // one CTA of a pair loads half a tile
+  DLMZ_TRY(t5::make_map_bf16(&mb, B, N, K, ldb, tc::BN, tc::BK));
   switch (epi) {
     case EPI_BF16: return tc::launch<EPI_BF16>(ma, mb, M, N, K, ep, s);
     case EPI_F32: return tc::launch<EPI_F32>(ma, mb, M, N, K, ep, s);
