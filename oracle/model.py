@@ -89,14 +89,45 @@ def tensor_shapes(cfg):
     return shapes
 
 
-class Weights:
-    """All parameters of a model as float64 arrays holding storage-dtype values."""
+class _LazyTensors:
+    """Tensors generated on first use (by the C restatement of the draws) for
+    full-size models: the embedding and the head are kept, layer tensors only
+    while their layer is the most recent one asked for, so a forward over 32
+    layers of an 8B-shaped model holds one layer at a time."""
 
-    def __init__(self, cfg, tensors=None):
+    def __init__(self, cfg):
+        self.cfg = cfg
+        self.shapes = tensor_shapes(cfg)
+        self.keep = {}
+        self.layer = {}
+        self.layer_id = None
+
+    def __getitem__(self, tid):
+        if tid in self.keep:
+            return self.keep[tid]
+        if tid in (TID_EMBED, TID_HEAD):
+            self.keep[tid] = W.init_tensor_c(self.cfg.seed, tid, self.shapes[tid], self.cfg.dtype)
+            return self.keep[tid]
+        l = (tid - 2) // 8
+        if l != self.layer_id:
+            self.layer, self.layer_id = {}, l
+        if tid not in self.layer:
+            self.layer[tid] = W.init_tensor_c(self.cfg.seed, tid, self.shapes[tid], self.cfg.dtype)
+        return self.layer[tid]
+
+
+class Weights:
+    """All parameters of a model as float64 arrays holding storage-dtype values.
+
+    ``lazy``: tensors are generated when first used, one layer at a time (for the
+    full-size models; needs oracle/build.py's liboracle.so)."""
+
+    def __init__(self, cfg, tensors=None, lazy=False):
         self.cfg = cfg
         shapes = tensor_shapes(cfg)
         if tensors is None:
-            tensors = {tid: W.init_tensor(cfg.seed, tid, shp, cfg.dtype) for tid, shp in shapes.items()}
+            tensors = (_LazyTensors(cfg) if lazy else
+                       {tid: W.init_tensor(cfg.seed, tid, shp, cfg.dtype) for tid, shp in shapes.items()})
         self.t = tensors
         self.g_attn = [np.ones(cfg.d) for _ in range(cfg.n_layers)]
         self.g_ffn = [np.ones(cfg.d) for _ in range(cfg.n_layers)]
@@ -142,7 +173,15 @@ def silu(x):
     return x / (1.0 + np.exp(-x))
 
 
-def attention(q, k, v, n_heads, n_kv_heads, head_dim, probs=None):
+def _matmul(a, b, dtype):
+    """a @ b with products and sums in ``dtype`` (float64, or float32 for the
+    accumulation-order experiment), returned as float64."""
+    if dtype == np.float64:
+        return a @ b
+    return (a.astype(dtype) @ b.astype(dtype)).astype(np.float64)
+
+
+def attention(q, k, v, n_heads, n_kv_heads, head_dim, probs=None, matmul_dtype=np.float64):
     """Bidirectional multi-head / grouped-query attention over one window.
 
     ``probs`` (a list): receives the head-averaged attention probabilities [L, L].
@@ -157,11 +196,11 @@ def attention(q, k, v, n_heads, n_kv_heads, head_dim, probs=None):
         qh = q[:, h * head_dim:(h + 1) * head_dim]
         kg = k[:, g * head_dim:(g + 1) * head_dim]
         vg = v[:, g * head_dim:(g + 1) * head_dim]
-        s = (qh @ kg.T) * scale
+        s = _matmul(qh, kg.T, matmul_dtype) * scale
         s = s - s.max(axis=1, keepdims=True)
         p = np.exp(s)
         p /= p.sum(axis=1, keepdims=True)
-        out[:, h * head_dim:(h + 1) * head_dim] = p @ vg
+        out[:, h * head_dim:(h + 1) * head_dim] = _matmul(p, vg, matmul_dtype)
         if pavg is not None:
             pavg += p / n_heads
     if probs is not None:
@@ -169,39 +208,44 @@ def attention(q, k, v, n_heads, n_kv_heads, head_dim, probs=None):
     return out
 
 
-def hidden(wts, state, probs=None):
+def hidden(wts, state, probs=None, matmul_dtype=np.float64):
     """Final normed hidden states [L, d] (the LM head input) for one window.
 
     ``probs`` (a list): receives each layer's head-averaged attention [L, L].
+    ``matmul_dtype``: float64 (the oracle), or float32 to run every
+    contraction with float32 products and sums while keeping every storage
+    rounding point -- the accumulation-order experiment that measures how far
+    two faithful evaluations of the same model drift apart at depth.
     """
     cfg = wts.cfg
     rnd = lambda a: W.storage_round(a, cfg.dtype)
     r32 = W.round_f32
     hd = cfg.head_dim
+    mm = lambda a, b: _matmul(a, b, matmul_dtype)
     x = r32(wts.embed[np.asarray(state)])
     for l in range(cfg.n_layers):
         h = rnd(rmsnorm(x, wts.g_attn[l], cfg.norm_eps))
-        q = h @ wts.layer(l, WQ).T
-        k = h @ wts.layer(l, WK).T
-        v = h @ wts.layer(l, WV).T
+        q = mm(h, wts.layer(l, WQ).T)
+        k = mm(h, wts.layer(l, WK).T)
+        v = mm(h, wts.layer(l, WV).T)
         q = rnd(rope(q, cfg.n_heads, hd, cfg.rope_theta))
         k = rnd(rope(k, cfg.n_kv_heads, hd, cfg.rope_theta))
         v = rnd(v)
-        o = rnd(attention(q, k, v, cfg.n_heads, cfg.n_kv_heads, hd, probs))
-        x = r32(x + o @ wts.layer(l, WO).T)
+        o = rnd(attention(q, k, v, cfg.n_heads, cfg.n_kv_heads, hd, probs, matmul_dtype))
+        x = r32(x + mm(o, wts.layer(l, WO).T))
         h = rnd(rmsnorm(x, wts.g_ffn[l], cfg.norm_eps))
-        a = rnd(silu(h @ wts.layer(l, WGATE).T) * (h @ wts.layer(l, WUP).T))
-        x = r32(x + a @ wts.layer(l, WDOWN).T)
+        a = rnd(silu(mm(h, wts.layer(l, WGATE).T)) * mm(h, wts.layer(l, WUP).T))
+        x = r32(x + mm(a, wts.layer(l, WDOWN).T))
     return rnd(rmsnorm(x, wts.g_final, cfg.norm_eps))
 
 
-def forward(wts, state, rows=None):
+def forward(wts, state, rows=None, matmul_dtype=np.float64):
     """Logits [len(rows), V] (float32 values in float64) for one window.
 
     ``state`` holds symbol ids in [0, V] (V = [MASK]); ``rows`` selects the
     positions whose distributions are needed (default: all).
     """
-    h = hidden(wts, state)
+    h = hidden(wts, state, matmul_dtype=matmul_dtype)
     if rows is not None:
         h = h[np.asarray(rows, dtype=np.int64)]
-    return W.round_f32(h @ wts.head.T)
+    return W.round_f32(_matmul(h, wts.head.T, matmul_dtype))

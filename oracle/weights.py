@@ -108,3 +108,61 @@ def init_tensor(seed, tid, shape, dtype):
     n = int(np.prod(shape))
     z = normal_draws(seed, tid, n) * STD
     return storage_round(z, dtype).reshape(shape)
+
+
+# ---- the same draws in plain C (oracle/csrc/normal_draws.c), for full-size models ----------
+_NATIVE = None
+
+
+def _native():
+    """ctypes handle of liboracle.so (built by oracle/build.py), or None when it is not built."""
+    global _NATIVE
+    if _NATIVE is None:
+        import ctypes
+        import os
+        path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "liboracle.so")
+        if not os.path.exists(path):
+            return None
+        lib = ctypes.CDLL(path)
+        lib.oracle_normal_range.restype = None
+        lib.oracle_normal_range.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64, ctypes.c_double,
+                                            ctypes.c_int, ctypes.c_void_p]
+        _NATIVE = lib
+    return _NATIVE
+
+
+_MODES = {None: 0, "f32": 1, "bf16": 2}
+
+
+def normal_draws_c(seed, tid, count, n0=0, threads=None, scale=1.0, dtype=None):
+    """Draws n0 .. n0+count-1 of tensor ``tid`` (as ``normal_draws``) times ``scale``,
+    rounded to ``dtype`` (None: no rounding), computed by the C restatement on
+    ``threads`` host threads (ctypes releases the interpreter lock)."""
+    import concurrent.futures as cf
+    import os
+    lib = _native()
+    if lib is None:
+        raise RuntimeError("liboracle.so is not built (python oracle/build.py)")
+    out = np.empty(count, dtype=np.float64)
+    st = tensor_state(seed, tid)
+    if threads is None:
+        threads = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    step = max(1 << 20, -(-count // max(1, threads)))
+    step += step & 1
+    base = out.ctypes.data
+
+    def run(a):
+        b = min(count, a + step)
+        lib.oracle_normal_range(st, n0 + a, b - a, scale, _MODES[dtype], base + 8 * a)
+
+    with cf.ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
+        list(ex.map(run, range(0, count, step)))
+    return out
+
+
+def init_tensor_c(seed, tid, shape, dtype):
+    """``init_tensor`` with the draws from the C restatement (same values up to the last
+    bits of the float64 log / cos / sin, so equal after rounding to bf16 except with
+    probability ~2^-44 per element)."""
+    n = int(np.prod(shape))
+    return normal_draws_c(seed, tid, n, scale=STD, dtype=dtype).reshape(shape)

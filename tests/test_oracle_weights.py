@@ -69,3 +69,38 @@ def test_round_bf16_ties_to_even():
 
 def test_two_pi_constant():
     assert math.tau == 2 * math.pi
+
+
+def test_c_draws_equal_the_numpy_definition():
+    # the C restatement (used for the full-size models) against the numpy definition:
+    # float64 draws within a few ulp (libm vs numpy log/cos/sin), identical after bf16 /
+    # float32 rounding, from even and odd starting elements
+    from oracle import build
+    build.build()
+    for tid, n0, count in ((3, 0, 100_001), (7, 12_345, 54_321), (1, 1, 4)):
+        ref = W.normal_draws(11, tid, n0 + count)[n0:]
+        got = W.normal_draws_c(11, tid, count, n0=n0, threads=3)
+        assert np.allclose(got, ref, rtol=1e-14, atol=1e-15)
+        assert np.array_equal(W.round_bf16(got * W.STD), W.round_bf16(ref * W.STD))
+    for dt in ("f32", "bf16"):
+        assert np.array_equal(W.init_tensor_c(5, 9, (64, 48), dt), W.init_tensor(5, 9, (64, 48), dt))
+    # the C storage rounding is the oracle's: ties to even at bf16's 8-bit significand, just above
+    # a tie, signs, zero, tiny and large magnitudes; float32 likewise
+    import ctypes
+    lib = W._native()
+    x = np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -(1.0 + 2.0 ** -8), 0.0, 1.0 + 2.0 ** -8 + 2.0 ** -30,
+                  3.0e-30, -7.25e12, 1.0 + 2.0 ** -24, 1.0 + 3 * 2.0 ** -24, 0.1])
+    for mode, ref in ((2, W.round_bf16(x)), (1, W.round_f32(x))):
+        out = np.empty_like(x)
+        lib.oracle_round.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p]
+        lib.oracle_round(x.ctypes.data, x.size, mode, out.ctypes.data)
+        assert np.array_equal(out, ref), mode
+
+
+def test_lazy_weights_forward_equals_eager():
+    from oracle import build
+    from oracle import model as M
+    build.build()
+    cfg = M.ModelConfig(n_layers=3, d=32, n_heads=4, n_kv_heads=2, ffn=64, vocab=50, dtype="bf16", seed=4)
+    s = np.array([1, 50, 7, 50, 49, 0, 3])
+    assert np.array_equal(M.forward(M.Weights(cfg, lazy=True), s), M.forward(M.Weights(cfg), s))
