@@ -80,6 +80,16 @@ DLMZ_API void dlmz_model_destroy(dlmz_model* m);
 DLMZ_API uint64_t dlmz_model_fingerprint(const dlmz_model* m);
 /* Copy the model configuration into *cfg. */
 DLMZ_API int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg);
+/* Memory budget of one denoising step's logits.  A step's LM head and
+ * quantiser run on its candidate rows only -- the masked positions of the
+ * active block of each window, the rows that get a distribution
+ * (Definition 3).  When the candidates' float32 logits [rows x V] exceed
+ * `bytes`, the head and the quantiser's scores run in slabs of rows, and
+ * after the selection the selected rows' logits are computed once more for
+ * the coder (bit-identical: a row's logits depend only on that row).
+ * 0 restores the default (24 GiB).  Streams do not depend on the budget.
+ * Errors: EINVAL (NULL model). */
+DLMZ_API int dlmz_model_set_logits_budget(dlmz_model* m, size_t bytes);
 
 /* ---- commitment schedule (Sec. 3.3) and initial context (Sec. 3.4) ---- */
 #define DLMZ_TOPK_CONF 0u   /* k most confident masked positions of the leftmost incomplete block */
@@ -271,6 +281,26 @@ DLMZ_API int dlmz_encode_step(dlmz_coder* c, const dlmz_k_policy* policy, const 
 DLMZ_API int dlmz_decode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits,
                      uint32_t row0, uint32_t rows_per_chunk, int32_t* d_state,
                      int32_t* d_committed, void* stream);
+/* One denoising step with the model's own distributions (Sec. 3.2), over
+ * the coder's batch (n_chunks windows of L positions, d_state [n_chunks x L],
+ * [MASK] = V): the forward pass of the batch (Definition 3), the LM head and
+ * the quantiser on the candidate rows only -- the masked positions of
+ * [row0, row0 + rows_per_chunk) in each window -- the selection of the policy
+ * (Sec. 3.3; confidence or entropy keys, or the k leftmost masked positions
+ * for UNIFORM / PROGRESSIVE with k = the step's size), then the coding
+ * (encode: the true symbols d_symbols [n_chunks x L]) or decoding of the
+ * selected positions, which are revealed in d_state.  d_committed (optional,
+ * [n_chunks]) receives the count per window.  The model's V must be the
+ * coder's and P the library's precision for it (16 for V <= 4096, else 24);
+ * policy->coder must be the coder's kind and policy->context NONE (a caller
+ * that wants an initial context reveals it in d_state itself).  Synchronises
+ * once with the host per call (the candidate count sizes the LM head).
+ * Errors: EINVAL, ENOMEM, ECUDA; stream corruption shows at dlmz_check. */
+DLMZ_API int dlmz_model_encode_step(dlmz_model* m, dlmz_coder* c, const dlmz_k_policy* policy, uint32_t row0,
+                                    uint32_t rows_per_chunk, const int32_t* d_symbols, int32_t* d_state,
+                                    int32_t* d_committed, void* stream);
+DLMZ_API int dlmz_model_decode_step(dlmz_model* m, dlmz_coder* c, const dlmz_k_policy* policy, uint32_t row0,
+                                    uint32_t rows_per_chunk, int32_t* d_state, int32_t* d_committed, void* stream);
 /* Terminate every stream (call once per encoded batch): bit lengths to
  * d_bits [n_chunks]; if d_bytes is not NULL each stream's ceil(bits/8) bytes
  * are copied to d_bytes + d_offsets[c], or to d_bytes + c * 2 *
@@ -282,6 +312,14 @@ DLMZ_API uint32_t dlmz_coder_capacity_units(const dlmz_coder* c);
 /* Synchronise and report any device-side error flag (ECORRUPT for a stream
  * that cannot come from the encoder, ETIMEOUT, EBADINPUT). */
 DLMZ_API int dlmz_check(void* stream);
+
+/* Failure-detection self-test (not part of the method): launches a kernel
+ * whose bounded mbarrier wait (the kind every pipeline kernel uses) gives up
+ * after limit_us microseconds (1 .. 1e6) because nothing arrives.  Returns
+ * DLMZ_ETIMEOUT when the timeout was detected and reported the way a stuck
+ * pipeline wait is; the device error word is cleared and the context stays
+ * usable.  Errors: EINVAL (limit), ECUDA. */
+DLMZ_API int dlmz_selftest_wait_timeout(uint32_t limit_us, void* stream);
 
 /* ---- live profiling (not part of the method) ------------------------------
  * Between dlmz_profile_begin and dlmz_profile_end the library records CUDA

@@ -33,8 +33,9 @@ static __constant__ uint32_t c_exp_table[256] = DLMZ_EXP_TABLE_INIT;
 // ---- selection ----------------------------------------------------------------------
 template <typename K>
 __global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask_id, int row0, int rpc,
-                              const K* __restrict__ keys, int n_rule, int k, int64_t tau_q, int k_min, int k_max,
-                              int kcap, int32_t* __restrict__ sel_count, int32_t* __restrict__ sel_pos) {
+                              const K* __restrict__ keys, const int32_t* __restrict__ row_map, int n_rule, int k,
+                              int64_t tau_q, int k_min, int k_max, int kcap, int32_t* __restrict__ sel_count,
+                              int32_t* __restrict__ sel_pos) {
   extern __shared__ uint64_t skey[];  // rpc keys, then rpc flags (as bytes)
   uint8_t* valid = reinterpret_cast<uint8_t*>(skey + rpc);
   __shared__ int red[32];
@@ -43,7 +44,9 @@ __global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask
   int nv = 0, nb = 0;
   for (int i = threadIdx.x; i < rpc; i += blockDim.x) {
     const bool ok = state ? state[(size_t)c * L + row0 + i] == mask_id : true;
-    const uint64_t key = keys ? (uint64_t)(int64_t)keys[(size_t)c * rpc + i] : 0;  // null: position order
+    // null keys: position order; with a row map only candidates have a key row
+    const int64_t kr = row_map ? (ok ? row_map[(size_t)c * rpc + i] : -1) : (int64_t)c * rpc + i;
+    const uint64_t key = keys && kr >= 0 ? (uint64_t)(int64_t)keys[kr] : 0;
     skey[i] = key;
     valid[i] = ok;
     nv += ok;
@@ -105,24 +108,22 @@ __global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask
 template <typename K>
 int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0, int rpc, const K* keys, int n_rule,
                 int k, int64_t tau_q, int k_min, int k_max, int kcap, int32_t* sel_count, int32_t* sel_pos,
-                cudaStream_t s) {
+                cudaStream_t s, const int32_t* row_map) {
   if (n_chunks == 0) return DLMZ_OK;
   const size_t smem = (size_t)rpc * 9 + 16;
   if (smem > 200 * 1024) return DLMZ_EINVAL;
-  static bool attr = false;
-  if (!attr) {
-    DLMZ_CUDA_TRY(cudaFuncSetAttribute(select_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024));
-    attr = true;
-  }
+  static PerDeviceOnce attr;
+  DLMZ_TRY(attr.run(
+      [] { return cudaFuncSetAttribute(select_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024); }));
   ProfScope prof(PROF_SELECT, s, 0, (double)n_chunks * rpc * (sizeof(K) + 4));
-  select_kernel<K><<<n_chunks, 256, smem, s>>>(state, L, mask_id, row0, rpc, keys, n_rule, k, tau_q, k_min, k_max,
-                                               kcap, sel_count, sel_pos);
+  select_kernel<K><<<n_chunks, 256, smem, s>>>(state, L, mask_id, row0, rpc, keys, row_map, n_rule, k, tau_q, k_min,
+                                               k_max, kcap, sel_count, sel_pos);
   return launch_status();
 }
 template int select_rows<uint64_t>(const int32_t*, int, int, int, int, int, const uint64_t*, int, int, int64_t, int,
-                                   int, int, int32_t*, int32_t*, cudaStream_t);
+                                   int, int, int32_t*, int32_t*, cudaStream_t, const int32_t*);
 template int select_rows<int32_t>(const int32_t*, int, int, int, int, int, const int32_t*, int, int, int64_t, int,
-                                  int, int, int32_t*, int32_t*, cudaStream_t);
+                                  int, int, int32_t*, int32_t*, cudaStream_t, const int32_t*);
 
 // ---- range coder -----------------------------------------------------------------------
 constexpr uint64_t RENORM = 1ull << 48;
@@ -214,7 +215,11 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
   const uint64_t dn = DECODE ? (a.in_bits[c] + 7) / 8 : 0;
   for (int j = 0; j < n; ++j) {
     const int pos = a.sel_pos[(size_t)c * a.kcap + j];
-    const size_t row = (size_t)c * a.rpc + (pos - a.row0);
+    // the row of this position's logits and stats: through the candidate map, the j-th
+    // selected row of the window, or the dense row of [row0, row0 + rpc)
+    const size_t row = a.row_map ? (size_t)a.row_map[(size_t)c * a.rpc + (pos - a.row0)]
+                     : a.sel_major ? (size_t)c * a.kcap + j
+                                   : (size_t)c * a.rpc + (pos - a.row0);
     const float* lr = a.logits + row * V;
     const float m = a.mx[row];
     const uint64_t Wr = a.W[row];

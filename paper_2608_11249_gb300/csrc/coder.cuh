@@ -18,7 +18,7 @@ struct CoderState {
 };
 
 struct CodeArgs {
-  const float* logits;       // [n_chunks * rpc x V]
+  const float* logits;       // [n_chunks * rpc x V], or rows found through row_map / sel_major
   const float* mx;           // per row: max logit
   const uint64_t* W;         // per row: W
   const int32_t* top;        // per row: lowest argmax
@@ -38,12 +38,16 @@ struct CodeArgs {
   int coder;                 // 0: range coder, 1: rANS, 2: symbol ranks (varints)
   uint64_t* pairs;           // rANS encoder: (c << 32 | f) per coded symbol [n_chunks x pair_cap]
   int pair_cap;
+  const int32_t* row_map;    // optional [n_chunks x rpc]: row of logits / mx / W / top of each candidate
+  int sel_major;             // without row_map: row of the j-th selected position = c * kcap + j
 };
 
+// keys of window c's position row0 + i: keys[row_map[c * rpc + i]] when row_map is
+// given (candidates only), else keys[c * rpc + i].
 template <typename K>
 int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0, int rpc, const K* keys, int n_rule,
                 int k, int64_t tau_q, int k_min, int k_max, int kcap, int32_t* sel_count, int32_t* sel_pos,
-                cudaStream_t s);
+                cudaStream_t s, const int32_t* row_map = nullptr);
 int code_step(const CodeArgs& a, bool decode, int n_chunks, cudaStream_t s);
 int coder_reset(CoderState* st, int n, cudaStream_t s);
 int coder_load(CoderState* st, int n, const uint8_t* bytes, const uint64_t* offsets, const uint32_t* bits, int coder,

@@ -61,6 +61,10 @@ int embed(const int32_t* state, int T_tokens, const T* E, int d, float* x, cudaS
 template <typename OutT>
 int rmsnorm(const float* x, int rows, int d, const float* g, float eps, OutT* h, int L, int row0,
             int rpc, cudaStream_t s);
+// h[r] = OutT(x[idx[r]] * g / sqrt(mean(x^2) + eps)) (rows gathered by token index).
+template <typename OutT>
+int rmsnorm_gather(const float* x, const int32_t* idx, int rows, int d, const float* g, float eps, OutT* h,
+                   cudaStream_t s);
 template <typename T>
 int rope_inplace(T* qkv, int T_tokens, int ld, int n_heads_rot, int head_dim, int L,
                  const float2* cs, cudaStream_t s);

@@ -59,11 +59,12 @@ template int embed<bf16>(const int32_t*, int, const bf16*, int, float*, cudaStre
 // ---- RMSNorm (one warp per row), optional row gather ------------------------------
 template <typename OutT>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int rows, int d, const float* __restrict__ g,
-                               float eps, OutT* __restrict__ h, int L, int row0, int rpc) {
+                               float eps, OutT* __restrict__ h, int L, int row0, int rpc,
+                               const int32_t* __restrict__ idx) {
   const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
-  const size_t src = rpc > 0 ? (size_t)(r / rpc) * L + row0 + (r % rpc) : (size_t)r;
+  const size_t src = idx ? (size_t)idx[r] : rpc > 0 ? (size_t)(r / rpc) * L + row0 + (r % rpc) : (size_t)r;
   const float* xr = x + src * d;
   float ss = 0.f;
   for (int i = lane; i < d; i += 32) ss += xr[i] * xr[i];
@@ -79,11 +80,22 @@ int rmsnorm(const float* x, int rows, int d, const float* g, float eps, OutT* h,
             cudaStream_t s) {
   if (rows == 0) return DLMZ_OK;
   ProfScope prof(PROF_LAYER, s, 0, (double)rows * d * (4 + sizeof(OutT)));
-  rmsnorm_kernel<OutT><<<(rows + 7) / 8, 256, 0, s>>>(x, rows, d, g, eps, h, L, row0, rpc);
+  rmsnorm_kernel<OutT><<<(rows + 7) / 8, 256, 0, s>>>(x, rows, d, g, eps, h, L, row0, rpc, nullptr);
   return launch_status();
 }
 template int rmsnorm<float>(const float*, int, int, const float*, float, float*, int, int, int, cudaStream_t);
 template int rmsnorm<bf16>(const float*, int, int, const float*, float, bf16*, int, int, int, cudaStream_t);
+
+template <typename OutT>
+int rmsnorm_gather(const float* x, const int32_t* idx, int rows, int d, const float* g, float eps, OutT* h,
+                   cudaStream_t s) {
+  if (rows == 0) return DLMZ_OK;
+  ProfScope prof(PROF_LAYER, s, 0, (double)rows * d * (4 + sizeof(OutT)));
+  rmsnorm_kernel<OutT><<<(rows + 7) / 8, 256, 0, s>>>(x, rows, d, g, eps, h, 0, 0, 0, idx);
+  return launch_status();
+}
+template int rmsnorm_gather<float>(const float*, const int32_t*, int, int, const float*, float, float*, cudaStream_t);
+template int rmsnorm_gather<bf16>(const float*, const int32_t*, int, int, const float*, float, bf16*, cudaStream_t);
 
 // ---- RoPE in place on the Q and K heads of the fused qkv buffer -----------------
 template <typename T>

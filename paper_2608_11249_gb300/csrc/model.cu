@@ -133,14 +133,15 @@ static int gemm(const T* A, const T* B, int M, int N, int K, int epi, const Gemm
   return gemm_simt<T>(A, K, B, K, M, N, K, epi, ep, s);
 }
 
-// maps (optional): every layer's head-averaged attention [n_layers][nc][L][L]; without
-// logits the LM head is skipped.
+// The layers of the forward (embedding through the last residual add) of nc
+// windows of L positions; the float32 residual stream is left in ws.x for the
+// LM head.  maps (optional): every layer's head-averaged attention
+// [n_layers][nc][L][L].
 template <typename T>
-static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int row0, int rpc, float* logits,
-                        cudaStream_t s, float* maps = nullptr) {
+static int layers_impl(dlmz_model* m, const int32_t* state, int nc, int L, cudaStream_t s, float* maps = nullptr) {
   const dlmz_model_config& c = m->cfg;
-  const int d = c.d, F = c.ffn, V = c.vocab, hd = m->hd, nq = m->nqkv;
-  const int Tt = nc * L, R = nc * rpc;
+  const int d = c.d, F = c.ffn, hd = m->hd, nq = m->nqkv;
+  const int Tt = nc * L;
   ForwardWorkspace& w = m->ws;
   DLMZ_TRY(w.x.ensure((size_t)Tt * d * 4));
   DLMZ_TRY(w.h.ensure((size_t)Tt * d * sizeof(T)));
@@ -148,7 +149,6 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
   DLMZ_TRY(w.attn.ensure((size_t)Tt * d * sizeof(T)));
   DLMZ_TRY(w.act.ensure((size_t)Tt * F * sizeof(T)));
   if (!m->tc) DLMZ_TRY(w.gu.ensure((size_t)Tt * 2 * F * 4));
-  DLMZ_TRY(w.hc.ensure((size_t)R * d * sizeof(T)));
   // tensor-core attention reads V transposed (keys contiguous), written by the QKV epilogue
   const bool tc_attn = m->tc && attention_tc_supported(L, hd);
   if (tc_attn) {
@@ -262,24 +262,54 @@ static int forward_impl(dlmz_model* m, const int32_t* state, int nc, int L, int 
       DLMZ_TRY(gemm<T>(act, reinterpret_cast<const T*>(m->wdown[l]), Tt, d, F, EPI_RESID_F32, ep, s));
     }
   }
-  if (!logits) return DLMZ_OK;
+  m->ws.x_tokens = Tt;
+  return DLMZ_OK;
+}
+
+// LM head on R rows of the residual stream left by the last layers_impl:
+// final RMSNorm of x rows (idx[r] when idx is given, else
+// (r / rpc) * L + row0 + r % rpc) and f32 logits [R x V].
+template <typename T>
+static int head_impl(dlmz_model* m, const int32_t* idx, int R, int L, int row0, int rpc, float* logits,
+                     cudaStream_t s) {
+  const dlmz_model_config& c = m->cfg;
+  const int d = c.d, V = c.vocab;
+  if (R == 0) return DLMZ_OK;
+  ForwardWorkspace& w = m->ws;
+  DLMZ_TRY(w.hc.ensure((size_t)R * d * sizeof(T)));
   T* hc = w.hc.as<T>();
-  DLMZ_TRY(rmsnorm<T>(x, R, d, m->gains, c.norm_eps, hc, L, row0, rpc, s));
-  ep = epi(logits, V);
+  if (idx) DLMZ_TRY(rmsnorm_gather<T>(w.x.as<float>(), idx, R, d, m->gains, c.norm_eps, hc, s));
+  else DLMZ_TRY(rmsnorm<T>(w.x.as<float>(), R, d, m->gains, c.norm_eps, hc, L, row0, rpc, s));
+  GemmEpilogue ep{};
+  ep.out = logits;
+  ep.ldo = V;
   return gemm<T>(hc, reinterpret_cast<const T*>(m->head), R, V, d, EPI_F32, ep, s);
 }
 
 int model_attention_maps(dlmz_model* m, const int32_t* state, int nc, int L, float* maps, cudaStream_t s) {
   if (nc <= 0 || L <= 0 || !maps) return DLMZ_EINVAL;
-  if (m->bf16) return forward_impl<bf16>(m, state, nc, L, 0, 1, nullptr, s, maps);
-  return forward_impl<float>(m, state, nc, L, 0, 1, nullptr, s, maps);
+  if (m->bf16) return layers_impl<bf16>(m, state, nc, L, s, maps);
+  return layers_impl<float>(m, state, nc, L, s, maps);
+}
+
+int model_layers(dlmz_model* m, const int32_t* state, int nc, int L, cudaStream_t s) {
+  if (nc <= 0 || L <= 0) return DLMZ_EINVAL;
+  if (m->bf16) return layers_impl<bf16>(m, state, nc, L, s);
+  return layers_impl<float>(m, state, nc, L, s);
+}
+
+int model_head(dlmz_model* m, const int32_t* idx, int n, float* logits, cudaStream_t s) {
+  if (n < 0 || (n > 0 && (!idx || !logits))) return DLMZ_EINVAL;
+  if (m->bf16) return head_impl<bf16>(m, idx, n, 0, 0, 0, logits, s);
+  return head_impl<float>(m, idx, n, 0, 0, 0, logits, s);
 }
 
 int model_forward(dlmz_model* m, const int32_t* state, int nc, int L, int row0, int rpc, float* logits,
                   cudaStream_t s) {
   if (nc <= 0 || L <= 0 || rpc <= 0 || row0 < 0 || row0 + rpc > L) return DLMZ_EINVAL;
-  if (m->bf16) return forward_impl<bf16>(m, state, nc, L, row0, rpc, logits, s);
-  return forward_impl<float>(m, state, nc, L, row0, rpc, logits, s);
+  DLMZ_TRY(model_layers(m, state, nc, L, s));
+  if (m->bf16) return head_impl<bf16>(m, nullptr, nc * rpc, L, row0, rpc, logits, s);
+  return head_impl<float>(m, nullptr, nc * rpc, L, row0, rpc, logits, s);
 }
 
 }  // namespace dlmz
@@ -410,6 +440,12 @@ extern "C" void dlmz_model_destroy(dlmz_model* m) {
 }
 
 extern "C" uint64_t dlmz_model_fingerprint(const dlmz_model* m) { return m ? m->fingerprint : 0; }
+
+extern "C" int dlmz_model_set_logits_budget(dlmz_model* m, size_t bytes) {
+  if (!m) return DLMZ_EINVAL;
+  m->logits_budget = bytes;
+  return DLMZ_OK;
+}
 
 extern "C" int dlmz_model_get_config(const dlmz_model* m, dlmz_model_config* cfg) {
   if (!m || !cfg) return DLMZ_EINVAL;

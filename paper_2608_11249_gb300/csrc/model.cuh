@@ -36,6 +36,7 @@ struct DevBuf {
 struct ForwardWorkspace {
   DevBuf x, h, qkv, attn, act, gu, hc, rope, vt, ssq;
   int rope_L = 0;
+  int64_t x_tokens = 0;  // rows of x written by the last model_layers
 };
 
 }  // namespace dlmz
@@ -54,6 +55,7 @@ struct dlmz_model {
   uint64_t fingerprint = 0;
   dlmz::ForwardWorkspace ws;
   void* pipe = nullptr;  // pipeline workspace (owned, see pipeline.cu)
+  size_t logits_budget = 0;  // bytes of candidate logits a step holds at once (0: the default)
 };
 
 namespace dlmz {
@@ -61,6 +63,15 @@ namespace dlmz {
 // [row0, row0+rpc) of every window.
 int model_forward(dlmz_model* m, const int32_t* state, int n_chunks, int L, int row0, int rpc, float* logits,
                   cudaStream_t s);
+// The layers of the forward (embedding through the last residual add) of a
+// batch; the float32 residual stream stays in the model's workspace until the
+// next call, for model_head.
+int model_layers(dlmz_model* m, const int32_t* state, int n_chunks, int L, cudaStream_t s);
+// LM head on n rows of the last model_layers batch: final RMSNorm of the
+// residual rows idx[0..n) (token index = window * L + position) and float32
+// logits [n x V].  Each row's logits depend only on that row, so a row gives
+// bit-identical logits in any call and at any place in idx.
+int model_head(dlmz_model* m, const int32_t* idx, int n, float* logits, cudaStream_t s);
 // Every layer's head-averaged attention probabilities [n_layers][n_chunks][L][L]
 // for the windows' states (no LM head).
 int model_attention_maps(dlmz_model* m, const int32_t* state, int n_chunks, int L, float* maps, cudaStream_t s);

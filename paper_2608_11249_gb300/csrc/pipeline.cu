@@ -31,13 +31,17 @@
 namespace dlmz {
 
 // ---- error word -------------------------------------------------------------------------
-static int* g_err = nullptr;
+static int* g_err[kMaxDevices] = {};
 int* device_error_word() {
-  if (!g_err) {
-    if (cudaMalloc(&g_err, sizeof(int)) != cudaSuccess) return nullptr;
-    cudaMemset(g_err, 0, sizeof(int));
+  const int dev = device_ordinal();
+  if (dev < 0) return nullptr;
+  if (!g_err[dev]) {
+    int* p = nullptr;
+    if (cudaMalloc(&p, sizeof(int)) != cudaSuccess) return nullptr;
+    cudaMemset(p, 0, sizeof(int));
+    g_err[dev] = p;
   }
-  return g_err;
+  return g_err[dev];
 }
 
 static int clear_device_error(cudaStream_t s) {
@@ -259,6 +263,12 @@ struct BatchContext {
 // ---- per-batch step state ---------------------------------------------------------
 struct StepBufs {
   DevBuf logits, W, Hq, top, mx, sel_count, sel_pos, committed, sum, pairs;
+  // candidate rows of a model step: per-window counts, offsets [nc + 1], token index of
+  // each candidate, the candidate row of each position of [row0, row0 + rpc) (-1: none),
+  // token index of each selected row and the stats of the recomputed selected rows
+  DevBuf cand_count, cand_off, cand_total, cand_tok, row_map, sel_tok, sW, sHq, stop, smx;
+  int64_t* host_total = nullptr;  // pinned: candidate count of the step, read while the layers run
+  cudaEvent_t total_ready = nullptr;
   int ensure(size_t rows, int V, int nc, int kcap) {
     DLMZ_TRY(logits.ensure(rows * (size_t)V * 4));
     DLMZ_TRY(W.ensure(rows * 8));
@@ -271,11 +281,148 @@ struct StepBufs {
     DLMZ_TRY(sum.ensure(8));
     return DLMZ_OK;
   }
+  int ensure_cand(int nc, int rpc, int kcap) {
+    DLMZ_TRY(cand_count.ensure((size_t)nc * 4));
+    DLMZ_TRY(cand_off.ensure((size_t)nc * 4 + 4));
+    DLMZ_TRY(cand_tok.ensure((size_t)nc * rpc * 4));
+    DLMZ_TRY(row_map.ensure((size_t)nc * rpc * 4));
+    DLMZ_TRY(sel_tok.ensure((size_t)nc * kcap * 4));
+    DLMZ_TRY(cand_total.ensure(8));
+    if (!host_total) {
+      void* h = nullptr;
+      if (cudaMallocHost(&h, 8) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return DLMZ_ENOMEM;
+      }
+      host_total = reinterpret_cast<int64_t*>(h);
+    }
+    if (!total_ready) DLMZ_CUDA_TRY(cudaEventCreateWithFlags(&total_ready, cudaEventDisableTiming));
+    return DLMZ_OK;
+  }
+  int ensure_sel_stats(size_t rows) {
+    DLMZ_TRY(sW.ensure(rows * 8));
+    DLMZ_TRY(sHq.ensure(rows * 4));
+    DLMZ_TRY(stop.ensure(rows * 4));
+    DLMZ_TRY(smx.ensure(rows * 4));
+    return DLMZ_OK;
+  }
   void release() {
     logits.release(); W.release(); Hq.release(); top.release(); mx.release();
     sel_count.release(); sel_pos.release(); committed.release(); sum.release(); pairs.release();
+    cand_count.release(); cand_off.release(); cand_total.release(); cand_tok.release(); row_map.release(); sel_tok.release();
+    sW.release(); sHq.release(); stop.release(); smx.release();
+    if (host_total) cudaFreeHost(host_total);
+    host_total = nullptr;
+    if (total_ready) cudaEventDestroy(total_ready);
+    total_ready = nullptr;
   }
 };
+
+// ---- candidate rows of a model step ------------------------------------------------
+// The candidates of a step are the masked positions of [row0, row0 + rpc) in each
+// window (Definition 3: one distribution per masked position); only they go
+// through the LM head and the quantiser.
+__device__ __forceinline__ int block_sum_i32(int v, int* red) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  int t = 0;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t += red[i];
+  return t;
+}
+
+__global__ void cand_count_kernel(const int32_t* __restrict__ state, int L, int mask_id, int row0, int rpc,
+                                  int32_t* __restrict__ counts) {
+  __shared__ int red[32];
+  const int c = blockIdx.x;
+  int n = 0;
+  for (int i = threadIdx.x; i < rpc; i += blockDim.x) n += state[(size_t)c * L + row0 + i] == mask_id;
+  n = block_sum_i32(n, red);
+  if (threadIdx.x == 0) counts[c] = n;
+}
+
+// offsets[i] = counts[0] + ... + counts[i - 1] for i <= nc, and *total = offsets[nc]; one CTA.
+__global__ void cand_scan_kernel(const int32_t* __restrict__ counts, int nc, int32_t* __restrict__ offsets,
+                                 int64_t* __restrict__ total) {
+  __shared__ int wsum[32];
+  __shared__ int carry;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int b = 0; b < nc; b += blockDim.x) {
+    const int i = b + threadIdx.x;
+    const int v = i < nc ? counts[i] : 0;
+    int inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += t;
+    }
+    if (lane == 31) wsum[w] = inc;
+    __syncthreads();
+    if (w == 0) {
+      int x = lane < nw ? wsum[lane] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += t;
+      }
+      if (lane < nw) wsum[lane] = x;  // inclusive over warps
+    }
+    __syncthreads();
+    const int pre = carry + (w > 0 ? wsum[w - 1] : 0) + inc - v;
+    if (i < nc) offsets[i] = pre;
+    __syncthreads();
+    if (threadIdx.x == 0) carry += wsum[nw - 1];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    offsets[nc] = carry;
+    *total = carry;
+  }
+}
+
+// Candidates of window c in ascending position: token index (c * L + position) at
+// offsets[c] + rank, and row_map[c * rpc + i] = that row (or -1 for a committed position).
+__global__ void cand_write_kernel(const int32_t* __restrict__ state, int L, int mask_id, int row0, int rpc,
+                                  const int32_t* __restrict__ offsets, int32_t* __restrict__ cand_tok,
+                                  int32_t* __restrict__ row_map) {
+  __shared__ int wcount[32];
+  const int c = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int base = offsets[c];
+  for (int i0 = 0; i0 < rpc; i0 += blockDim.x) {
+    const int i = i0 + threadIdx.x;
+    const bool ok = i < rpc && state[(size_t)c * L + row0 + i] == mask_id;
+    const unsigned bal = __ballot_sync(0xffffffffu, ok);
+    if (lane == 0) wcount[w] = __popc(bal);
+    __syncthreads();
+    int off = base, tot = 0;
+    for (int j = 0; j < nw; ++j) {
+      if (j < w) off += wcount[j];
+      tot += wcount[j];
+    }
+    if (i < rpc) {
+      const int r = ok ? off + __popc(bal & ((1u << lane) - 1)) : -1;
+      row_map[(size_t)c * rpc + i] = r;
+      if (ok) cand_tok[r] = c * L + row0 + i;
+    }
+    base += tot;
+    __syncthreads();
+  }
+}
+
+// Token index of the j-th selected position of each window (row c * kcap + j); rows
+// past a window's count repeat its position 0 (their logits are never read).
+__global__ void sel_tok_kernel(const int32_t* __restrict__ sel_count, const int32_t* __restrict__ sel_pos, int nc,
+                               int L, int kcap, int32_t* __restrict__ tok) {
+  const int64_t n = (int64_t)nc * kcap;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const int c = (int)(i / kcap), j = (int)(i % kcap);
+    tok[i] = c * L + (j < sel_count[c] ? sel_pos[i] : 0);
+  }
+}
 
 static int kcap_for(const dlmz_k_policy& p, int rpc) {
   int k = p.kind != DLMZ_ENTROPY ? (int)p.k : (p.k_max ? (int)p.k_max : rpc);
@@ -285,7 +432,75 @@ static int kcap_for(const dlmz_k_policy& p, int rpc) {
 
 static int64_t tau_q_of(float tau) { return (int64_t)floor((double)tau * 65536.0); }
 
-// quantise + select + code one step on logits of rows [row0, row0+rpc) of each window
+static int precision_for(uint32_t V) { return V <= 4096 ? 16 : 24; }
+
+// Where a step's symbols come from and go to (encoder: symbols, streams; decoder: the
+// file's streams), and the coder state of the batch's windows.
+struct StepIO {
+  const int32_t* symbols;
+  int32_t* state;
+  CoderState* cst;
+  uint8_t* ebytes;
+  uint64_t cap_bytes;
+  const uint8_t* in_bytes;
+  const uint64_t* in_off;
+  const uint32_t* in_bits;
+  bool decode;
+  int32_t* committed;
+};
+
+// Selection (Sec. 3.3) on the keys in sb.W (confidence) / sb.Hq (entropy); a key row is
+// found through row_map when given.
+static int select_step(StepBufs& sb, const int32_t* state, int nc, int L, int V, const dlmz_k_policy& pol, int row0,
+                       int rpc, int kcap, const int32_t* row_map, cudaStream_t s) {
+  if (pol.kind != DLMZ_ENTROPY)  // left-to-right schedules: the k leftmost masked rows (keys ignored)
+    return select_rows<uint64_t>(state, nc, L, V, row0, rpc, pol.kind == DLMZ_TOPK_CONF ? sb.W.as<uint64_t>() : nullptr,
+                                 0, (int)pol.k, 0, 0, 0, kcap, sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), s,
+                                 row_map);
+  return select_rows<int32_t>(state, nc, L, V, row0, rpc, sb.Hq.as<int32_t>(), 1, 0, tau_q_of(pol.tau_bits),
+                              (int)pol.k_min, (int)pol.k_max, kcap, sb.sel_count.as<int32_t>(),
+                              sb.sel_pos.as<int32_t>(), s, row_map);
+}
+
+// Frequency of the selected rows, code (or decode) and reveal (Sec. 3.2).
+static int code_rows(StepBufs& sb, const StepIO& io, const float* logits, const float* mx, const uint64_t* W,
+                     const int32_t* top, const int32_t* row_map, bool sel_major, int nc, int L, int V, int P,
+                     const dlmz_k_policy& pol, int row0, int rpc, int kcap, cudaStream_t s) {
+  CodeArgs a{};
+  a.logits = logits;
+  a.mx = mx;
+  a.W = W;
+  a.top = top;
+  a.row_map = row_map;
+  a.sel_major = sel_major ? 1 : 0;
+  a.sel_count = sb.sel_count.as<int32_t>();
+  a.sel_pos = sb.sel_pos.as<int32_t>();
+  a.symbols = io.symbols;
+  a.state = io.state;
+  a.state_c = io.cst;
+  a.bytes = io.ebytes;
+  a.cap_bytes = io.cap_bytes;
+  a.in_bytes = io.in_bytes;
+  a.in_offsets = io.in_off;
+  a.in_bits = io.in_bits;
+  a.committed = io.committed;
+  a.err = device_error_word();
+  a.V = V;
+  a.P = P;
+  a.L = L;
+  a.row0 = row0;
+  a.rpc = rpc;
+  a.kcap = kcap;
+  a.coder = (int)pol.coder;
+  if (pol.coder == DLMZ_CODER_RANS && !io.decode) {  // one (c, f) pair per position of every window
+    DLMZ_TRY(sb.pairs.ensure((size_t)nc * L * 8));
+    a.pairs = sb.pairs.as<uint64_t>();
+    a.pair_cap = L;
+  }
+  return code_step(a, io.decode, nc, s);
+}
+
+// quantise + select + code one step on caller-given logits of rows [row0, row0+rpc) of each window
 static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int P, const dlmz_k_policy& pol,
                     int row0, int rpc, const int32_t* symbols, int32_t* state, CoderState* cst, uint8_t* ebytes,
                     uint64_t cap_bytes, const uint8_t* in_bytes, const uint64_t* in_off, const uint32_t* in_bits,
@@ -295,44 +510,77 @@ static int run_step(StepBufs& sb, const float* logits, int nc, int L, int V, int
   DLMZ_TRY(sb.ensure(rows, 1, nc, kcap));
   DLMZ_TRY(quantize_rows(logits, rows, V, P, nullptr, sb.W.as<uint64_t>(), nullptr, sb.Hq.as<int32_t>(),
                          sb.top.as<int32_t>(), sb.mx.as<float>(), s));
-  if (pol.kind != DLMZ_ENTROPY)  // left-to-right schedules: the k leftmost masked rows (keys ignored)
-    DLMZ_TRY(select_rows<uint64_t>(state, nc, L, V, row0, rpc,
-                                   pol.kind == DLMZ_TOPK_CONF ? sb.W.as<uint64_t>() : nullptr, 0, (int)pol.k, 0, 0,
-                                   0, kcap, sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), s));
-  else
-    DLMZ_TRY(select_rows<int32_t>(state, nc, L, V, row0, rpc, sb.Hq.as<int32_t>(), 1, 0, tau_q_of(pol.tau_bits),
-                                  (int)pol.k_min, (int)pol.k_max, kcap, sb.sel_count.as<int32_t>(),
-                                  sb.sel_pos.as<int32_t>(), s));
-  CodeArgs a{};
-  a.logits = logits;
-  a.mx = sb.mx.as<float>();
-  a.W = sb.W.as<uint64_t>();
-  a.top = sb.top.as<int32_t>();
-  a.sel_count = sb.sel_count.as<int32_t>();
-  a.sel_pos = sb.sel_pos.as<int32_t>();
-  a.symbols = symbols;
-  a.state = state;
-  a.state_c = cst;
-  a.bytes = ebytes;
-  a.cap_bytes = cap_bytes;
-  a.in_bytes = in_bytes;
-  a.in_offsets = in_off;
-  a.in_bits = in_bits;
-  a.committed = committed;
-  a.err = device_error_word();
-  a.V = V;
-  a.P = P;
-  a.L = L;
-  a.row0 = row0;
-  a.rpc = rpc;
-  a.kcap = kcap;
-  a.coder = (int)pol.coder;
-  if (pol.coder == DLMZ_CODER_RANS && !decode) {  // one (c, f) pair per position of every window
-    DLMZ_TRY(sb.pairs.ensure((size_t)nc * L * 8));
-    a.pairs = sb.pairs.as<uint64_t>();
-    a.pair_cap = L;
+  DLMZ_TRY(select_step(sb, state, nc, L, V, pol, row0, rpc, kcap, nullptr, s));
+  const StepIO io{symbols, state, cst, ebytes, cap_bytes, in_bytes, in_off, in_bits, decode, committed};
+  return code_rows(sb, io, logits, sb.mx.as<float>(), sb.W.as<uint64_t>(), sb.top.as<int32_t>(), nullptr, false, nc,
+                   L, V, P, pol, row0, rpc, kcap, s);
+}
+
+// Bytes of float32 logits one model step may hold at once (rows beyond it go through
+// the LM head in slabs).
+static size_t logits_budget(const dlmz_model* m) {
+  return m->logits_budget ? m->logits_budget : ((size_t)24 << 30);
+}
+
+// One step of the iterative pipeline with the model's own distributions: the
+// forward over the batch, the LM head and the quantiser on the candidate rows
+// only (the masked positions of [row0, row0 + rpc) in each window), selection,
+// and the coding of the selected symbols.  When the candidates' logits exceed the
+// budget, the head and the quantiser's scores run in slabs of rows, and after
+// the selection the selected rows' logits are computed once more for the coder
+// (bit-identical: a row's logits depend only on that row).
+static int model_step(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int nc, int L, int row0, int rpc,
+                      const StepIO& io, cudaStream_t s) {
+  const int V = (int)m->cfg.vocab, P = precision_for(m->cfg.vocab);
+  const int kcap = kcap_for(pol, rpc);
+  DLMZ_TRY(sb.ensure_cand(nc, rpc, kcap));
+  // the candidates depend only on the state: list them first, so their number reaches
+  // the host while the layers run
+  int32_t* off = sb.cand_off.as<int32_t>();
+  int32_t* cand = sb.cand_tok.as<int32_t>();
+  int32_t* row_map = sb.row_map.as<int32_t>();
+  cand_count_kernel<<<nc, 256, 0, s>>>(io.state, L, V, row0, rpc, sb.cand_count.as<int32_t>());
+  DLMZ_TRY(launch_status());
+  cand_scan_kernel<<<1, 1024, 0, s>>>(sb.cand_count.as<int32_t>(), nc, off, sb.cand_total.as<int64_t>());
+  DLMZ_TRY(launch_status());
+  cand_write_kernel<<<nc, 256, 0, s>>>(io.state, L, V, row0, rpc, off, cand, row_map);
+  DLMZ_TRY(launch_status());
+  DLMZ_CUDA_TRY(cudaMemcpyAsync(sb.host_total, sb.cand_total.p, 8, cudaMemcpyDeviceToHost, s));
+  DLMZ_CUDA_TRY(cudaEventRecord(sb.total_ready, s));
+  DLMZ_TRY(model_layers(m, io.state, nc, L, s));
+  DLMZ_CUDA_TRY(cudaEventSynchronize(sb.total_ready));
+  const int64_t M = *sb.host_total;
+  if (M < 0 || M > (int64_t)nc * rpc) return DLMZ_ECORRUPT;
+  const int64_t sel_rows = (int64_t)nc * kcap;
+  int64_t slab = (int64_t)(logits_budget(m) / ((size_t)V * 4));
+  if (slab < sel_rows) slab = sel_rows;
+  if (slab < 1) slab = 1;
+  const bool slabbed = M > slab;
+  const size_t mrows = (size_t)(M > 0 ? M : 1);
+  DLMZ_TRY(sb.ensure(mrows, 0, nc, kcap));  // scores of every candidate, selection buffers
+  DLMZ_TRY(sb.logits.ensure((slabbed ? (size_t)slab : mrows) * V * 4));
+  float* logits = sb.logits.as<float>();
+  for (int64_t r0 = 0; r0 < M; r0 += slab) {
+    const int n = (int)(M - r0 < slab ? M - r0 : slab);
+    DLMZ_TRY(model_head(m, cand + r0, n, logits, s));
+    DLMZ_TRY(quantize_rows(logits, n, V, P, nullptr, sb.W.as<uint64_t>() + r0, nullptr, sb.Hq.as<int32_t>() + r0,
+                           sb.top.as<int32_t>() + r0, sb.mx.as<float>() + r0, s));
   }
-  return code_step(a, decode, nc, s);
+  DLMZ_TRY(select_step(sb, io.state, nc, L, V, pol, row0, rpc, kcap, row_map, s));
+  if (!slabbed)
+    return code_rows(sb, io, logits, sb.mx.as<float>(), sb.W.as<uint64_t>(), sb.top.as<int32_t>(), row_map, false, nc,
+                     L, V, P, pol, row0, rpc, kcap, s);
+  // the selected rows once more, row c * kcap + j for the j-th selected position of window c
+  DLMZ_TRY(sb.ensure_sel_stats((size_t)sel_rows));
+  int32_t* stok = sb.sel_tok.as<int32_t>();
+  sel_tok_kernel<<<grid_for(sel_rows), 256, 0, s>>>(sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), nc, L, kcap,
+                                                   stok);
+  DLMZ_TRY(launch_status());
+  DLMZ_TRY(model_head(m, stok, (int)sel_rows, logits, s));
+  DLMZ_TRY(quantize_rows(logits, (int)sel_rows, V, P, nullptr, sb.sW.as<uint64_t>(), nullptr, sb.sHq.as<int32_t>(),
+                         sb.stop.as<int32_t>(), sb.smx.as<float>(), s));
+  return code_rows(sb, io, logits, sb.smx.as<float>(), sb.sW.as<uint64_t>(), sb.stop.as<int32_t>(), nullptr, true, nc,
+                   L, V, P, pol, row0, rpc, kcap, s);
 }
 
 static int validate_policy(const dlmz_k_policy* p) {
@@ -352,7 +600,6 @@ static int validate_policy(const dlmz_k_policy* p) {
   return DLMZ_EINVAL;
 }
 
-static int precision_for(uint32_t V) { return V <= 4096 ? 16 : 24; }
 
 static uint64_t cap_bytes_for(uint32_t L, int P) {
   const uint64_t units = ((uint64_t)L * P + 80) / 16 + 4;
@@ -364,8 +611,9 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
                      int32_t* state, CoderState* cst, uint8_t* ebytes, uint64_t cap_bytes, const uint8_t* in_bytes,
                      const uint64_t* in_off, const uint32_t* in_bits, bool decode, const BatchContext& bx,
                      cudaStream_t s) {
-  const int V = (int)m->cfg.vocab, P = precision_for(m->cfg.vocab);
+  const int V = (int)m->cfg.vocab;
   const int ce = bx.ce;
+  const StepIO io{symbols, state, cst, ebytes, cap_bytes, in_bytes, in_off, in_bits, decode, nullptr};
   fill_i32<<<grid_for((int64_t)nc * Lb), 256, 0, s>>>(state, (int64_t)nc * Lb, V);
   DLMZ_TRY(launch_status());
   if (ce > 0) {
@@ -392,12 +640,7 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
       for (int w = 0; w < (bx.pos.empty() ? 1 : nc); ++w) most = std::max(most, Bl - ctx_in(w, b0, b0 + Bl));
       const int steps = (most + (int)pol.k - 1) / (int)pol.k;
       if (steps == 0) continue;
-      DLMZ_TRY(sb.ensure((size_t)nc * Bl, V, nc, kcap_for(pol, Bl)));
-      for (int t = 0; t < steps; ++t) {
-        DLMZ_TRY(model_forward(m, state, nc, Lb, b0, Bl, sb.logits.as<float>(), s));
-        DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, pol, b0, Bl, symbols, state, cst, ebytes,
-                          cap_bytes, in_bytes, in_off, in_bits, decode, nullptr, s));
-      }
+      for (int t = 0; t < steps; ++t) DLMZ_TRY(model_step(m, sb, pol, nc, Lb, b0, Bl, io, s));
     }
   } else if (pol.kind == DLMZ_UNIFORM || pol.kind == DLMZ_PROGRESSIVE) {
     // every window has n = Lb - ce masked positions, so one schedule serves the batch; step k
@@ -426,20 +669,17 @@ static int run_batch(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int 
       }
       dlmz_k_policy sp = pol;
       sp.k = (uint32_t)u;
-      DLMZ_TRY(sb.ensure((size_t)nc * (hi - lo), V, nc, kcap_for(sp, hi - lo)));
-      DLMZ_TRY(model_forward(m, state, nc, Lb, lo, hi - lo, sb.logits.as<float>(), s));
-      DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, sp, lo, hi - lo, symbols, state, cst, ebytes,
-                        cap_bytes, in_bytes, in_off, in_bits, decode, nullptr, s));
+      DLMZ_TRY(model_step(m, sb, sp, nc, Lb, lo, hi - lo, io, s));
       t += u;
     }
   } else {
-    DLMZ_TRY(sb.ensure((size_t)nc * Lb, V, nc, kcap_for(pol, Lb)));
+    DLMZ_TRY(sb.ensure(1, 0, nc, kcap_for(pol, Lb)));
+    StepIO eio = io;
+    eio.committed = sb.committed.as<int32_t>();
     int64_t remaining = (int64_t)nc * (Lb - ce);
     for (int64_t step = 0; remaining > 0; ++step) {
       if (step > (int64_t)Lb) return DLMZ_ECORRUPT;  // every step commits >= 1 per live window
-      DLMZ_TRY(model_forward(m, state, nc, Lb, 0, Lb, sb.logits.as<float>(), s));
-      DLMZ_TRY(run_step(sb, sb.logits.as<float>(), nc, Lb, V, P, pol, 0, Lb, symbols, state, cst, ebytes, cap_bytes,
-                        in_bytes, in_off, in_bits, decode, sb.committed.as<int32_t>(), s));
+      DLMZ_TRY(model_step(m, sb, pol, nc, Lb, 0, Lb, eio, s));
       sum_i32_kernel<<<1, 256, 0, s>>>(sb.committed.as<int32_t>(), nc, sb.sum.as<unsigned long long>());
       DLMZ_TRY(launch_status());
       unsigned long long done = 0;
@@ -471,10 +711,12 @@ static PipeWs& pipe_of(dlmz_model* m) {
 static int default_batch(const dlmz_model* m, uint32_t L, uint32_t n_chunks) {
   size_t freeb = 0, total = 0;
   cudaMemGetInfo(&freeb, &total);
-  size_t budget = freeb / 2;
+  const size_t lb = logits_budget(m);
+  size_t budget = (freeb > lb ? freeb - lb : 0) / 2;
   const size_t cap = (size_t)48 << 30;
   if (budget > cap) budget = cap;
-  const size_t per_chunk = (size_t)L * (model_workspace_per_token(m) + 8 + 4ull * m->cfg.vocab + 64);
+  // forward workspace and per-position step state; the candidate logits have their own budget
+  const size_t per_chunk = (size_t)L * (model_workspace_per_token(m) + 64);
   size_t b = per_chunk ? budget / per_chunk : 1;
   if (b > 1024) b = 1024;
   if (b < 1) b = 1;
@@ -1029,7 +1271,10 @@ int dlmz_attention_bf16(const void* d_qkv, uint32_t ld, uint32_t n_chunks, uint3
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int nc = (int)n_chunks, l = (int)L, nh = (int)n_heads, nkv = (int)n_kv_heads, hd = (int)head_dim;
   if (attention_tc_supported(l, hd)) {
-    static DevBuf vt;  // V^T scratch of the tensor-core kernel
+    static DevBuf vt_dev[kMaxDevices];  // V^T scratch of the tensor-core kernel, one per device
+    const int dev = device_ordinal();
+    if (dev < 0) return DLMZ_ECUDA;
+    DevBuf& vt = vt_dev[dev];
     DLMZ_TRY(vt.ensure((size_t)nc * nkv * attention_vt_rows(hd) * l * 2));
     DLMZ_TRY(attention_vt_from_rows(qkv, (int)ld, (int)(d + (uint64_t)nkv * hd), nc, l, nkv, hd, vt.p, s));
     return attention_bf16_tc(qkv, (int)ld, vt.p, nc, l, nh, nkv, hd, (int)d, out, s);
@@ -1049,7 +1294,10 @@ int dlmz_quantize(const float* d_logits, uint32_t rows, uint32_t V, uint32_t P, 
 int dlmz_select_smallest(const uint64_t* d_keys, uint32_t groups, uint32_t group_size, uint32_t k, int32_t* d_out,
                          void* stream) {
   if (!d_keys || !d_out || k == 0 || k > group_size || group_size > 4096) return DLMZ_EINVAL;
-  static DevBuf counts;
+  static DevBuf counts_dev[kMaxDevices];  // one count per group, one buffer per device
+  const int dev = device_ordinal();
+  if (dev < 0) return DLMZ_ECUDA;
+  DevBuf& counts = counts_dev[dev];
   DLMZ_TRY(counts.ensure((size_t)groups * 4 + 4));
   return select_rows<uint64_t>(nullptr, (int)groups, (int)group_size, -1, 0, (int)group_size, d_keys, 0, (int)k, 0, 0,
                                0, (int)k, counts.as<int32_t>(), d_out, reinterpret_cast<cudaStream_t>(stream));
@@ -1124,6 +1372,31 @@ static int step_common(dlmz_coder* c, const dlmz_k_policy* pol, const float* d_l
   return run_step(c->sb, d_logits, c->nc, c->L, c->V, c->P, *pol, (int)row0, (int)rpc, d_symbols, d_state,
                   c->cst.as<CoderState>(), c->bytes.as<uint8_t>(), c->cap, c->in_bytes, c->in_off, c->in_bits, decode,
                   d_committed, reinterpret_cast<cudaStream_t>(stream));
+}
+
+static int model_step_common(dlmz_model* m, dlmz_coder* c, const dlmz_k_policy* pol, uint32_t row0, uint32_t rpc,
+                             const int32_t* d_symbols, int32_t* d_state, int32_t* d_committed, bool decode,
+                             void* stream) {
+  if (!m || !c || !d_state || validate_policy(pol) != DLMZ_OK) return DLMZ_EINVAL;
+  if ((int)pol->coder != c->coder || pol->context != DLMZ_CONTEXT_NONE) return DLMZ_EINVAL;
+  if ((int)m->cfg.vocab != c->V || precision_for(m->cfg.vocab) != c->P) return DLMZ_EINVAL;
+  if (rpc == 0 || row0 + rpc > (uint32_t)c->L) return DLMZ_EINVAL;
+  if (!decode && !d_symbols) return DLMZ_EINVAL;
+  if (decode && !c->in_bytes) return DLMZ_EINVAL;
+  const StepIO io{d_symbols, d_state, c->cst.as<CoderState>(), c->bytes.as<uint8_t>(), c->cap, c->in_bytes,
+                  c->in_off, c->in_bits, decode, d_committed};
+  return model_step(m, c->sb, *pol, c->nc, c->L, (int)row0, (int)rpc, io, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int dlmz_model_encode_step(dlmz_model* m, dlmz_coder* c, const dlmz_k_policy* policy, uint32_t row0,
+                           uint32_t rows_per_chunk, const int32_t* d_symbols, int32_t* d_state, int32_t* d_committed,
+                           void* stream) {
+  return model_step_common(m, c, policy, row0, rows_per_chunk, d_symbols, d_state, d_committed, false, stream);
+}
+
+int dlmz_model_decode_step(dlmz_model* m, dlmz_coder* c, const dlmz_k_policy* policy, uint32_t row0,
+                           uint32_t rows_per_chunk, int32_t* d_state, int32_t* d_committed, void* stream) {
+  return model_step_common(m, c, policy, row0, rows_per_chunk, nullptr, d_state, d_committed, true, stream);
 }
 
 int dlmz_encode_step(dlmz_coder* c, const dlmz_k_policy* policy, const float* d_logits, uint32_t row0,

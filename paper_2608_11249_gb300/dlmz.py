@@ -61,6 +61,7 @@ _sig("dlmz_model_create", c_int, POINTER(ModelConfig), POINTER(c_void_p))
 _sig("dlmz_model_destroy", None, _P)
 _sig("dlmz_model_fingerprint", c_uint64, _P)
 _sig("dlmz_model_get_config", c_int, _P, POINTER(ModelConfig))
+_sig("dlmz_model_set_logits_budget", c_int, _P, c_size_t)
 _sig("dlmz_compress", c_int, _P, _P, c_size_t, c_uint32, POINTER(KPolicy), POINTER(POINTER(c_uint8)), POINTER(c_size_t))
 _sig("dlmz_compress_ex", c_int, _P, _P, c_size_t, c_uint32, POINTER(KPolicy), c_uint32, POINTER(POINTER(c_uint8)),
      POINTER(c_size_t))
@@ -85,8 +86,11 @@ _sig("dlmz_coder_load_decoder", c_int, _P, _P, _P, _P, _P)
 _sig("dlmz_encode_step", c_int, _P, POINTER(KPolicy), _P, c_uint32, c_uint32, _P, _P, _P, _P)
 _sig("dlmz_decode_step", c_int, _P, POINTER(KPolicy), _P, c_uint32, c_uint32, _P, _P, _P)
 _sig("dlmz_coder_finish", c_int, _P, _P, _P, _P, _P)
+_sig("dlmz_model_encode_step", c_int, _P, _P, POINTER(KPolicy), c_uint32, c_uint32, _P, _P, _P, _P)
+_sig("dlmz_model_decode_step", c_int, _P, _P, POINTER(KPolicy), c_uint32, c_uint32, _P, _P, _P)
 _sig("dlmz_coder_capacity_units", c_uint32, _P)
 _sig("dlmz_check", c_int, _P)
+_sig("dlmz_selftest_wait_timeout", c_int, c_uint32, _P)
 _sig("dlmz_profile_begin", c_int)
 _sig("dlmz_profile_end", c_int, POINTER(Profile))
 
@@ -130,6 +134,10 @@ class Model:
     def fingerprint(self):
         return lib.dlmz_model_fingerprint(self.h)
 
+    def set_logits_budget(self, nbytes):
+        """Bytes of candidate logits one step holds at once (0: the library default)."""
+        _ok(lib.dlmz_model_set_logits_budget(self.h, nbytes), "dlmz_model_set_logits_budget")
+
     def compress(self, data, chunk_len, pol, batch_chunks=0):
         buf = bytes(data)
         out = POINTER(c_uint8)()
@@ -170,6 +178,15 @@ class Model:
         _ok(lib.dlmz_forward_logits(self.h, d_state, n_chunks, L, row0, rows_per_chunk, d_logits, stream),
             "dlmz_forward_logits")
 
+    def encode_step(self, coder, pol, row0, rpc, d_symbols, d_state, d_committed=None, stream=0):
+        """One denoising step with this model's distributions, coding into ``coder`` (a Coder)."""
+        _ok(lib.dlmz_model_encode_step(self.h, coder.h, byref(pol), row0, rpc, d_symbols, d_state, d_committed,
+                                       stream), "dlmz_model_encode_step")
+
+    def decode_step(self, coder, pol, row0, rpc, d_state, d_committed=None, stream=0):
+        _ok(lib.dlmz_model_decode_step(self.h, coder.h, byref(pol), row0, rpc, d_state, d_committed, stream),
+            "dlmz_model_decode_step")
+
     def context_scores(self, d_symbols, n_chunks, L, d_scores, stream=0):
         _ok(lib.dlmz_context_scores(self.h, d_symbols, n_chunks, L, d_scores, stream), "dlmz_context_scores")
 
@@ -207,6 +224,11 @@ def profile_end(prof):
 
 def check(stream=0):
     _ok(lib.dlmz_check(stream), "dlmz_check")
+
+
+def selftest_wait_timeout(limit_us, stream=0):
+    """Return code of dlmz_selftest_wait_timeout (DLMZ_ETIMEOUT when the bounded wait gave up)."""
+    return lib.dlmz_selftest_wait_timeout(limit_us, stream)
 
 
 class Coder:

@@ -103,6 +103,10 @@ CASES = [
     (256, 80, 2, S.Policy(kind=S.ENTROPY, tau_bits=2.0, k_min=2, k_max=5)),
     (5000, 40, 2, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=64)),
     (5000, 33, 2, S.Policy(kind=S.TOPK_CONF, k=16, block=0)),
+    # the large vocabularies (P = 24): 8B-shaped top-16 over the whole window, 7B-shaped entropy
+    # threshold 0.5 bits with m = 1 and cap 64
+    (126464, 40, 2, S.Policy(kind=S.TOPK_CONF, k=16, block=0)),
+    (152064, 24, 2, S.Policy(kind=S.ENTROPY, tau_bits=0.5, k_min=1, k_max=64)),
 ]
 
 

@@ -234,3 +234,90 @@ def test_corrupt_containers_are_rejected(dev):
         else:
             assert out == data
     d.check()
+
+
+SLAB_CASES = [
+    # model, data kind, n, chunk_len, policy (kind, k, block, tau, k_min, k_max), context, batch_chunks
+    ((1, 64, 4, 2, 128, 5000, "f32"), "tokens", 700, 100, (S.TOPK_CONF, 8, 0, 0.0, 1, 0), (OX.NONE, 0, 0), 3),
+    ((2, 256, 4, 4, 256, 5000, "bf16"), "tokens", 500, 128, (S.ENTROPY, 0, 0, 0.5, 1, 8), (OX.RANDOM, 9, 2), 2),
+    ((1, 64, 4, 2, 128, 5000, "f32"), "tokens", 400, 100, (S.UNIFORM, 6, 0, 0.0, 1, 0), (OX.NONE, 0, 0), 0),
+    ((1, 32, 2, 2, 64, 256, "f32"), "bytes", 900, 300, (S.TOPK_CONF, 4, 64, 0.0, 1, 0), (OX.RANDOM, 20, 7), 2),
+]
+
+
+@pytest.mark.parametrize("ci", range(len(SLAB_CASES)))
+def test_candidate_slabs_give_identical_files(dev, ci):
+    """The LM head and quantiser run on the candidate rows; with a logits budget of a few
+    rows they run in slabs and the selected rows are recomputed for the coder.  The file
+    must not depend on the budget, and either model decodes it."""
+    d = dlmz()
+    spec, kind, n, L, (k0, k, blk, tau, kmin, kmax), ctx, bc = SLAB_CASES[ci]
+    data = _data(kind, n, spec[5])
+    pol = d.policy(k0, k, blk, tau, kmin, kmax, 65536, ctx[0], ctx[1], ctx[2])
+    a = _model(d, spec, 120 + ci)
+    blob = a.compress(data, L, pol, bc)
+    b = _model(d, spec, 120 + ci)
+    b.set_logits_budget(7 * spec[5] * 4)  # 7 rows of logits: many slabs per step
+    assert b.compress(data, L, pol, bc) == blob
+    assert b.decompress(blob) == data
+    assert a.decompress(blob) == data
+
+
+@pytest.mark.parametrize("spec,V,L,nc,pol_args", [
+    ((2, 256, 4, 4, 256, 256, "bf16"), 256, 128, 4, (S.TOPK_CONF, 8, 64, 0.0, 1, 0)),
+    ((1, 64, 4, 2, 128, 5000, "f32"), 5000, 96, 3, (S.ENTROPY, 0, 0, 0.5, 1, 8)),
+])
+def test_model_step_api_matches_whole_file(dev, spec, V, L, nc, pol_args):
+    """dlmz_model_encode_step / dlmz_model_decode_step over one batch: the streams equal those of
+    the dlmz_compress file of the same windows, and decoding recovers the symbols."""
+    import torch
+    from oracle import quantizer as Q
+    d = dlmz()
+    m = _model(d, spec, 150)
+    kind = "bytes" if V == 256 else "tokens"
+    data = _data(kind, nc * L, V)
+    sym = np.frombuffer(data, dtype=np.uint8 if kind == "bytes" else "<u4").astype(np.int32).reshape(nc, L)
+    k0, k, blk, tau, kmin, kmax = pol_args
+    pol = d.policy(k0, k, blk, tau, kmin, kmax)
+    blob = m.compress(data, L, pol, nc)
+    _, want = OC.read(blob)
+    P = Q.precision_for_vocab(V)
+    coder = d.Coder(nc, L, V, P)
+    coder.reset_encoder()
+    d_sym = to_dev(sym)
+    state = to_dev(np.full((nc, L), V, dtype=np.int32))
+    committed = torch.zeros(nc, dtype=torch.int32, device="cuda")
+    B = blk or L
+
+    def run(step_fn):
+        if k0 == S.TOPK_CONF:
+            for b0 in range(0, L, B):
+                for _ in range(-(-min(B, L - b0) // k)):
+                    step_fn(b0, min(B, L - b0))
+        else:
+            for _ in range(L + 1):
+                if int((state == V).sum().item()) == 0:
+                    break
+                step_fn(0, L)
+
+    run(lambda r0, rpc: m.encode_step(coder, pol, r0, rpc, ptr(d_sym), ptr(state), ptr(committed)))
+    d.check()
+    assert np.array_equal(state.cpu().numpy(), sym)
+    bits = torch.empty(nc, dtype=torch.int32, device="cuda")
+    cap = coder.capacity_units * 2
+    raw = torch.zeros(nc * cap, dtype=torch.uint8, device="cuda")
+    coder.finish(ptr(bits), ptr(raw))
+    d.check()
+    bits_h = bits.cpu().numpy().astype(np.int64)
+    raw_h = raw.cpu().numpy()
+    got = [(int(bits_h[c]), bytes(raw_h[c * cap:c * cap + (bits_h[c] + 7) // 8])) for c in range(nc)]
+    assert got == [(int(b), bytes(s)) for b, s in want]
+    packed = np.frombuffer(b"".join(s for _, s in got) + b"\0" * 8, dtype=np.uint8)
+    offs = np.concatenate([[0], np.cumsum([(b + 7) // 8 for b in bits_h])[:-1]]).astype(np.int64)
+    dec = d.Coder(nc, L, V, P)
+    d_packed, d_offs, d_bits = to_dev(packed), to_dev(offs), to_dev(bits_h.astype(np.int32))
+    dec.load_decoder(ptr(d_packed), ptr(d_offs), ptr(d_bits))
+    state.copy_(to_dev(np.full((nc, L), V, dtype=np.int32)))
+    run(lambda r0, rpc: m.decode_step(dec, pol, r0, rpc, ptr(state), ptr(committed)))
+    d.check()
+    assert np.array_equal(state.cpu().numpy(), sym)
