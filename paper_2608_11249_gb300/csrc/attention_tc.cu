@@ -1,12 +1,13 @@
 // Bidirectional attention on the 5th-generation tensor cores (Definition 3:
 // every position attends to every position of its window, no mask).
 //
-// Persistent CTAs (two per SM) walk work items (128 queries, head, window); 6 warps:
+// Persistent CTAs (two per SM at head dim 64, one at 128) walk work items
+// (128 queries, head, window); 6 warps:
 //   warp 0      TMA: Q once per item (2-stage ring, so the next item's Q is
 //               in flight during this item); per key tile of 128: K and V^T
 //               (keys contiguous, written so by the QKV epilogue), each
 //               through a 2-stage ring, K requested one tile ahead of V.
-//   warp 1      allocates 256 TMEM columns (S: 128, P: 64, O: head_dim) and
+//   warp 1      allocates TMEM (S: 128 columns, P: 64, O: head_dim) and
 //               issues S_j = Q K_j^T (A and B in shared memory) and
 //               O += P_j V_j (A = P_j in TMEM) with tcgen05.mma from one thread.
 //   warps 2-5   softmax, one thread per query row (its TMEM lane): the row of
@@ -17,6 +18,8 @@
 //               by more than 8 (log2 units), so P <= 2^8; finally O / l -> bf16,
 //               deferred into the next item's first tile so the next S is
 //               taken (and the MMA warp goes on) before the last P V is waited for.
+// At head dim 128 the item's output is drained from TMEM in 32-column chunks
+// after P has been handed over (the 128 S registers and O never coexist).
 // GQA: query head h reads KV head h / (n_heads / n_kv_heads).  Requires the
 // window length to be a multiple of 128.  All waits are bounded.
 #include "kernels.cuh"
@@ -27,15 +30,22 @@ namespace fat {
 
 constexpr int BQ = 128, BK = 128;
 constexpr int THREADS = 192;
-constexpr int TMEM_COLS = 256;
 constexpr float RESCALE_THRESHOLD = 8.0f;
+
+// TMEM columns: S [0, 128), P [128, 192) (f16 pairs), O from O_COL (a multiple of head_dim).
+template <int HD>
+struct Tmem {
+  static constexpr int O_COL = HD == 64 ? 192 : 256;
+  static constexpr int COLS = HD == 64 ? 256 : 512;
+  static constexpr int CTAS_PER_SM = HD == 64 ? 2 : 1;
+};
 
 template <int HD>
 struct Smem {
-  static_assert(HD == 64, "one 128-byte swizzle row per Q / K row");
-  static constexpr int QT = BQ * HD * 2;             // one query tile [128 x 64] bf16
+  static_assert(HD == 64 || HD == 128, "Q / K rows of one or two 128-byte swizzle blocks");
+  static constexpr int QT = BQ * HD * 2;             // one query tile: HD / 64 blocks of [128 x 64] bf16
   static constexpr int Q = 0;                        // 2 query tiles
-  static constexpr int KT = BK * HD * 2;             // one key tile [128 x 64] bf16
+  static constexpr int KT = BK * HD * 2;             // one key tile: HD / 64 blocks of [128 x 64] bf16
   static constexpr int K = Q + 2 * QT;               // 2 key tiles
   static constexpr int VTT = HD * BK * 2;            // one V^T tile: 2 blocks of [HD x 64] f16 (keys 0-63, 64-127)
   static constexpr int VT = K + 2 * KT;              // 2 V^T tiles
@@ -76,13 +86,13 @@ __device__ __forceinline__ void fma2(float& y0, float& y1, float x0, float x1, f
   asm("mov.b64 {%0, %1}, %2;" : "=f"(y0), "=f"(y1) : "l"(y));
 }
 
-// One query row of an item's output: O / l -> bf16, HD values from 16-byte stores.
-template <int HD>
-__device__ __forceinline__ void write_row(bf16* __restrict__ dst, const uint32_t (&o)[HD], float l) {
+// N values of one query row of an item's output: O / l -> bf16, from 16-byte stores.
+template <int N>
+__device__ __forceinline__ void write_row(bf16* __restrict__ dst, const uint32_t* o, float l) {
   const float inv = 1.0f / l;
   uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-  for (int t = 0; t < HD / 8; ++t) {
+  for (int t = 0; t < N / 8; ++t) {
     uint32_t u[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -94,8 +104,20 @@ __device__ __forceinline__ void write_row(bf16* __restrict__ dst, const uint32_t
   }
 }
 
+// This thread's output row of the item (TMEM lane) drained from O in chunks of 32
+// columns (head dim 128: the S registers are dead here, so the chunks stay small).
 template <int HD>
-__global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 registers per thread
+__device__ __forceinline__ void drain_row(uint32_t tO_lane, bf16* __restrict__ dst, float l) {
+#pragma unroll 1
+  for (int c = 0; c < HD / 32; ++c) {
+    float v[32];
+    t5::tmem_ld32(tO_lane + c * 32, v);
+    write_row<32>(dst + c * 32, reinterpret_cast<const uint32_t*>(v), l);
+  }
+}
+
+template <int HD>
+__global__ void __launch_bounds__(THREADS, Tmem<HD>::CTAS_PER_SM)  // head dim 64: two CTAs per SM, <= 168 registers
     fa_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt, int n_chunks,
                  int L, int nh, int nkv, int d, bf16* __restrict__ out, float scale_log2, int* err) {
   using S = Smem<HD>;
@@ -144,12 +166,12 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
     mbar_init(o_free, 4 * 32);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) t5::tmem_alloc(smem_u32(&tmem_slot), TMEM_COLS);
+  if (warp == 1) t5::tmem_alloc(smem_u32(&tmem_slot), Tmem<HD>::COLS);
   t5::fence_before();
   __syncthreads();
   t5::fence_after();
   const uint32_t tmem = tmem_slot;
-  const uint32_t tS = tmem, tP = tmem + BK, tO = tmem + BK + BK / 2;
+  const uint32_t tS = tmem, tP = tmem + BK, tO = tmem + Tmem<HD>::O_COL;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -315,14 +337,24 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
         if (!__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (J - 1) & 1, &abort_flag, err))) break;
         t5::fence_after();
         if (j == 0) {
-          uint32_t o[HD];
-          t5::tmem_ld64(tO + lane_off, o);
-          t5::tmem_st64(tP + lane_off, sr);
-          t5::fence_before();
-          mbar_arrive(o_free);  // O is in registers: this item's first PV may overwrite it
-          mbar_arrive(p_ready);
+          if constexpr (HD == 64) {
+            uint32_t o[HD];
+            t5::tmem_ld64(tO + lane_off, o);
+            t5::tmem_st64(tP + lane_off, sr);
+            t5::fence_before();
+            mbar_arrive(o_free);  // O is in registers: this item's first PV may overwrite it
+            mbar_arrive(p_ready);
+            write_row<HD>(row_of(J / nt - 1), o, l_pend);  // the previous item's output, off the MMA warp's path
+          } else {
+            // P first (the MMA warp still waits for o_free before this item's first PV), then O in chunks
+            t5::tmem_st64(tP + lane_off, sr);
+            t5::fence_before();
+            mbar_arrive(p_ready);
+            drain_row<HD>(tO + lane_off, row_of(J / nt - 1), l_pend);
+            t5::fence_before();
+            mbar_arrive(o_free);
+          }
           p_stored = true;
-          write_row<HD>(row_of(J / nt - 1), o, l_pend);  // the previous item's output, off the MMA warp's path
           pend = false;
         } else if (__any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 where not needed)
 #pragma unroll 1
@@ -348,10 +380,8 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
     if (pend && !abort_flag) {  // the last item's epilogue
       if (__all_sync(0xffffffffu, mbar_wait_bounded(o_done, (total - 1) & 1, &abort_flag, err))) {
         t5::fence_after();
-        uint32_t o[HD];
-        t5::tmem_ld64(tO + lane_off, o);
+        drain_row<HD>(tO + lane_off, row_of((total - 1) / nt), l_pend);
         t5::fence_before();
-        write_row<HD>(row_of((total - 1) / nt), o, l_pend);
       }
     }
   }
@@ -359,13 +389,13 @@ __global__ void __launch_bounds__(THREADS, 2)  // two CTAs per SM: at most 168 r
   __syncthreads();
   if (warp == 1) {
     t5::fence_after();
-    t5::tmem_dealloc(tmem, TMEM_COLS);
+    t5::tmem_dealloc(tmem, Tmem<HD>::COLS);
   }
 }
 
 }  // namespace fat
 
-bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 && hd == 64; }
+bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 && (hd == 64 || hd == 128); }
 
 int attention_vt_rows(int hd) { return hd; }
 
@@ -410,19 +440,29 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
   DLMZ_TRY(t5::make_map_bf16(&mqk, qkv, (uint64_t)n_chunks * L, ld, ld, 128, 64));
   DLMZ_TRY(t5::make_map_f16(&mvt, vt, (uint64_t)n_chunks * nkv * hd, L, L, hd, 64));
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
-  constexpr int SM = fat::Smem<64>::TOTAL;
-  static bool attr = false;
-  if (!attr) {
-    DLMZ_CUDA_TRY(cudaFuncSetAttribute(fat::fa_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM));
-    attr = true;
-  }
-  // persistent: two CTAs per SM (shared memory and 256 TMEM columns each) walk the work items
+  // persistent: two CTAs (head dim 64) or one (128) per SM walk the work items
   const int64_t items = (int64_t)n_chunks * nh * (L / fat::BQ);
   if (items > 0x7fffffff) return DLMZ_EINVAL;
-  const int grid = items < 2 * num_sms() ? (int)items : 2 * num_sms();
   ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
-  fat::fa_tc_kernel<64><<<grid, fat::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
-                                                      device_error_word());
+  if (hd == 64) {
+    constexpr int SM = fat::Smem<64>::TOTAL;
+    static PerDeviceOnce attr;
+    DLMZ_TRY(attr.run(
+        [] { return cudaFuncSetAttribute(fat::fa_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
+    const int cap = fat::Tmem<64>::CTAS_PER_SM * num_sms();
+    const int grid = items < cap ? (int)items : cap;
+    fat::fa_tc_kernel<64><<<grid, fat::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
+                                                        device_error_word());
+  } else {
+    constexpr int SM = fat::Smem<128>::TOTAL;
+    static PerDeviceOnce attr;
+    DLMZ_TRY(attr.run(
+        [] { return cudaFuncSetAttribute(fat::fa_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
+    const int cap = fat::Tmem<128>::CTAS_PER_SM * num_sms();
+    const int grid = items < cap ? (int)items : cap;
+    fat::fa_tc_kernel<128><<<grid, fat::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
+                                                         device_error_word());
+  }
   return launch_status();
 }
 

@@ -26,6 +26,10 @@ CASES = [
     (1024, 2, 4, 4, 64, "drift"),    # tcgen05: 8 key tiles per item, running max raised across tiles
     (512, 3, 8, 1, 64, "drift"),     # tcgen05: 8:1 GQA
     (256, 2, 4, 2, 64, "flat"),      # tcgen05: small scores
+    (1024, 2, 32, 32, 128, "drift"), # tcgen05 head_dim 128: the 8B-shaped MHA (32 heads) at windows of 1024
+    (2048, 1, 28, 4, 128, "drift"),  # tcgen05 head_dim 128: the 7B-shaped 7:1 GQA at windows of 2048
+    (256, 3, 8, 2, 128, "flat"),     # tcgen05 head_dim 128: small scores, 4:1 GQA
+    (128, 160, 2, 1, 128, "drift"),  # tcgen05 head_dim 128: 320 one-tile items, ~2 per persistent CTA
     (96, 2, 4, 2, 64, "drift"),      # CUDA-core mma kernel (L % 128 != 0)
     (64, 2, 2, 1, 128, "drift"),     # CUDA-core mma kernel, head_dim 128
     (40, 3, 4, 2, 32, "drift"),      # CUDA-core scalar kernel, head_dim 32
