@@ -20,7 +20,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libdlmz.so")
 SOURCES = ["model.cu", "gemm_tc.cu", "layers.cu", "attention.cu", "quantize.cu", "coder.cu", "pipeline.cu",
            "profile.cu", "noalloc.cu",
-           "attention_tc.cu", "context.cu"]
+           "attention_tc.cu", "context.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden", "-I" + os.path.join(ROOT, "include")]
 
