@@ -4,7 +4,8 @@
   launch configuration: sampled windows' logits vs the oracle, and a full
   512 KiB batch round trip through the device-resident API;
 * layers of the 8B-shaped (d=4096, 32 heads, FFN 12288) and 7B GQA-shaped
-  (d=3584, 28/4 heads, FFN 18944) models, one layer deep, sampled rows;
+  (d=3584, 28/4 heads, FFN 18944) models, one layer deep, sampled rows, within
+  twice the divergence of the oracle's own float32-contraction evaluation;
 * the isolated quantise+select workload (65536 x 126464 logits) at full size,
   sampled rows and groups bit-exact;
 * the tiny float32 byte model, full round trip, compressed size vs the oracle
@@ -23,16 +24,10 @@ from tests.gpu_helpers import dlmz, ptr, to_dev
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
 
-def _tolerance(dm):
-    """2e-2 at the byte model's width; bf16 storage noise grows with the logit scale sqrt(d).
-
-    Measured: the oracle with bf16 vs float32 activation storage (same bf16
-    weights) differs by max 0.038 / rms 0.0073 at d = 4096 (one layer).
-    """
-    return 2e-2 * max(1.0, np.sqrt(dm / 512.0))
-
-
-def _forward_sampled(d, spec, nc, L, row0, rpc, sample, seed, tol):
+def _forward_sampled(d, spec, nc, L, row0, rpc, sample, seed, tol=None):
+    """GPU logits of sampled windows vs the oracle.  ``tol``: a fixed max-abs bound (rms a
+    quarter of it); None: at most twice the divergence of the oracle's own float32-contraction
+    evaluation on the same rows (the wide layers, where bf16 rounding flips spread)."""
     import torch
     nl, dm, nh, nkv, F, V, dt = spec
     m = d.Model(nl, dm, nh, nkv, F, V, d.BF16 if dt == "bf16" else d.FP32, seed=seed)
@@ -45,11 +40,17 @@ def _forward_sampled(d, spec, nc, L, row0, rpc, sample, seed, tol):
     got = logits.view(nc, rpc, V)
     w = OM.Weights(OM.ModelConfig(*spec, seed=seed))
     for c in sample:
-        ref = OM.forward(w, state[c], rows=np.arange(row0, row0 + rpc))
+        rows = np.arange(row0, row0 + rpc)
+        ref = OM.forward(w, state[c], rows=rows)
         diff = got[c].cpu().numpy() - ref
         err = float(np.max(np.abs(diff)))
         rms = float(np.sqrt(np.mean(diff ** 2)))
-        assert err <= tol and rms <= tol / 4, (c, err, rms)
+        if tol is not None:
+            assert err <= tol and rms <= tol / 4, (c, err, rms)
+        else:
+            alt = OM.forward(w, state[c], rows=rows, matmul_dtype=np.float32) - ref
+            nerr, nrms = float(np.max(np.abs(alt))), float(np.sqrt(np.mean(alt ** 2)))
+            assert err <= 2 * nerr and rms <= 2 * nrms, (c, err, rms, nerr, nrms)
     m.close()
 
 
@@ -75,7 +76,7 @@ def test_byte_workload_full_batch(dev):
                                   (1, 3584, 28, 4, 18944, 1024, "bf16")])   # 7B GQA-shaped layer, 7:1
 def test_large_model_layers(dev, spec):
     d = dlmz()
-    _forward_sampled(d, spec, 3, 256, 0, 256, [0, 2], 5, _tolerance(spec[1]))
+    _forward_sampled(d, spec, 3, 256, 0, 256, [0, 2], 5)
 
 
 def test_isolated_quantize_select_full_size(dev):
