@@ -23,10 +23,18 @@ Weights are stored [out x in] (row = one output feature).  Arithmetic is
 float64; a tensor that the model stores between operations is rounded to
 its storage dtype at that point:
 
-* bf16 models: weights, E, the normed activations h, q/k/v after RoPE, the
-  attention output and the SwiGLU product are bfloat16; the residual stream
-  x and the logits are float32.
+* bf16 models: weights, E, the projection inputs, q/k/v after RoPE, the
+  attention output, the SwiGLU product and the LM-head input are bfloat16;
+  the residual stream x and the logits are float32.
 * f32 models: every stored tensor is float32.
+
+The RMSNorm in front of the QKV and gate/up projections is applied as a row
+scale of the projection's result (mathematically the same block): the
+projection reads x g rounded to the storage dtype and its float result is
+multiplied by 1 / sqrt(mean(x^2) + eps) of the float32 residual x, before
+RoPE and SiLU.  The final RMSNorm in front of the LM head is applied to x
+directly and its result stored.  (The paper fixes no precision; these
+storage points are the reading both implementations follow.)
 
 Parity: pinned by closed forms (uniform attention when Wq = Wk = 0,
 logits = head(norm(E[s])) when Wo = Wd = 0, permutation equivariance with
@@ -145,6 +153,11 @@ class Weights:
         return self.t[TID_HEAD]
 
 
+def rms_scale(x, eps):
+    """1 / sqrt(mean(x^2) + eps), per row (a column vector)."""
+    return 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps)
+
+
 def rmsnorm(x, g, eps):
     """x / sqrt(mean(x^2) + eps) * g, per row."""
     ms = np.mean(x * x, axis=-1, keepdims=True)
@@ -224,17 +237,21 @@ def hidden(wts, state, probs=None, matmul_dtype=np.float64):
     mm = lambda a, b: _matmul(a, b, matmul_dtype)
     x = r32(wts.embed[np.asarray(state)])
     for l in range(cfg.n_layers):
-        h = rnd(rmsnorm(x, wts.g_attn[l], cfg.norm_eps))
-        q = mm(h, wts.layer(l, WQ).T)
-        k = mm(h, wts.layer(l, WK).T)
-        v = mm(h, wts.layer(l, WV).T)
+        # pre-norm as a row scale of the projections: (x g / rms(x)) W^T = (x g) W^T / rms(x),
+        # with x g stored in the model's dtype and the scale applied to the float result
+        rs = rms_scale(x, cfg.norm_eps)
+        h = rnd(x * wts.g_attn[l])
+        q = rs * mm(h, wts.layer(l, WQ).T)
+        k = rs * mm(h, wts.layer(l, WK).T)
+        v = rs * mm(h, wts.layer(l, WV).T)
         q = rnd(rope(q, cfg.n_heads, hd, cfg.rope_theta))
         k = rnd(rope(k, cfg.n_kv_heads, hd, cfg.rope_theta))
         v = rnd(v)
         o = rnd(attention(q, k, v, cfg.n_heads, cfg.n_kv_heads, hd, probs, matmul_dtype))
         x = r32(x + mm(o, wts.layer(l, WO).T))
-        h = rnd(rmsnorm(x, wts.g_ffn[l], cfg.norm_eps))
-        a = rnd(silu(mm(h, wts.layer(l, WGATE).T)) * mm(h, wts.layer(l, WUP).T))
+        rs = rms_scale(x, cfg.norm_eps)
+        h = rnd(x * wts.g_ffn[l])
+        a = rnd(silu(rs * mm(h, wts.layer(l, WGATE).T)) * (rs * mm(h, wts.layer(l, WUP).T)))
         x = r32(x + mm(a, wts.layer(l, WDOWN).T))
     return rnd(rmsnorm(x, wts.g_final, cfg.norm_eps))
 

@@ -69,11 +69,13 @@ __device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&p);
 }
 
-__device__ __forceinline__ float tanh_approx(float x) {
-  float y;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
+// The value a bfloat16 store of x would hold (V is kept in f16 for the
+// attention kernel, after the same bf16 rounding as every stored tensor).
+__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+// silu(g) = g / (1 + e^-g): ex2-based exponential and reciprocal, a few ulp
+// of float32 (the product is then stored in bf16).
+__device__ __forceinline__ float silu_f32(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
 // Global data an epilogue chunk needs besides the accumulator (residual
 // values or RoPE (cos, sin) pairs), loaded one chunk ahead to hide latency.
@@ -161,10 +163,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
       float u[32];
       tmem_ld32(tbase + BN / 2 + c * 32, u);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float hg = 0.5f * rs * v[i];
-        v[i] = fmaf(hg, tanh_approx(hg), hg) * (rs * u[i]);  // silu(g) = g/2 (1 + tanh(g/2))
-      }
+      for (int i = 0; i < 32; ++i) v[i] = silu_f32(rs * v[i]) * (rs * u[i]);
     } else if constexpr (EPI == EPI_ROPE_BF16) {
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] *= rs;
@@ -221,8 +220,11 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
         const float4 a = *reinterpret_cast<const float4*>(stg + (j * 32 + ((p0 + 4 * (j & 7)) & 31)) * 4);
         const float4 b = *reinterpret_cast<const float4*>(stg + (j * 32 + ((p0 + 4 + 4 * (j & 7)) & 31)) * 4);
         const float w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        float r[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) r[e] = bf16_round(w[e]);
         *reinterpret_cast<uint4*>(vb + (size_t)j * ep.L + p0) =
-            make_uint4(pack2_f16(w[0], w[1]), pack2_f16(w[2], w[3]), pack2_f16(w[4], w[5]), pack2_f16(w[6], w[7]));
+            make_uint4(pack2_f16(r[0], r[1]), pack2_f16(r[2], r[3]), pack2_f16(r[4], r[5]), pack2_f16(r[6], r[7]));
       }
     } else {
 #pragma unroll

@@ -170,7 +170,7 @@ def test_bf16_model_rounds_storage():
     assert np.max(np.abs(a - b)) < 2e-2  # bf16 storage vs float32 storage of the same draws
 
 
-def _torch_block_forward(cfg, t, state):
+def _torch_block_forward(cfg, t, state, bf16=False):
     """Definition 3's LLaDA-style block restated with PyTorch float64 CPU library calls.
 
     Written from the block definition (pre-norm RMSNorm, rotary embedding as a
@@ -178,12 +178,18 @@ def _torch_block_forward(cfg, t, state):
     scaled_dot_product_attention without a mask, SwiGLU = silu(gate) * up,
     residual adds, final RMSNorm, untied head), not from oracle/model.py.  A
     tensor the model stores is rounded to float32 (torch's own conversion).
+    ``bf16``: the bf16 storage points instead -- the residual stays float32,
+    the projections read bfloat16(x) and their results are scaled by the
+    RMSNorm factor of x (the norm as a row scale), q/k after RoPE, v, the
+    attention output, the SwiGLU product and the final normed rows are
+    bfloat16 (torch's conversion through float32).
     """
     import torch
     import torch.nn.functional as F
 
     f64 = torch.float64
     st = lambda a: a.to(torch.float32).to(f64)
+    sb = (lambda a: a.to(torch.float32).to(torch.bfloat16).to(f64)) if bf16 else st
     T = {k: torch.from_numpy(np.asarray(v, dtype=np.float64)) for k, v in t.items()}
     hd, L = cfg.d // cfg.n_heads, len(state)
     idx = torch.as_tensor(np.asarray(state), dtype=torch.long)
@@ -202,18 +208,21 @@ def _torch_block_forward(cfg, t, state):
 
     x = st(T[M.TID_EMBED][idx])
     g = cfg.n_heads // cfg.n_kv_heads
+    def proj(x, which):  # the normed projection: norm(x) W^T, or with bf16 storage bf16(x) W^T * scale
+        if not bf16:
+            return F.linear(st(norm(x)), which)
+        return F.linear(sb(x), which) * torch.rsqrt((x * x).mean(-1, keepdim=True) + cfg.norm_eps)
+
     for l in range(cfg.n_layers):
         P = lambda which: T[M.layer_tid(l, which)]
-        h = st(norm(x))
-        q = st(rope(F.linear(h, P(M.WQ)), cfg.n_heads)).view(L, cfg.n_heads, hd).transpose(0, 1)
-        k = st(rope(F.linear(h, P(M.WK)), cfg.n_kv_heads)).view(L, cfg.n_kv_heads, hd).transpose(0, 1)
-        v = st(F.linear(h, P(M.WV))).view(L, cfg.n_kv_heads, hd).transpose(0, 1)
+        q = sb(rope(proj(x, P(M.WQ)), cfg.n_heads)).view(L, cfg.n_heads, hd).transpose(0, 1)
+        k = sb(rope(proj(x, P(M.WK)), cfg.n_kv_heads)).view(L, cfg.n_kv_heads, hd).transpose(0, 1)
+        v = sb(proj(x, P(M.WV))).view(L, cfg.n_kv_heads, hd).transpose(0, 1)
         o = F.scaled_dot_product_attention(q, k.repeat_interleave(g, 0), v.repeat_interleave(g, 0), is_causal=False)
-        x = st(x + F.linear(st(o.transpose(0, 1).reshape(L, cfg.d)), P(M.WO)))
-        h = st(norm(x))
-        a = st(F.silu(F.linear(h, P(M.WGATE))) * F.linear(h, P(M.WUP)))
+        x = st(x + F.linear(sb(o.transpose(0, 1).reshape(L, cfg.d)), P(M.WO)))
+        a = sb(F.silu(proj(x, P(M.WGATE))) * proj(x, P(M.WUP)))
         x = st(x + F.linear(a, P(M.WDOWN)))
-    return st(F.linear(st(norm(x)), T[M.TID_HEAD])).numpy()
+    return st(F.linear(sb(norm(x)), T[M.TID_HEAD])).numpy()
 
 
 def test_forward_matches_independent_torch_block():
@@ -235,6 +244,21 @@ def test_forward_matches_independent_torch_block():
     for l in range(cfg.n_layers):
         t2[M.layer_tid(l, M.WGATE)], t2[M.layer_tid(l, M.WUP)] = t[M.layer_tid(l, M.WUP)], t[M.layer_tid(l, M.WGATE)]
     assert np.max(np.abs(_torch_block_forward(cfg, t2, s) - ref)) > 1e-1
+
+
+def test_bf16_forward_matches_independent_torch_block():
+    # the bf16 storage points (the projections read bf16(x), the norm scales their results)
+    pytest.importorskip("torch")
+    cfg = M.ModelConfig(n_layers=2, d=32, n_heads=4, n_kv_heads=2, ffn=48, vocab=11, dtype="bf16", seed=3)
+    rng = np.random.default_rng(23)
+    t = {tid: W.round_bf16(rng.normal(scale=0.4 if tid >= 2 else 1.0, size=shp))
+         for tid, shp in M.tensor_shapes(cfg).items()}
+    w = M.Weights(cfg, tensors=t)
+    s = np.array([3, 11, 0, 7, 11, 2, 10, 5, 11])
+    ours = M.forward(w, s)
+    ref = _torch_block_forward(cfg, t, s, bf16=True)
+    print("bf16 oracle vs torch restatement: max-abs %.3g" % np.max(np.abs(ours - ref)))
+    assert np.max(np.abs(ours - ref)) <= 1e-4 * max(1.0, np.max(np.abs(ref)))
 
 
 def test_ffn_closed_form_single_layer():
