@@ -395,6 +395,302 @@ __global__ void __launch_bounds__(THREADS, Tmem<HD>::CTAS_PER_SM)  // head dim 6
 
 }  // namespace fat
 
+// ---- two query tiles per CTA --------------------------------------------------------------
+// Persistent, one CTA per SM, work items (256 queries = query tiles A and B, head, window):
+// each K and V^T tile brought into shared memory serves both query tiles, so the bytes
+// moved from L2 per tensor-core FLOP are half those of one query tile per CTA.  10 warps:
+//   warp 0      TMA: per key tile K_j then V^T_{j-1} (2-stage rings), Q_A and Q_B once per
+//               item (each released as soon as the item's last S of that tile is issued).
+//   warp 1      allocates all 512 TMEM columns -- S_A [0,128), S_B [128,256),
+//               O_A [256, 256+HD), O_B [256+HD, 256+2HD); P_X is written over the first 64
+//               columns of S_X -- and issues, per key tile j,
+//                  PV_A(j), S_A(j+1), PV_B(j), S_B(j+1)
+//               so each softmax group works on its tile while the tensor core runs the
+//               other tile's two products.  The tcgen05.mma operations of one thread run
+//               in issue order, so S_X(j+1) overwrites P_X(j) only after PV_X(j) has read
+//               it, and the commit after S_X(j+1) also covers PV_X(j): a softmax group that
+//               sees S_X(j+1) may rescale or read O_X.
+//   warps 2-5   softmax of query tile A (one thread per row, as in fat::fa_tc_kernel);
+//   warps 6-9   the same for query tile B.
+// An item's output (O_X / l) is written at the next item's first tile of X, before the
+// first P V of that item overwrites O_X.  Requires the window length to be a multiple of
+// 256.  All waits are bounded.
+namespace fa2 {
+
+constexpr int BQ = 128, BK = 128;
+constexpr int THREADS = 320;
+constexpr float RESCALE_THRESHOLD = 8.0f;
+
+template <int HD>
+struct Smem {
+  static_assert(HD == 64 || HD == 128, "Q / K rows of one or two 128-byte swizzle blocks");
+  static constexpr int QT = BQ * HD * 2;   // one query tile
+  static constexpr int Q = 0;              // Q_A, Q_B
+  static constexpr int KT = BK * HD * 2;   // one key tile
+  static constexpr int K = Q + 2 * QT;     // 2 key stages
+  static constexpr int VTT = HD * BK * 2;  // one V^T tile (f16)
+  static constexpr int VT = K + 2 * KT;    // 2 V^T stages
+  static constexpr int BARS = VT + 2 * VTT;
+  // + barriers + alignment slack; at least 116 KB so that one CTA holds an SM (it takes all of TMEM)
+  static constexpr int TOTAL = BARS + 256 + 1024 > 116 * 1024 ? BARS + 256 + 1024 : 116 * 1024;
+};
+
+template <int HD>
+__global__ void __launch_bounds__(THREADS, 1)
+    fa2_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt, int n_chunks,
+               int L, int nh, int nkv, int d, bf16* __restrict__ out, float scale_log2, int* err) {
+  using S = Smem<HD>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+  const uint32_t base = (smem_u32(smem_raw) + 1023) & ~1023u;
+  const uint32_t sQ = base + S::Q, sK = base + S::K, sVt = base + S::VT;
+  const uint32_t bar = base + S::BARS;
+  auto k_full = [&](int st) { return bar + 8 * st; };
+  auto k_empty = [&](int st) { return bar + 16 + 8 * st; };
+  auto v_full = [&](int st) { return bar + 32 + 8 * st; };
+  auto v_empty = [&](int st) { return bar + 48 + 8 * st; };
+  auto q_full = [&](int x) { return bar + 64 + 8 * x; };
+  auto q_empty = [&](int x) { return bar + 80 + 8 * x; };
+  auto s_full = [&](int x) { return bar + 96 + 8 * x; };
+  auto p_ready = [&](int x) { return bar + 112 + 8 * x; };
+  auto o_free = [&](int x) { return bar + 128 + 8 * x; };
+  auto fin = [&](int x) { return bar + 144 + 8 * x; };
+  const uint32_t drain_bar = bar + 160;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nt = L / BK, npair = L / (2 * BQ);
+  const int items = n_chunks * nh * npair;
+  const int n_my = blockIdx.x < items ? (items - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  const int total = n_my * nt;
+  auto item_of = [&](int it, int& w, int& h, int& q0) {  // q0: first query of tile A
+    const int id = (int)blockIdx.x + it * (int)gridDim.x;
+    q0 = (id % npair) * 2 * BQ;
+    h = (id / npair) % nh;
+    w = id / (npair * nh);
+  };
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(k_full(x), 1);
+      mbar_init(k_empty(x), 1);
+      mbar_init(v_full(x), 1);
+      mbar_init(v_empty(x), 1);
+      mbar_init(q_full(x), 1);
+      mbar_init(q_empty(x), 1);
+      mbar_init(s_full(x), 1);
+      mbar_init(p_ready(x), 4 * 32);
+      mbar_init(o_free(x), 4 * 32);
+      mbar_init(fin(x), 1);
+    }
+    mbar_init(drain_bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) t5::tmem_alloc(smem_u32(&tmem_slot), 512);
+  t5::fence_before();
+  __syncthreads();
+  t5::fence_after();
+  const uint32_t tmem = tmem_slot;
+  auto tS = [&](int x) { return tmem + x * BK; };
+  auto tO = [&](int x) { return tmem + 2 * BK + x * HD; };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t kpend = 0, vpend = 0, kpar = 0, vpar = 0, qpend = 0, qpar = 0;
+      for (int J = 0; J <= total && !abort_flag; ++J) {
+        if (J < total) {
+          const int it = J / nt, j = J % nt;
+          int w, h, q0;
+          item_of(it, w, h, q0);
+          const int g = h / (nh / nkv);
+          const int st = J & 1;
+          const uint32_t ph = (J >> 1) & 1;
+          if (!mbar_wait_bounded(k_empty(st), ph ^ 1, &abort_flag, err)) break;
+          mbar_arrive_expect_tx(k_full(st), BK * HD * 2);
+          for (int kb = 0; kb < HD / 64; ++kb)
+            t5::tma_load_2d(sK + st * S::KT + kb * BK * 128, &tmQK, d + g * HD + kb * 64, w * L + j * BK, k_full(st));
+          kpend |= 1u << st;
+          kpar = (kpar & ~(1u << st)) | (ph << st);
+        }
+        if (J >= 1) {  // V^T_{J-1}: the P V products of tile J-1 come before the S products of tile J
+          const int Jv = J - 1, it = Jv / nt, j = Jv % nt;
+          int w, h, q0;
+          item_of(it, w, h, q0);
+          const int g = h / (nh / nkv);
+          const int st = Jv & 1;
+          const uint32_t ph = (Jv >> 1) & 1;
+          if (!mbar_wait_bounded(v_empty(st), ph ^ 1, &abort_flag, err)) break;
+          mbar_arrive_expect_tx(v_full(st), BK * HD * 2);
+          for (int kk = 0; kk < 2; ++kk)
+            t5::tma_load_2d(sVt + st * S::VTT + kk * HD * 128, &tmVt, j * BK + kk * 64, (w * nkv + g) * HD,
+                            v_full(st));
+          vpend |= 1u << st;
+          vpar = (vpar & ~(1u << st)) | (ph << st);
+        }
+        if (J < total && J % nt == 0) {  // the item's query tiles, each once the previous item's last S_X is issued
+          const int it = J / nt;
+          int w, h, q0;
+          item_of(it, w, h, q0);
+          const uint32_t ph = it & 1;
+          bool ok = true;
+          for (int x = 0; x < 2 && ok; ++x) {
+            if (!mbar_wait_bounded(q_empty(x), ph ^ 1, &abort_flag, err)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(q_full(x), BQ * HD * 2);
+            for (int kb = 0; kb < HD / 64; ++kb)
+              t5::tma_load_2d(sQ + x * S::QT + kb * BQ * 128, &tmQK, h * HD + kb * 64, w * L + q0 + x * BQ, q_full(x));
+            qpend |= 1u << x;
+            qpar = (qpar & ~(1u << x)) | (ph << x);
+          }
+          if (!ok) break;
+        }
+      }
+      if (abort_flag) {  // let our own copies land before the CTA can exit
+        volatile int never = 0;
+        for (int st = 0; st < 2; ++st) {
+          if (qpend & (1u << st)) mbar_wait_bounded(q_full(st), (qpar >> st) & 1, &never, err, 100000000ull);
+          if (kpend & (1u << st)) mbar_wait_bounded(k_full(st), (kpar >> st) & 1, &never, err, 100000000ull);
+          if (vpend & (1u << st)) mbar_wait_bounded(v_full(st), (vpar >> st) & 1, &never, err, 100000000ull);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
+      constexpr uint32_t ID_O = t5::idesc_f16(BQ, HD);
+      bool issued = false;
+      // S_X(J) = Q_X K_J^T; tile A waits for K_J (and, at an item's first tile, each tile for its Q)
+      auto issue_s = [&](int x, int J) -> bool {
+        const int st = J & 1, it = J / nt;
+        if (J % nt == 0 && !mbar_wait_bounded(q_full(x), it & 1, &abort_flag, err)) return false;
+        if (x == 0 && !mbar_wait_bounded(k_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
+        t5::fence_after();
+        for (int kb = 0; kb < HD / 64; ++kb)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            t5::mma_bf16(tS(x), t5::sw128_desc(sQ + x * S::QT + kb * BQ * 128 + 32 * k),
+                         t5::sw128_desc(sK + st * S::KT + kb * BK * 128 + 32 * k), ID_S, (kb | k) != 0);
+        t5::commit(s_full(x));
+        if (x == 1) t5::commit(k_empty(st));
+        if (J % nt == nt - 1) t5::commit(q_empty(x));
+        issued = true;
+        return true;
+      };
+      // O_X (+)= P_X(J) V_J, P_X in the first 64 columns of S_X (8 columns per 16 keys)
+      auto issue_pv = [&](int x, int J) -> bool {
+        const int st = J & 1, it = J / nt, j = J % nt;
+        if (!mbar_wait_bounded(p_ready(x), J & 1, &abort_flag, err)) return false;
+        if (x == 0 && !mbar_wait_bounded(v_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
+        // the first P V of an item overwrites O_X: the softmax group must have read the previous item's O_X
+        if (j == 0 && it > 0 && !mbar_wait_bounded(o_free(x), (it - 1) & 1, &abort_flag, err)) return false;
+        t5::fence_after();
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          t5::mma_tmem_a(tO(x), tS(x) + 8 * k, t5::sw128_desc(sVt + st * S::VTT + (k >> 2) * HD * 128 + 32 * (k & 3)),
+                         ID_O, (j | k) != 0);
+        if (x == 1) t5::commit(v_empty(st));
+        if (J == total - 1) t5::commit(fin(x));
+        return true;
+      };
+      bool ok = total == 0 || (issue_s(0, 0) && issue_s(1, 0));
+      for (int J = 0; ok && J < total; ++J) {
+        if (!issue_pv(0, J)) break;
+        if (J + 1 < total && !issue_s(0, J + 1)) break;
+        if (!issue_pv(1, J)) break;
+        if (J + 1 < total && !issue_s(1, J + 1)) break;
+      }
+      if (abort_flag && issued) {
+        volatile int never = 0;
+        t5::commit(drain_bar);
+        mbar_wait_bounded(drain_bar, 0, &never, err, 100000000ull);
+      }
+    }
+  } else {
+    const int x = (warp - 2) >> 2;  // query tile of this softmax group
+    const int q = warp & 3;         // TMEM lane quadrant of this warp
+    const int r = q * 32 + lane;    // query row within the tile (= TMEM lane)
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const uint32_t tSx = tS(x) + lane_off, tOx = tO(x) + lane_off;
+    auto row_of = [&](int it) {
+      int w, h, q0;
+      item_of(it, w, h, q0);
+      return out + ((size_t)w * L + q0 + x * BQ + r) * d + (size_t)h * HD;
+    };
+    float m = -INFINITY, l = 0.0f, l_pend = 0.0f;
+    bool pend = false;
+    for (int J = 0; J < total; ++J) {
+      const int j = J % nt;
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(s_full(x), J & 1, &abort_flag, err))) break;
+      t5::fence_after();
+      uint32_t sr[BK];
+      t5::tmem_ld128(tSx, sr);
+      float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+      for (int i = 0; i < BK / 2; ++i)
+        m4[i & 3] = fat::max3(m4[i & 3], __uint_as_float(sr[2 * i]), __uint_as_float(sr[2 * i + 1]));
+      float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+      mx *= scale_log2;
+      float f = 1.0f;
+      bool need = false;
+      if (j == 0) {
+        m = mx;
+        l = 0.0f;
+      } else if (mx > m + RESCALE_THRESHOLD) {
+        need = true;
+        f = t5::ex2(m - mx);
+        m = mx;
+      }
+#pragma unroll
+      for (int c = 0; c < BK / 2; ++c) {
+        float x0, x1;
+        fat::fma2(x0, x1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), scale_log2, scale_log2, -m, -m);
+        sr[c] = t5::ex2_f16x2(t5::pack_f16x2(x0, x1));
+      }
+      l = l * f + fat::row_sum_f16x2(sr);
+      // S_X(J) complete means every earlier product is too: O_X holds the sum through tile J - 1
+      if (j == 0 && pend) {  // the previous item's output, before this item's first P V overwrites O_X
+        fat::drain_row<HD>(tOx, row_of(J / nt - 1), l_pend);
+        t5::fence_before();
+        mbar_arrive(o_free(x));
+        pend = false;
+      } else if (j > 0 && __any_sync(0xffffffffu, need)) {  // the whole warp rescales its O rows (f = 1 elsewhere)
+#pragma unroll 1
+        for (int c = 0; c < HD / 16; ++c) {
+          uint32_t oc[16];
+          t5::tmem_ld16(tOx + c * 16, oc);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) oc[i] = __float_as_uint(__uint_as_float(oc[i]) * f);
+          t5::tmem_st16(tOx + c * 16, oc);
+        }
+      }
+      t5::tmem_st64(tSx, sr);  // P_X(J) over the first 64 columns of S_X
+      t5::fence_before();
+      mbar_arrive(p_ready(x));
+      if (j == nt - 1) {
+        pend = true;
+        l_pend = l;
+      }
+    }
+    if (pend && !abort_flag) {  // the last item's output
+      if (__all_sync(0xffffffffu, mbar_wait_bounded(fin(x), 0, &abort_flag, err))) {
+        t5::fence_after();
+        fat::drain_row<HD>(tOx, row_of((total - 1) / nt), l_pend);
+        t5::fence_before();
+      }
+    }
+  }
+  t5::fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    t5::fence_after();
+    t5::tmem_dealloc(tmem, 512);
+  }
+}
+
+}  // namespace fa2
+
 bool attention_tc_supported(int L, int hd) { return L > 0 && L % fat::BK == 0 && (hd == 64 || hd == 128); }
 
 int attention_vt_rows(int hd) { return hd; }
@@ -444,7 +740,25 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
   const int64_t items = (int64_t)n_chunks * nh * (L / fat::BQ);
   if (items > 0x7fffffff) return DLMZ_EINVAL;
   ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
-  if (hd == 64) {
+  if (L % (2 * fa2::BQ) == 0) {  // two query tiles per CTA, one CTA per SM
+    const int64_t items2 = items / 2;
+    const int grid = items2 < num_sms() ? (int)items2 : num_sms();
+    if (hd == 64) {
+      constexpr int SM = fa2::Smem<64>::TOTAL;
+      static PerDeviceOnce attr;
+      DLMZ_TRY(attr.run(
+          [] { return cudaFuncSetAttribute(fa2::fa2_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
+      fa2::fa2_kernel<64><<<grid, fa2::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
+                                                        device_error_word());
+    } else {
+      constexpr int SM = fa2::Smem<128>::TOTAL;
+      static PerDeviceOnce attr;
+      DLMZ_TRY(attr.run(
+          [] { return cudaFuncSetAttribute(fa2::fa2_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
+      fa2::fa2_kernel<128><<<grid, fa2::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
+                                                         device_error_word());
+    }
+  } else if (hd == 64) {
     constexpr int SM = fat::Smem<64>::TOTAL;
     static PerDeviceOnce attr;
     DLMZ_TRY(attr.run(
