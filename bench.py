@@ -12,13 +12,15 @@ One benchmark step = one denoising step of compression plus the matching
 denoising step of decompression over a whole batch (512 windows x 1024
 tokens): the forward pass of the batch, the LM head and quantiser on the
 candidate rows (the still-masked positions), selection, and coding
-(decoding) of 16 tokens per window.  The encoder runs W + K denoising steps
+(decoding) of 16 tokens per window.  The encoder runs W + K + 1 denoising steps
 of the batch and terminates its streams; the decoder then replays the same
-W + K steps from those streams and must reproduce the encoder's state.  The
-first W steps of each direction are warm-up, the last K are timed (CUDA
+W + K + 1 steps from those streams and must reproduce the encoder's state.
+The first W steps of each direction are warm-up, the next K are timed (CUDA
 events on the library's stream, device synchronised around each timed
-segment).  ``value`` = input bytes coded (and decoded) per step x K / the
-summed time; compress and decompress are also reported separately.
+segment), and one more untimed step per direction records CUDA events
+around every launch for the per-kernel split and the rooflines.  ``value`` =
+input bytes coded (and decoded) per step x K / the summed time; compress and
+decompress are also reported separately.
 
 ``secondary`` holds the small byte-level workload (8 layers, d = 512, V =
 256; one 512 KiB batch compressed and decompressed per step) and the
@@ -43,6 +45,7 @@ sys.path.insert(0, ROOT)
 METRIC = "input bytes/sec compress+decompress on 1 GB300; bits/byte; % of roofline"
 C4 = dict(n_layers=32, d=4096, n_heads=32, n_kv_heads=32, ffn=12288, vocab=126464, seed=0)
 C4_TOKENS, C4_CHUNK, C4_BATCH, C4_K = 1 << 20, 1024, 512, 16
+PROF_STEPS = 1  # untimed denoising steps per direction whose launches carry events (the kernel split)
 C4_WORKLOAD = ("8B-shaped masked DLM, bf16, random-init: 32 layers d=4096 32 heads (hd 128) FFN 12288 V=126464, "
                "bidirectional attention; 2^20 Zipf(1.05) bigram tokens, windows of 1024 tokens, 512 windows per "
                "batch, top-16 by confidence per step over the whole window, 24-bit CDFs")
@@ -201,25 +204,27 @@ def oracle_child(threads):
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-def cpu_baseline():
-    """The oracle on the host cores: all cores (the figure) and one thread (beside it)."""
+def cpu_baseline(one_thread=False):
+    """The oracle on the host cores: all cores (the figure) and, on request, one thread beside it."""
     cores = host_cores()
     allc = oracle_child(0)
-    one = oracle_child(1)
     step_bytes = C4_K * 4  # one denoising step codes 16 tokens of 4 bytes per window
     val = step_bytes / (2.0 * allc["per_step_s"])  # compress + decompress each run the step
-    return {
+    out = {
         "value": val, "unit": "B/s", "cores": cores, "kind": "oracle",
         "sample": ("one denoising step of one 1024-token window of the headline workload, compress + decompress: "
                    "one float64 transformer layer timed x 32 layers, LM head + quantiser timed on 64 candidate "
                    "rows scaled to the 520 of an average step, selection + range coding of 16 symbols; "
                    "weight generation excluded; extrapolated"),
-        "threads": {"all": cores, "one": 1},
-        "value_one_thread": step_bytes / (2.0 * one["per_step_s"]),
+        "threads": "BLAS threads = all %d host cores" % cores,
         "seconds_per_window_step": allc["per_step_s"],
-        "seconds_per_window_step_one_thread": one["per_step_s"],
         "parts": allc["parts"],
     }
+    if one_thread:  # ~7 minutes on a 16-core Grace host
+        one = oracle_child(1)
+        out["value_one_thread"] = step_bytes / (2.0 * one["per_step_s"])
+        out["seconds_per_window_step_one_thread"] = one["per_step_s"]
+    return out
 
 
 def run_reference(args):
@@ -285,7 +290,7 @@ def run_c4(args, dlmz, torch, rank, ws, dev):
     state = torch.full((nc, L), V, dtype=torch.int32, device=dev)
     committed = torch.zeros(nc, dtype=torch.int32, device=dev)
     pol = dlmz.policy(dlmz.TOPK_CONF, k, 0)
-    n_steps = args.warmup + args.steps
+    n_steps = args.warmup + args.steps + PROF_STEPS
     if n_steps * k > L:
         raise SystemExit("at most %d denoising steps per window" % (L // k))
     P = 24
@@ -300,19 +305,27 @@ def run_c4(args, dlmz, torch, rank, ws, dev):
             torch.distributed.barrier()
         torch.cuda.synchronize()
 
+    launches = [0]
+
     def phase(fn):
-        """W untimed steps, then K steps timed with events on the stream (profiled)."""
+        """W untimed steps, K steps timed with events on the stream, then PROF_STEPS untimed steps with
+        per-launch events for the kernel split (kept out of the timed region)."""
         for i in range(args.warmup):
             fn()
         barrier()
-        prof = dlmz.Profile()
-        dlmz.profile_begin()
+        n0 = dlmz.launch_count()
         e0, e1 = _events()
         e0.record()
         for i in range(args.steps):
             fn()
         e1.record()
         e1.synchronize()
+        launches[0] += dlmz.launch_count() - n0
+        barrier()
+        prof = dlmz.Profile()
+        dlmz.profile_begin()
+        for i in range(PROF_STEPS):
+            fn()
         dlmz.profile_end(prof)
         barrier()
         _prof_add(prof_acc, prof)
@@ -377,6 +390,7 @@ def run_c4(args, dlmz, torch, rank, ws, dev):
         "compress_Bps": ws * step_bytes * args.steps / (enc_ms / 1000.0),
         "decompress_Bps": ws * step_bytes * args.steps / (dec_ms / 1000.0),
         "bits_per_token_stream": stream_bits / float(revealed), "prof": prof_acc, "clocks": clk, "e2e": e2e,
+        "launches": launches[0],
     }
 
 
@@ -518,13 +532,15 @@ def run(args):
                                "achieved": a_ach, "peak": tf_sus, "unit": "TFLOP/s", "frac": a_ach / tf_sus},
         "roofline_quantize": {"bound": "hbm", "achieved": q_ach, "peak": hbm, "unit": "GB/s", "frac": q_ach / hbm},
         "kernel_time_split": split,
-        "gpu_launches": p["launches"],
+        "gpu_launches": r["launches"],
+        "kernel_split_source": ("%d untimed denoising step(s) per direction after the timed ones, CUDA events "
+                                "around every launch" % PROF_STEPS),
         "clocks": r["clocks"],
         "e2e": r["e2e"],
         "secondary": secondary,
     }
     if ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline()
+        line["cpu_baseline"] = cpu_baseline(args.cpu_one_thread)
     print(json.dumps(line))
     if ws > 1:
         torch.distributed.destroy_process_group()
@@ -539,6 +555,7 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
+    ap.add_argument("--cpu-one-thread", action="store_true", help="also time the oracle on one host thread")
     ap.add_argument("--oracle-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.oracle_child:

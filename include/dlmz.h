@@ -336,6 +336,11 @@ typedef struct {
   double bytes[8];
 } dlmz_profile;
 DLMZ_API int dlmz_profile_begin(void);
+/* Number of kernels the library has launched since it was loaded (all
+ * devices and streams; counted whether or not profiling is on, at no device
+ * cost), so a caller can count the launches of a timed region without the
+ * per-launch events of dlmz_profile_begin. */
+DLMZ_API uint64_t dlmz_launch_count(void);
 /* Synchronises the device and fills *out. */
 DLMZ_API int dlmz_profile_end(dlmz_profile* out);
 

@@ -1,5 +1,6 @@
 // Live per-kernel-class profiler: CUDA event pairs recorded on each launch's
 // stream while enabled, summed at dlmz_profile_end.
+#include <atomic>
 #include <vector>
 
 #include "common.cuh"
@@ -14,6 +15,7 @@ struct Pending {
 };
 bool g_on = false;
 uint64_t g_launches = 0;
+std::atomic<uint64_t> g_total{0};  // every launch since the library was loaded
 std::vector<Pending> g_pending;
 std::vector<cudaEvent_t> g_pool;
 cudaEvent_t g_open[PROF_NCLASS];
@@ -33,6 +35,7 @@ cudaEvent_t take_event() {
 bool prof_on() { return g_on; }
 
 void prof_count_launch() {
+  g_total.fetch_add(1, std::memory_order_relaxed);
   if (g_on) ++g_launches;
 }
 
@@ -51,6 +54,8 @@ void prof_record(int cls, cudaStream_t s, bool start, double flops, double bytes
 }  // namespace dlmz
 
 using namespace dlmz;
+
+extern "C" uint64_t dlmz_launch_count(void) { return g_total.load(std::memory_order_relaxed); }
 
 extern "C" int dlmz_profile_begin(void) {
   for (auto& p : g_pending) {

@@ -93,6 +93,7 @@ _sig("dlmz_check", c_int, _P)
 _sig("dlmz_selftest_wait_timeout", c_int, c_uint32, _P)
 _sig("dlmz_profile_begin", c_int)
 _sig("dlmz_profile_end", c_int, POINTER(Profile))
+_sig("dlmz_launch_count", c_uint64)
 
 
 def _ok(rc, where):
@@ -220,6 +221,11 @@ def profile_begin():
 
 def profile_end(prof):
     _ok(lib.dlmz_profile_end(byref(prof)), "dlmz_profile_end")
+
+
+def launch_count():
+    """Kernels launched by the library so far (dlmz_launch_count)."""
+    return int(lib.dlmz_launch_count())
 
 
 def check(stream=0):
