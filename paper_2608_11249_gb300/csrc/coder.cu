@@ -25,24 +25,51 @@
 #include "kernels.cuh"
 #include "coder.cuh"
 #include "exp_table.inc"
+#include "intq.cuh"
 
 namespace dlmz {
 
-static __constant__ uint32_t c_exp_table[256] = DLMZ_EXP_TABLE_INIT;
+static __constant__ uint32_t c_exp_table_c[256] = DLMZ_EXP_TABLE_INIT;
 
 // ---- selection ----------------------------------------------------------------------
+// CTA per window.  The n smallest candidates under (key, position) are those with key < K* plus
+// the lowest-position ones with key == K*, where K* is the n-th smallest key: a most-significant-
+// digit-first radix select (8 passes of 8-bit digits, a shared histogram each) finds K* and how
+// many of its ties are taken, then one ordered pass writes the selected positions ascending.
+constexpr int SEL_T = 256;  // threads per window (one histogram bin per thread)
+
+// exclusive prefix sum over the CTA of one value per thread (SEL_T threads); *total gets the sum
+__device__ __forceinline__ int sel_block_scan(int v, int* wtot, int* total) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int inc = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += t;
+  }
+  if (lane == 31) wtot[w] = inc;
+  __syncthreads();
+  const int tv = lane < SEL_T / 32 ? wtot[lane] : 0;
+  const int pre = __reduce_add_sync(0xffffffffu, lane < w ? tv : 0);
+  *total = __reduce_add_sync(0xffffffffu, tv);
+  __syncthreads();  // wtot may be rewritten by the next scan
+  return pre + inc - v;
+}
+
 template <typename K>
-__global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask_id, int row0, int rpc,
-                              const K* __restrict__ keys, const int32_t* __restrict__ row_map, int n_rule, int k,
-                              int64_t tau_q, int k_min, int k_max, int kcap, int32_t* __restrict__ sel_count,
-                              int32_t* __restrict__ sel_pos) {
+__global__ void __launch_bounds__(SEL_T) select_kernel(const int32_t* __restrict__ state, int L, int mask_id, int row0,
+                                                       int rpc, const K* __restrict__ keys,
+                                                       const int32_t* __restrict__ row_map, int n_rule, int k,
+                                                       int64_t tau_q, int k_min, int k_max, int kcap,
+                                                       int32_t* __restrict__ sel_count, int32_t* __restrict__ sel_pos) {
   extern __shared__ uint64_t skey[];  // rpc keys, then rpc flags (as bytes)
   uint8_t* valid = reinterpret_cast<uint8_t*>(skey + rpc);
-  __shared__ int red[32];
-  __shared__ int s_nsel;
+  __shared__ int hist[SEL_T];
+  __shared__ int wtot[SEL_T / 32];
+  __shared__ int s_bin, s_below;
   const int c = blockIdx.x;
   int nv = 0, nb = 0;
-  for (int i = threadIdx.x; i < rpc; i += blockDim.x) {
+  for (int i = threadIdx.x; i < rpc; i += SEL_T) {
     const bool ok = state ? state[(size_t)c * L + row0 + i] == mask_id : true;
     // null keys: position order; with a row map only candidates have a key row
     const int64_t kr = row_map ? (ok ? row_map[(size_t)c * rpc + i] : -1) : (int64_t)c * rpc + i;
@@ -52,55 +79,65 @@ __global__ void select_kernel(const int32_t* __restrict__ state, int L, int mask
     nv += ok;
     nb += ok && (int64_t)key <= tau_q;
   }
-  // block sums of nv, nb
-#pragma unroll
-  for (int o = 16; o; o >>= 1) {
-    nv += __shfl_xor_sync(0xffffffffu, nv, o);
-    nb += __shfl_xor_sync(0xffffffffu, nb, o);
+  int tv, tb;
+  sel_block_scan(nv, wtot, &tv);
+  sel_block_scan(nb, wtot, &tb);
+  int n;
+  if (n_rule == 0) {
+    n = min(k, tv);
+  } else {
+    n = tb < k_min ? min(k_min, tv) : tb;
+    if (k_max > 0 && n > k_max) n = k_max;
   }
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = nv | (nb << 16);
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int tv = 0, tb = 0;
-    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) {
-      tv += red[i] & 0xffff;
-      tb += red[i] >> 16;
+  const int nsel = min(n, kcap);
+  // K* = the nsel-th smallest key; `need` of its ties (lowest positions first) are taken
+  uint64_t kstar = ~0ull;
+  int need = 0x7fffffff;
+  if (nsel > 0 && nsel < tv) {
+    uint64_t prefix = 0, pmask = 0;
+    int rank = nsel - 1;  // 0-based rank of K* among the candidates still matching the prefix
+#pragma unroll 1
+    for (int shift = 56; shift >= 0; shift -= 8) {
+      hist[threadIdx.x] = 0;
+      __syncthreads();
+      for (int i = threadIdx.x; i < rpc; i += SEL_T) {
+        const uint64_t key = skey[i];
+        if (valid[i] && (key & pmask) == prefix) atomicAdd(&hist[(int)(key >> shift) & 255], 1);
+      }
+      __syncthreads();
+      const int cnt = hist[threadIdx.x];
+      int tot;
+      const int below = sel_block_scan(cnt, wtot, &tot);
+      if (below <= rank && rank < below + cnt) {  // exactly one bin holds the rank
+        s_bin = threadIdx.x;
+        s_below = below;
+      }
+      __syncthreads();
+      prefix |= (uint64_t)s_bin << shift;
+      pmask |= 0xFFull << shift;
+      rank -= s_below;
     }
-    int n;
-    if (n_rule == 0) {
-      n = min(k, tv);
-    } else {
-      n = tb < k_min ? min(k_min, tv) : tb;
-      if (k_max > 0 && n > k_max) n = k_max;
-    }
-    s_nsel = min(n, kcap);
+    kstar = prefix;
+    need = rank + 1;
   }
-  __syncthreads();
-  const int nsel = s_nsel;
-  // rank every candidate; selected iff rank < nsel; write ascending positions
-  __shared__ int wcount[32];
-  int base = 0;
-  for (int i0 = 0; i0 < rpc; i0 += blockDim.x) {
+  // ordered pass: candidate i is selected iff key < K*, or key == K* and fewer than `need` ties
+  // precede it (with nsel >= #candidates every candidate is selected)
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int ties = 0, base = 0;
+  for (int i0 = 0; i0 < rpc; i0 += SEL_T) {
     const int i = i0 + threadIdx.x;
-    bool sel = false;
-    if (i < rpc && valid[i]) {
-      const uint64_t ki = skey[i];
-      int rank = 0;
-      for (int j = 0; j < rpc; ++j)
-        rank += valid[j] && (skey[j] < ki || (skey[j] == ki && j < i));
-      sel = rank < nsel;
-    }
-    const unsigned bal = __ballot_sync(0xffffffffu, sel);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    if (lane == 0) wcount[w] = __popc(bal);
-    __syncthreads();
-    int off = base;
-    for (int j = 0; j < w; ++j) off += wcount[j];
-    if (sel) sel_pos[(size_t)c * kcap + off + __popc(bal & ((1u << lane) - 1))] = row0 + i;
-    int tot = 0;
-    for (int j = 0; j < (int)(blockDim.x >> 5); ++j) tot += wcount[j];
+    const bool ok = i < rpc && valid[i] && nsel > 0;
+    const uint64_t key = ok ? skey[i] : 0;
+    const bool tie = ok && key == kstar;
+    int tot;
+    const int tie_before = ties + sel_block_scan(tie ? 1 : 0, wtot, &tot);
+    ties += tot;
+    const bool sel = ok && (nsel >= tv || key < kstar || (tie && tie_before < need));
+    const int off = base + sel_block_scan(sel ? 1 : 0, wtot, &tot);
+    if (sel) sel_pos[(size_t)c * kcap + off] = row0 + i;
     base += tot;
-    __syncthreads();
+    (void)lane;
+    (void)w;
   }
   if (threadIdx.x == 0) sel_count[c] = nsel;
 }
@@ -116,7 +153,7 @@ int select_rows(const int32_t* state, int n_chunks, int L, int mask_id, int row0
   DLMZ_TRY(attr.run(
       [] { return cudaFuncSetAttribute(select_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024); }));
   ProfScope prof(PROF_SELECT, s, 0, (double)n_chunks * rpc * (sizeof(K) + 4));
-  select_kernel<K><<<n_chunks, 256, smem, s>>>(state, L, mask_id, row0, rpc, keys, row_map, n_rule, k, tau_q, k_min,
+  select_kernel<K><<<n_chunks, SEL_T, smem, s>>>(state, L, mask_id, row0, rpc, keys, row_map, n_rule, k, tau_q, k_min,
                                                k_max, kcap, sel_count, sel_pos);
   return launch_status();
 }
@@ -197,11 +234,12 @@ __device__ __forceinline__ uint64_t block_excl_scan(uint64_t v, uint64_t* wsum, 
 template <bool DECODE>
 __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
   __shared__ uint32_t T[256];
+  __shared__ uint32_t tabf[QW0 + 1];  // floor(w(q) R / W) of the current row (0 from QW0 on)
   __shared__ uint64_t wsum[CT / 32];
   __shared__ uint64_t s_slot, s_cs, s_fs;
   __shared__ int s_sym;
   __shared__ CoderState st;
-  for (int i = threadIdx.x; i < 256; i += CT) T[i] = c_exp_table[i];
+  for (int i = threadIdx.x; i < 256; i += CT) T[i] = c_exp_table_c[i];
   const int c = blockIdx.x;
   const int n = a.sel_count[c];
   if (threadIdx.x == 0) st = a.state_c[c];
@@ -224,21 +262,24 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
     const float m = a.mx[row];
     const uint64_t Wr = a.W[row];
     const int top = a.top[row];
-    auto qv = [&](float x) -> int {
-      return isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f))
-                         : 8191;
-    };
-    uint64_t sseg = 0;
-    for (int v = v0; v < v1; ++v) {
-      const float x = lr[v];
-      const int q = isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f)) : 8191;
-      sseg += 1 + (uint64_t)(T[q & 255] >> (q >> 8)) * R / Wr;
+    // this row's floor(w(q) R / W) for every code (division-free, K = floor(R 2^64 / W)); the
+    // barrier at the end of the previous symbol leaves the table free
+    {
+      uint64_t K = 0;
+      if ((threadIdx.x & 31) == 0) K = recip_scaled((uint32_t)R, Wr);
+      K = __shfl_sync(0xffffffffu, K, 0);
+      for (int b = threadIdx.x; b <= QW0; b += CT) tabf[b] = b < QW0 ? floor_wr_over_w(quant_w(T, b), (uint32_t)R, Wr, K) : 0u;
+      __syncthreads();
     }
+    // floor(w_v R / W) of element v (codes from QW0 on weigh nothing, non-finite values land there)
+    auto flo_of = [&](int v) -> uint64_t { return tabf[code_index(__fsub_rn(m, lr[v]))]; };
+    uint64_t sseg = 0;
+    for (int v = v0; v < v1; ++v) sseg += 1 + flo_of(v);
     uint64_t total;
     const uint64_t pre = block_excl_scan(sseg, wsum, &total);
     const uint64_t D = (1ull << P) - total;
     // f_v of this row (the same integer table the coders use)
-#define FREQ(v_) (1 + (uint64_t)(T[qv(lr[v_]) & 255] >> (qv(lr[v_]) >> 8)) * R / Wr + ((v_) == top ? D : 0))
+#define FREQ(v_) (1 + flo_of(v_) + ((v_) == top ? D : 0))
     const uint64_t lo = pre + (v0 > top ? D : 0);
     const uint64_t hi = lo + sseg + (top >= v0 && top < v1 ? D : 0);
     if (!DECODE) {
@@ -246,9 +287,7 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       if (sym >= v0 && sym < v1) {
         uint64_t cum = lo;
         for (int v = v0; v < v1; ++v) {
-          const float x = lr[v];
-          const int q = isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f)) : 8191;
-          const uint64_t f = 1 + (uint64_t)(T[q & 255] >> (q >> 8)) * R / Wr + (v == top ? D : 0);
+          const uint64_t f = FREQ(v);
           if (v == sym) {
             s_cs = cum;
             s_fs = f;
@@ -358,9 +397,7 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
       } else if (slot >= lo && slot < hi) {
         uint64_t cum = lo;
         for (int v = v0; v < v1; ++v) {
-          const float x = lr[v];
-          const int q = isfinite(x) ? __float2int_rn(fminf(__fmul_rn(__fsub_rn(m, x), __uint_as_float(DLMZ_QSCALE_BITS)), 8191.f)) : 8191;
-          const uint64_t f = 1 + (uint64_t)(T[q & 255] >> (q >> 8)) * R / Wr + (v == top ? D : 0);
+          const uint64_t f = FREQ(v);
           if (slot < cum + f) {
             s_sym = v;
             s_cs = cum;

@@ -13,6 +13,7 @@
 // result is independent of thread layout and reduction order.
 #include "kernels.cuh"
 #include "exp_table.inc"
+#include "intq.cuh"
 
 namespace dlmz {
 
@@ -23,7 +24,6 @@ __device__ __forceinline__ int quant_q(float m, float l) {
   return __float2int_rn(fminf(t, 8191.0f));
 }
 
-__device__ __forceinline__ uint32_t quant_w(const uint32_t* T, int q) { return T[q & 255] >> (q >> 8); }
 
 // Digit-by-digit binary logarithm: ~floor(2^16 log2 W) for W >= 2^31.
 __device__ __forceinline__ uint32_t log2q16(uint64_t W) {
@@ -286,23 +286,10 @@ __global__ void __launch_bounds__(QT) quantize_cta_kernel(const float* __restric
 // the CDF pass looks floor(w(q) R / W) up in the same shared table, rewritten
 // in place.  Every CDF partial sum is at most 2^P <= 2^24, so the scan runs
 // in 32-bit integers.
-// floor(w R / W) without a division: K = floor(R 2^64 / W) per row (R < W), the
-// estimate (w K) >> 64 is floor(w R / W) or one less, and (e + 1) W <= w R
-// (both sides < 2^64) decides which.
+// floor(w R / W) without a division: K = floor(R 2^64 / W) per row (R < W); see intq.cuh.
 constexpr int NQ = 8192;       // codes q = 0 .. 8191
-// w(q) = T[q & 255] >> (q >> 8) is 0 for q > 7936 (T[j] < 2^31 for j >= 1; w(7936) = T[0] >> 31 = 1):
-// those codes add nothing to W, A or D and need no bin
-constexpr int QW0 = 31 * 256 + 1;
 constexpr int QNT = 256;       // threads per CTA
 constexpr int QCPS = 4;        // CTAs per SM (4 x 33 KB shared memory, 64 registers per thread)
-
-__device__ __forceinline__ uint32_t floor_wr_over_w(uint32_t w, uint32_t R, uint64_t Wsum, uint64_t K) {
-  const uint64_t lo = (uint64_t)w * (uint32_t)K;          // w * K_lo
-  const uint64_t hi = (uint64_t)w * (uint32_t)(K >> 32);  // w * K_hi
-  const uint32_t est = (uint32_t)((hi + (lo >> 32)) >> 32);
-  const uint64_t x = (uint64_t)w * R;
-  return est + (((uint64_t)(est + 1) * Wsum) <= x ? 1u : 0u);
-}
 
 template <int NT, int CPS>
 __global__ void __launch_bounds__(NT, CPS)

@@ -3,6 +3,9 @@
     python -m paper_2608_11249_gb300.kernel_bench forward --chunks 64
         one forward (Definition 3) of the 8-layer d=512 bf16 byte model over
         `chunks` windows of 512 positions (LM head on a 128-row block), repeated --reps times
+    python -m paper_2608_11249_gb300.kernel_bench forward --model 8b --layers 2 --chunks 64
+        the same for `layers` layers of the 8B-shaped model (d=4096, 32 heads, FFN 12288,
+        V=126464) over windows of 1024 positions (LM head on 16 rows per window)
     python -m paper_2608_11249_gb300.kernel_bench quantize --rows 2048 --vocab 126464
         the quantiser (CDF + scores) on spiked N(0,3) logits rows
     python -m paper_2608_11249_gb300.kernel_bench gemm --m 32768 --n 4096 --k 512
@@ -36,10 +39,18 @@ def main():
     ap.add_argument("--n", type=int, default=4096)
     ap.add_argument("--k", type=int, default=512)
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--model", choices=["byte", "8b"], default="byte")
+    ap.add_argument("--layers", type=int, default=2)
     a = ap.parse_args()
     torch.cuda.set_device(0)
     g = torch.Generator(device="cuda").manual_seed(0)
-    if a.what == "forward":
+    if a.what == "forward" and a.model == "8b":
+        V, L, rpc = 126464, 1024, 16
+        m = dlmz.Model(a.layers, 4096, 32, 32, 12288, V, dlmz.BF16, seed=0)
+        state = torch.randint(0, V + 1, (a.chunks, L), dtype=torch.int32, device="cuda", generator=g)
+        logits = torch.empty(a.chunks * rpc, V, dtype=torch.float32, device="cuda")
+        fn = lambda: m.forward_logits(state.data_ptr(), a.chunks, L, 0, rpc, logits.data_ptr())
+    elif a.what == "forward":
         m = dlmz.Model(8, 512, 8, 8, 2048, 256, dlmz.BF16, seed=0)
         L = 512
         state = torch.randint(0, 257, (a.chunks, L), dtype=torch.int32, device="cuda", generator=g)

@@ -19,7 +19,9 @@ def _rows(V, n, seed):
 
 
 @pytest.mark.parametrize("V,n", [(2, 9), (4, 33), (37, 70), (256, 300), (300, 50), (512, 40), (1000, 20), (1001, 7),
-                                 (5000, 17), (126464, 5), (152064, 3)])
+                                 (5000, 17), (126464, 5), (152064, 3),
+                                 # more rows than SMs: each CTA of the large-vocabulary kernel walks several rows
+                                 (1000, 1300), (4100, 700)])
 def test_quantize_bit_exact(dev, V, n):
     import torch
     d = dlmz()

@@ -50,6 +50,8 @@ def _forward_sampled(d, spec, nc, L, row0, rpc, sample, seed, tol=None):
         else:
             alt = OM.forward(w, state[c], rows=rows, matmul_dtype=np.float32) - ref
             nerr, nrms = float(np.max(np.abs(alt))), float(np.sqrt(np.mean(alt ** 2)))
+            print("%s window %d: GPU vs oracle max-abs %.4g rms %.4g; oracle float32 vs float64 max-abs %.4g rms %.4g"
+                  % (spec[:6], c, err, rms, nerr, nrms))
             assert err <= 2 * nerr and rms <= 2 * nrms, (c, err, rms, nerr, nrms)
     m.close()
 
