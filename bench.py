@@ -55,6 +55,9 @@ C2_WORKLOAD = ("small byte-level masked DLM, bf16, 8 layers d=512 8 heads FFN 20
                "Markov/Zipf(1.1) bytes; windows of 512 B, 1024 windows per batch, block 128, top-k 8 by "
                "confidence, 16-bit CDFs")
 C3_ROWS, C3_V, C3_GROUP, C3_TOPK = 65536, 126464, 1024, 32
+# Mean DRAM bytes per tcgen05 GEMM launch of an 8B-shaped layer at 512 windows, scaled from an ncu
+# capture of the same kernels at 16 windows (B is re-read once per row group, so traffic grows with M)
+GEMM_TRAFFIC_PER_LAUNCH = 53.2e9
 CLASSES = ["gemm_tcgen05", "gemm_cuda_core", "attention", "quantize", "select", "code", "norm_rope_embed", "other"]
 
 
@@ -526,7 +529,11 @@ def run(args):
                                                   "down+residual, LM head on candidate rows)",
                      "achieved": g_ach, "peak": tf_sus, "unit": "TFLOP/s", "frac": g_ach / tf_sus,
                      "peak_source": "%s bf16_tflops_sustained (kernel timed inside a long step)" % src,
-                     "traffic": None, "launches": p["n"][gi],
+                     "traffic": GEMM_TRAFFIC_PER_LAUNCH,
+                     "traffic_source": ("dram__bytes_read.sum + dram__bytes_write.sum of one layer's four GEMM "
+                                        "launches at 16 windows (one ncu capture), mean per launch x 32 to 512 "
+                                        "windows (traffic grows with the tokens)"),
+                     "launches": p["n"][gi],
                      "avg_launch_ms": p["ms"][gi] / p["n"][gi] if p["n"][gi] else None},
         "roofline_attention": {"bound": "tensor", "kernel": "tcgen05 bidirectional attention, head dim 128",
                                "achieved": a_ach, "peak": tf_sus, "unit": "TFLOP/s", "frac": a_ach / tf_sus},

@@ -10,6 +10,10 @@
         the quantiser (CDF + scores) on spiked N(0,3) logits rows
     python -m paper_2608_11249_gb300.kernel_bench gemm --m 32768 --n 4096 --k 512
         one bf16 tensor-core GEMM with float32 output
+    python -m paper_2608_11249_gb300.kernel_bench step --layers 1 --chunks 16
+        one denoising step of compression (forward, LM head and quantiser on the
+        candidates, selection, range coding of 16 tokens per window) of the
+        8B-shaped model with `layers` layers over `chunks` windows of 1024 tokens
 
 Prints the mean CUDA-event time per repetition.
 """
@@ -31,7 +35,7 @@ def main():
     from paper_2608_11249_gb300 import dlmz
 
     ap = argparse.ArgumentParser()
-    ap.add_argument("what", choices=["forward", "quantize", "gemm"])
+    ap.add_argument("what", choices=["forward", "quantize", "gemm", "step"])
     ap.add_argument("--chunks", type=int, default=64)
     ap.add_argument("--rows", type=int, default=2048)
     ap.add_argument("--vocab", type=int, default=126464)
@@ -44,7 +48,18 @@ def main():
     a = ap.parse_args()
     torch.cuda.set_device(0)
     g = torch.Generator(device="cuda").manual_seed(0)
-    if a.what == "forward" and a.model == "8b":
+    if a.what == "step":
+        from paper_2608_11249_gb300 import sources
+        V, L, k = 126464, 1024, 16
+        m = dlmz.Model(a.layers, 4096, 32, 32, 12288, V, dlmz.BF16, seed=0)
+        sym = torch.from_numpy(sources.zipf_bigram_tokens(a.chunks * L, V, seed=0).astype(np.int32)).cuda()
+        state = torch.full((a.chunks, L), V, dtype=torch.int32, device="cuda")
+        enc = dlmz.Coder(a.chunks, L, V, 24)
+        enc.reset_encoder()
+        pol = dlmz.policy(dlmz.TOPK_CONF, k, 0)
+        a.reps = min(a.reps, L // k - 1)
+        fn = lambda: m.encode_step(enc, pol, 0, L, sym.data_ptr(), state.data_ptr())
+    elif a.what == "forward" and a.model == "8b":
         V, L, rpc = 126464, 1024, 16
         m = dlmz.Model(a.layers, 4096, 32, 32, 12288, V, dlmz.BF16, seed=0)
         state = torch.randint(0, V + 1, (a.chunks, L), dtype=torch.int32, device="cuda", generator=g)
