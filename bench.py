@@ -219,11 +219,11 @@ def cpu_baseline(one_thread=False):
                    "one float64 transformer layer timed x 32 layers, LM head + quantiser timed on 64 candidate "
                    "rows scaled to the 520 of an average step, selection + range coding of 16 symbols; "
                    "weight generation excluded; extrapolated"),
-        "threads": "BLAS threads = all %d host cores" % cores,
+        "threads": "BLAS threads = all %d host cores (value); one thread (value_one_thread)" % cores,
         "seconds_per_window_step": allc["per_step_s"],
         "parts": allc["parts"],
     }
-    if one_thread:  # ~7 minutes on a 16-core Grace host
+    if one_thread:  # the sample's wall time on one thread: under a minute on a Grace host
         one = oracle_child(1)
         out["value_one_thread"] = step_bytes / (2.0 * one["per_step_s"])
         out["seconds_per_window_step_one_thread"] = one["per_step_s"]
@@ -547,7 +547,7 @@ def run(args):
         "secondary": secondary,
     }
     if ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_one_thread)
+        line["cpu_baseline"] = cpu_baseline(not args.no_cpu_one_thread)
     print(json.dumps(line))
     if ws > 1:
         torch.distributed.destroy_process_group()
@@ -562,7 +562,7 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
-    ap.add_argument("--cpu-one-thread", action="store_true", help="also time the oracle on one host thread")
+    ap.add_argument("--no-cpu-one-thread", action="store_true", help="time the oracle on all host cores only")
     ap.add_argument("--oracle-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.oracle_child:

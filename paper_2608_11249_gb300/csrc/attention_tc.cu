@@ -414,7 +414,7 @@ __global__ void __launch_bounds__(THREADS, Tmem<HD>::CTAS_PER_SM)  // head dim 6
 //   warps 6-9   the same for query tile B.
 // An item's output (O_X / l) is written at the next item's first tile of X, before the
 // first P V of that item overwrites O_X.  Requires the window length to be a multiple of
-// 256.  All waits are bounded.
+// 256; used at head dim 128.  All waits are bounded.
 namespace fa2 {
 
 constexpr int BQ = 128, BK = 128;
@@ -740,24 +740,17 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
   const int64_t items = (int64_t)n_chunks * nh * (L / fat::BQ);
   if (items > 0x7fffffff) return DLMZ_EINVAL;
   ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
-  if (L % (2 * fa2::BQ) == 0) {  // two query tiles per CTA, one CTA per SM
+  if (hd == 128 && L % (2 * fa2::BQ) == 0) {
+    // two query tiles per CTA, one CTA per SM (at head dim 64 the one-tile kernel, two CTAs per SM,
+    // measured faster: 37.6 against 40.1 ms per byte-model forward over 1024 windows of 512)
     const int64_t items2 = items / 2;
     const int grid = items2 < num_sms() ? (int)items2 : num_sms();
-    if (hd == 64) {
-      constexpr int SM = fa2::Smem<64>::TOTAL;
-      static PerDeviceOnce attr;
-      DLMZ_TRY(attr.run(
-          [] { return cudaFuncSetAttribute(fa2::fa2_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
-      fa2::fa2_kernel<64><<<grid, fa2::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
-                                                        device_error_word());
-    } else {
-      constexpr int SM = fa2::Smem<128>::TOTAL;
-      static PerDeviceOnce attr;
-      DLMZ_TRY(attr.run(
-          [] { return cudaFuncSetAttribute(fa2::fa2_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
-      fa2::fa2_kernel<128><<<grid, fa2::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
-                                                         device_error_word());
-    }
+    constexpr int SM = fa2::Smem<128>::TOTAL;
+    static PerDeviceOnce attr;
+    DLMZ_TRY(attr.run(
+        [] { return cudaFuncSetAttribute(fa2::fa2_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM); }));
+    fa2::fa2_kernel<128><<<grid, fa2::THREADS, SM, s>>>(mqk, mvt, n_chunks, L, nh, nkv, d, out, scale_log2,
+                                                       device_error_word());
   } else if (hd == 64) {
     constexpr int SM = fat::Smem<64>::TOTAL;
     static PerDeviceOnce attr;

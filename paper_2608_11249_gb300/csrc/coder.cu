@@ -440,11 +440,330 @@ __global__ void __launch_bounds__(CT) code_kernel(CodeArgs a) {
   }
 }
 
+// ---- row-parallel range / rANS coding ----------------------------------------------------------
+// The frequencies of the selected rows do not depend on one another: one CTA per selected row
+// (grid kcap x windows) computes them from the row's logits in one pass, and only the coder itself,
+// which is sequential within a window, runs per window afterwards.
+constexpr int RT_ROWS = 256;
+
+__device__ __forceinline__ size_t selected_row(const CodeArgs& a, int c, int j, int pos) {
+  return a.row_map ? (size_t)a.row_map[(size_t)c * a.rpc + (pos - a.row0)]
+       : a.sel_major ? (size_t)c * a.kcap + j
+                     : (size_t)c * a.rpc + (pos - a.row0);
+}
+
+// shared table floor(w(q) R / W) of one row for every code (0 from QW0 on); all threads call it
+__device__ void build_floor_table(uint32_t* tabf, const uint32_t* T, uint32_t R, uint64_t Wr) {
+  uint64_t K = 0;
+  if ((threadIdx.x & 31) == 0) K = recip_scaled(R, Wr);
+  K = __shfl_sync(0xffffffffu, K, 0);
+  for (int b = threadIdx.x; b <= QW0; b += blockDim.x) tabf[b] = b < QW0 ? floor_wr_over_w(quant_w(T, b), R, Wr, K) : 0u;
+  __syncthreads();
+}
+
+// floor(w R / W) of one element: from the shared table for large vocabularies; directly (K) for
+// vocabularies below the table's 7938 entries, where building the table would cost more than the row
+struct RowFloor {
+  const uint32_t* tabf;
+  const uint32_t* T;
+  uint32_t R;
+  uint64_t W, K;
+  bool table;
+  __device__ __forceinline__ uint32_t operator()(float m, float x) const {
+    const uint32_t q = code_index(__fsub_rn(m, x));
+    if (table) return tabf[q];
+    return q < (uint32_t)QW0 ? floor_wr_over_w(quant_w(T, (int)q), R, W, K) : 0u;
+  }
+};
+
+__device__ RowFloor row_floor(uint32_t* tabf, const uint32_t* T, uint32_t R, uint64_t Wr, int V) {
+  RowFloor rf{tabf, T, R, Wr, 0, V > QW0};
+  if (rf.table) {
+    build_floor_table(tabf, T, R, Wr);
+  } else {
+    uint64_t K = 0;
+    if ((threadIdx.x & 31) == 0) K = recip_scaled(R, Wr);
+    rf.K = __shfl_sync(0xffffffffu, K, 0);
+  }
+  return rf;
+}
+
+// block sum of one u32 per thread (RT_ROWS threads); every thread gets the total
+__device__ __forceinline__ uint32_t rows_block_sum(uint32_t v, uint32_t* red) {
+  v = __reduce_add_sync(0xffffffffu, v);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  const uint32_t t = __reduce_add_sync(0xffffffffu, (threadIdx.x & 31) < RT_ROWS / 32 ? red[threadIdx.x & 31] : 0u);
+  __syncthreads();
+  return t;
+}
+
+// Encoder: (c_s, f_s) of the true symbol s of selected row j of window c:
+// c_s = s + sum_{v<s} floor(w_v R / W) + (top < s ? D : 0), f_s = 1 + floor(w_s R / W) + (s == top ? D : 0),
+// D = R - sum_v floor(w_v R / W).
+__global__ void __launch_bounds__(RT_ROWS) enc_rows_kernel(CodeArgs a) {
+  __shared__ uint32_t T[256];
+  __shared__ uint32_t tabf[QW0 + 1];
+  __shared__ uint32_t red[RT_ROWS / 32];
+  const int c = blockIdx.y, j = blockIdx.x;
+  if (j >= a.sel_count[c]) return;
+  for (int i = threadIdx.x; i < 256; i += RT_ROWS) T[i] = c_exp_table_c[i];
+  const int pos = a.sel_pos[(size_t)c * a.kcap + j];
+  const size_t row = selected_row(a, c, j, pos);
+  const int V = a.V, sym = a.symbols[(size_t)c * a.L + pos];
+  const float* lr = a.logits + row * V;
+  const float m = a.mx[row];
+  const uint64_t Wr = a.W[row];
+  const int top = a.top[row];
+  const uint32_t R = (1u << a.P) - (uint32_t)V;
+  __syncthreads();
+  const RowFloor flo = row_floor(tabf, T, R, Wr, V);
+  uint32_t s_all = 0, s_lt = 0;
+  if ((V & 3) == 0 && (reinterpret_cast<uintptr_t>(lr) & 15) == 0) {
+    const float4* l4 = reinterpret_cast<const float4*>(lr);
+    for (int i = threadIdx.x; i < (V >> 2); i += RT_ROWS) {
+      const float4 x = l4[i];
+      const int v = 4 * i;
+      const uint32_t f0 = flo(m, x.x), f1 = flo(m, x.y), f2 = flo(m, x.z), f3 = flo(m, x.w);
+      s_all += f0 + f1 + f2 + f3;
+      s_lt += (v < sym ? f0 : 0u) + (v + 1 < sym ? f1 : 0u) + (v + 2 < sym ? f2 : 0u) + (v + 3 < sym ? f3 : 0u);
+    }
+  } else {
+    for (int v = threadIdx.x; v < V; v += RT_ROWS) {
+      const uint32_t f = flo(m, lr[v]);
+      s_all += f;
+      s_lt += v < sym ? f : 0u;
+    }
+  }
+  s_all = rows_block_sum(s_all, red);
+  s_lt = rows_block_sum(s_lt, red);
+  if (threadIdx.x == 0) {
+    const uint32_t D = R - s_all;
+    const uint64_t cs = (uint64_t)sym + s_lt + (top < sym ? D : 0u);
+    const uint64_t fs = 1ull + flo(m, lr[sym]) + (sym == top ? D : 0u);
+    a.rowcf[(size_t)c * a.kcap + j] = (cs << 32) | fs;
+  }
+}
+
+// Encoder, per window (one thread): code the window's selected symbols in ascending position.
+__global__ void enc_seq_kernel(CodeArgs a, int n_chunks) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n_chunks) return;
+  const int n = a.sel_count[c];
+  CoderState t = a.state_c[c];
+  uint8_t* ebuf = a.bytes + (size_t)c * a.cap_bytes;
+  for (int j = 0; j < n; ++j) {
+    const int pos = a.sel_pos[(size_t)c * a.kcap + j];
+    const uint64_t cf = a.rowcf[(size_t)c * a.kcap + j];
+    const uint64_t cs = cf >> 32, fs = cf & 0xFFFFFFFFull;
+    if (a.coder == 1) {  // buffered; coded in reverse when the window is finished
+      if (t.n_units < (uint32_t)a.pair_cap) a.pairs[(size_t)c * a.pair_cap + t.n_units] = (cs << 32) | fs;
+      else atomicOr(a.err, ERR_CAPACITY);
+      t.n_units++;
+    } else {
+      enc_symbol(t, ebuf, a.cap_bytes / 2, a.P, cs, fs, a.err);
+    }
+    a.state[(size_t)c * a.L + pos] = a.symbols[(size_t)c * a.L + pos];
+  }
+  a.state_c[c] = t;
+  if (a.committed) a.committed[c] = n;
+}
+
+// Decoder, per selected row: the row's coarse CDF (prefix sums of 1 + floor(w R / W) at the starts
+// of its segments of CODE_SEG elements, without D), D and K = floor(R 2^64 / W).
+__global__ void __launch_bounds__(RT_ROWS) dec_rows_kernel(CodeArgs a) {
+  __shared__ uint32_t T[256];
+  __shared__ uint32_t tabf[QW0 + 1];
+  __shared__ uint32_t wtot[RT_ROWS / 32];
+  const int c = blockIdx.y, j = blockIdx.x;
+  if (j >= a.sel_count[c]) return;
+  for (int i = threadIdx.x; i < 256; i += RT_ROWS) T[i] = c_exp_table_c[i];
+  const int pos = a.sel_pos[(size_t)c * a.kcap + j];
+  const size_t row = selected_row(a, c, j, pos);
+  const int V = a.V, nseg = a.nseg;
+  const float* lr = a.logits + row * V;
+  const float m = a.mx[row];
+  const uint64_t Wr = a.W[row];
+  const uint32_t R = (1u << a.P) - (uint32_t)V;
+  const size_t cj = (size_t)c * a.kcap + j;
+  uint32_t* cum = a.segcum + cj * (nseg + 1);
+  __syncthreads();
+  const RowFloor flo = row_floor(tabf, T, R, Wr, V);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool vec = (V & 3) == 0 && (reinterpret_cast<uintptr_t>(lr) & 15) == 0;
+  // segment sums, one warp per segment (coalesced)
+  for (int sg = warp; sg < nseg; sg += RT_ROWS / 32) {
+    const int base = sg * CODE_SEG;
+    uint32_t sum = 0;
+    if (vec) {
+      const float4* l4 = reinterpret_cast<const float4*>(lr + base);
+#pragma unroll
+      for (int i = 0; i < CODE_SEG / 128; ++i) {
+        const int e = 4 * (lane + 32 * i);
+        if (base + e < V) {  // V % 4 == 0: the float4 is wholly in the row
+          const float4 x = l4[lane + 32 * i];
+          sum += 4u + flo(m, x.x) + flo(m, x.y) + flo(m, x.z) + flo(m, x.w);
+        }
+      }
+    } else {
+      for (int e = lane; e < CODE_SEG; e += 32)
+        if (base + e < V) sum += 1u + flo(m, lr[base + e]);
+    }
+    sum = __reduce_add_sync(0xffffffffu, sum);
+    if (lane == 0) cum[sg] = sum;
+  }
+  __syncthreads();  // the segment sums are visible to the block
+  // exclusive prefix over the segments, RT_ROWS at a time
+  uint32_t carry = 0;
+  for (int s0 = 0; s0 < nseg; s0 += RT_ROWS) {
+    const int sg = s0 + threadIdx.x;
+    const uint32_t v = sg < nseg ? cum[sg] : 0u;
+    uint32_t inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += t;
+    }
+    if (lane == 31) wtot[warp] = inc;
+    __syncthreads();
+    const uint32_t tv = lane < RT_ROWS / 32 ? wtot[lane] : 0u;
+    const uint32_t pre = carry + __reduce_add_sync(0xffffffffu, lane < warp ? tv : 0u) + inc - v;
+    carry += __reduce_add_sync(0xffffffffu, tv);
+    if (sg < nseg) cum[sg] = pre;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    cum[nseg] = carry;                      // V + sum_v floor(w_v R / W)
+    a.rowD[cj] = (1u << a.P) - carry;       // = R - sum_v floor(w_v R / W)
+    a.rowK[cj] = flo.table ? recip_scaled(R, Wr) : flo.K;
+  }
+}
+
+// Decoder, one warp per window: for each selected row in ascending position, the slot from the
+// coder state, the segment holding it (a search over the coarse CDF), the symbol inside that
+// segment (a warp scan of its frequencies), then the coder update.
+constexpr int DEC_WARPS = 4;
+__global__ void __launch_bounds__(32 * DEC_WARPS) dec_seq_kernel(CodeArgs a, int n_chunks) {
+  __shared__ uint32_t T[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) T[i] = c_exp_table_c[i];
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x * DEC_WARPS + (threadIdx.x >> 5);
+  if (c >= n_chunks) return;  // warp-uniform
+  const int n = a.sel_count[c], V = a.V, P = a.P, nseg = a.nseg;
+  const uint32_t R = (1u << P) - (uint32_t)V;
+  const uint8_t* dbuf = a.in_bytes + (a.in_offsets ? a.in_offsets[c] : 0);
+  const uint64_t dn = (a.in_bits[c] + 7) / 8;
+  CoderState st = a.state_c[c];  // every lane keeps a copy; lane 0's updates are broadcast
+  for (int j = 0; j < n; ++j) {
+    const int pos = a.sel_pos[(size_t)c * a.kcap + j];
+    const size_t row = selected_row(a, c, j, pos);
+    const size_t cj = (size_t)c * a.kcap + j;
+    const float* lr = a.logits + row * V;
+    const float m = a.mx[row];
+    const uint64_t Wr = a.W[row], K = a.rowK[cj];
+    const uint32_t D = a.rowD[cj];
+    const int top = a.top[row];
+    const uint32_t* cum = a.segcum + cj * (nseg + 1);
+    uint64_t slot;
+    if (a.coder == 1) {
+      slot = st.low & ((1ull << P) - 1);  // x mod 2^P
+    } else {
+      slot = st.low / (st.rng >> P);     // the decoder keeps val = code - low in .low
+      if (slot >= (1ull << P)) {
+        if (lane == 0) atomicOr(a.err, ERR_CORRUPT);
+        slot = (1ull << P) - 1;
+      }
+    }
+    // CDF at the start of segment s: cum[s] + D when the top element lies before it
+    auto start = [&](int sg) -> uint64_t { return (uint64_t)cum[sg] + ((int64_t)sg * CODE_SEG > top ? D : 0u); };
+    int lo = 0, hi = nseg;  // start(lo) <= slot; the answer is in [lo, hi)
+    while (hi - lo > 1) {
+      const int step = (hi - lo + 31) / 32;
+      const int sg = lo + lane * step;
+      const bool le = sg < hi && start(sg) <= slot;
+      const unsigned b = __ballot_sync(0xffffffffu, le);
+      const int l = 31 - __clz(b);  // lane 0 always qualifies (start(lo) <= slot)
+      lo = lo + l * step;
+      hi = min(hi, lo + step);
+    }
+    // the symbol inside segment lo
+    const int base = lo * CODE_SEG;
+    uint64_t cb = start(lo);
+    int sym = -1;
+    uint64_t cs = 0, fs = 1;
+    for (int e0 = 0; e0 < CODE_SEG && sym < 0; e0 += 32) {
+      const int v = base + e0 + lane;
+      uint32_t f = 0;
+      if (v < V) {
+        const uint32_t q = code_index(__fsub_rn(m, lr[v]));
+        f = 1u + (q < (uint32_t)QW0 ? floor_wr_over_w(quant_w(T, (int)q), R, Wr, K) : 0u) + (v == top ? D : 0u);
+      }
+      uint32_t inc = f;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += t;
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, v < V && cb + inc > slot);
+      if (hit) {
+        const int l = __ffs(hit) - 1;
+        const uint32_t incl = __shfl_sync(0xffffffffu, inc, l), fl = __shfl_sync(0xffffffffu, f, l);
+        sym = base + e0 + l;
+        cs = cb + incl - fl;
+        fs = fl;
+      }
+      cb += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    if (sym < 0) {  // only for a damaged stream: the slot lies beyond the row's total
+      if (lane == 0) atomicOr(a.err, ERR_CORRUPT);
+      sym = 0;
+      cs = 0;
+      fs = 1;
+    }
+    if (a.coder == 1) {
+      st.low = fs * (st.low >> P) + slot - cs;
+      if (st.low < RANS_L) {
+        st.low = (st.low << 32) | word_at(dbuf, dn, 8 + 4ull * st.n_units);
+        st.n_units++;
+      }
+    } else {
+      const uint64_t r = st.rng >> P;
+      st.low -= r * cs;
+      st.rng = r * fs;
+      while (st.rng < RENORM) {
+        st.low = (st.low << 16) | unit_at(dbuf, dn, st.n_units++);
+        st.rng <<= 16;
+      }
+    }
+    if (lane == 0) a.state[(size_t)c * a.L + pos] = sym;
+  }
+  if (lane == 0) {
+    a.state_c[c] = st;
+    if (a.committed) a.committed[c] = n;
+  }
+}
+
 int code_step(const CodeArgs& a, bool decode, int n_chunks, cudaStream_t s) {
   if (n_chunks == 0) return DLMZ_OK;
   ProfScope prof(PROF_CODE, s, 0, 0);
-  if (decode) code_kernel<true><<<n_chunks, CT, 0, s>>>(a);
-  else code_kernel<false><<<n_chunks, CT, 0, s>>>(a);
+  const bool rows = a.coder != 2 && a.kcap > 0 && a.kcap <= 65535 && (decode ? (a.segcum && a.rowK && a.rowD) : a.rowcf != nullptr);
+  if (!rows) {  // symbol ranks: one CTA per window does everything
+    if (decode) code_kernel<true><<<n_chunks, CT, 0, s>>>(a);
+    else code_kernel<false><<<n_chunks, CT, 0, s>>>(a);
+    return launch_status();
+  }
+  const dim3 grid((unsigned)a.kcap, (unsigned)n_chunks);
+  if (n_chunks > 65535) return DLMZ_EINVAL;
+  if (!decode) {
+    enc_rows_kernel<<<grid, RT_ROWS, 0, s>>>(a);
+    DLMZ_TRY(launch_status());
+    enc_seq_kernel<<<(n_chunks + 127) / 128, 128, 0, s>>>(a, n_chunks);
+  } else {
+    dec_rows_kernel<<<grid, RT_ROWS, 0, s>>>(a);
+    DLMZ_TRY(launch_status());
+    dec_seq_kernel<<<(n_chunks + DEC_WARPS - 1) / DEC_WARPS, 32 * DEC_WARPS, 0, s>>>(a, n_chunks);
+  }
   return launch_status();
 }
 

@@ -40,7 +40,15 @@ struct CodeArgs {
   int pair_cap;
   const int32_t* row_map;    // optional [n_chunks x rpc]: row of logits / mx / W / top of each candidate
   int sel_major;             // without row_map: row of the j-th selected position = c * kcap + j
+  // scratch of the row-parallel range / rANS path, [n_chunks x kcap] selected rows:
+  uint64_t* rowcf;           // encoder: (c_s << 32) | f_s of each selected row
+  uint32_t* segcum;          // decoder: per row nseg + 1 prefix sums of 1 + floor(w R / W) at segment starts
+  uint64_t* rowK;            // decoder: floor(R 2^64 / W) of each selected row
+  uint32_t* rowD;            // decoder: the remainder D of each selected row
+  int nseg;                  // decoder: segments of CODE_SEG elements per row
 };
+
+constexpr int CODE_SEG = 512;  // elements per segment of a row's coarse CDF (decoder)
 
 // keys of window c's position row0 + i: keys[row_map[c * rpc + i]] when row_map is
 // given (candidates only), else keys[c * rpc + i].

@@ -263,6 +263,7 @@ struct BatchContext {
 // ---- per-batch step state ---------------------------------------------------------
 struct StepBufs {
   DevBuf logits, W, Hq, top, mx, sel_count, sel_pos, committed, sum, pairs;
+  DevBuf rowcf, segcum, rowK, rowD;  // row-parallel coder scratch, one entry per selected row
   // candidate rows of a model step: per-window counts, offsets [nc + 1], token index of
   // each candidate, the candidate row of each position of [row0, row0 + rpc) (-1: none),
   // token index of each selected row and the stats of the recomputed selected rows
@@ -496,6 +497,21 @@ static int code_rows(StepBufs& sb, const StepIO& io, const float* logits, const 
     DLMZ_TRY(sb.pairs.ensure((size_t)nc * L * 8));
     a.pairs = sb.pairs.as<uint64_t>();
     a.pair_cap = L;
+  }
+  if (pol.coder != DLMZ_CODER_RANKS) {
+    const size_t nrows = (size_t)nc * kcap;
+    a.nseg = (V + CODE_SEG - 1) / CODE_SEG;
+    if (io.decode) {
+      DLMZ_TRY(sb.segcum.ensure(nrows * (a.nseg + 1) * 4));
+      DLMZ_TRY(sb.rowK.ensure(nrows * 8));
+      DLMZ_TRY(sb.rowD.ensure(nrows * 4));
+      a.segcum = sb.segcum.as<uint32_t>();
+      a.rowK = sb.rowK.as<uint64_t>();
+      a.rowD = sb.rowD.as<uint32_t>();
+    } else {
+      DLMZ_TRY(sb.rowcf.ensure(nrows * 8));
+      a.rowcf = sb.rowcf.as<uint64_t>();
+    }
   }
   return code_step(a, io.decode, nc, s);
 }

@@ -30,8 +30,8 @@ CASES = [
     (2048, 1, 28, 4, 128, "drift"),  # tcgen05 head_dim 128: the 7B-shaped 7:1 GQA at windows of 2048
     (256, 3, 8, 2, 128, "flat"),     # tcgen05 head_dim 128: small scores, 4:1 GQA
     (128, 160, 2, 1, 128, "drift"),  # tcgen05 head_dim 128: 320 one-tile items, ~2 per persistent CTA
-    (256, 400, 2, 1, 64, "drift"),   # tcgen05, two query tiles per CTA: 800 items, ~5 per persistent CTA
-    (512, 160, 2, 2, 128, "drift"),  # the same at head_dim 128: 640 items of 4 key tiles
+    (256, 400, 2, 1, 64, "drift"),   # tcgen05 one-tile kernel: 1600 items, ~5 per persistent CTA
+    (512, 160, 2, 2, 128, "drift"),  # tcgen05 head_dim 128, two query tiles per CTA: 640 items of 4 key tiles
     (96, 2, 4, 2, 64, "drift"),      # CUDA-core mma kernel (L % 128 != 0)
     (64, 2, 2, 1, 128, "drift"),     # CUDA-core mma kernel, head_dim 128
     (40, 3, 4, 2, 32, "drift"),      # CUDA-core scalar kernel, head_dim 32
