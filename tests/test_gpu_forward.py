@@ -50,7 +50,10 @@ def test_gemm_tensor_core_vs_float64(dev):
     import torch
     d = dlmz()
     rng = np.random.default_rng(3)
-    for (M, N, K) in [(128, 256, 64), (300, 512, 192), (1000, 768, 512), (77, 256, 2048)]:
+    # the last two cases give each persistent CTA several tiles, so both accumulators and every
+    # ring stage turn over many times
+    for (M, N, K) in [(128, 256, 64), (300, 512, 192), (1000, 768, 512), (77, 256, 2048), (8192, 2048, 256),
+                      (2560, 1280, 1024)]:
         A = torch.from_numpy(rng.normal(size=(M, K)).astype(np.float32)).to(torch.bfloat16)
         B = torch.from_numpy(rng.normal(size=(N, K)).astype(np.float32)).to(torch.bfloat16)
         ref = A.double() @ B.double().T
