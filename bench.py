@@ -23,7 +23,9 @@ input bytes coded (and decoded) per step x K / the summed time; compress and
 decompress are also reported separately.
 
 ``secondary`` holds the small byte-level workload (8 layers, d = 512, V =
-256; one 512 KiB batch compressed and decompressed per step) and the
+256; one 512 KiB batch compressed and decompressed per step), a timed prefix
+of the 7B GQA-shaped entropy-schedule workload (64 windows of 2048 tokens,
+V = 152064; two denoising steps each way) and the
 isolated quantise + select workload (65536 x 126464 float32 logits, 24-bit
 CDFs plus scores, top-32 of groups of 1024) at full size.
 
@@ -397,6 +399,68 @@ def run_c4(args, dlmz, torch, rank, ws, dev):
     }
 
 
+C5 = dict(n_layers=28, d=3584, n_heads=28, n_kv_heads=4, ffn=18944, vocab=152064, seed=0)
+C5_CHUNK, C5_BATCH, C5_TAU, C5_KMIN, C5_KMAX = 2048, 64, 0.5, 1, 64
+
+
+def secondary_c5(dlmz, torch, dev, steps=2, warmup=1):
+    """The 7B GQA-shaped workload, a timed prefix: one batch of 64 windows of 2048 tokens, entropy
+    threshold 0.5 bits (at least 1, at most 64 positions per step); `warmup` + `steps` denoising
+    steps of compression, then the same steps of decompression (which must reproduce the state)."""
+    import numpy as np
+    from paper_2608_11249_gb300 import sources
+    stream = torch.cuda.current_stream().cuda_stream
+    V, L, nc = C5["vocab"], C5_CHUNK, C5_BATCH
+    m = dlmz.Model(C5["n_layers"], C5["d"], C5["n_heads"], C5["n_kv_heads"], C5["ffn"], V, dlmz.BF16, seed=C5["seed"])
+    sym = torch.from_numpy(sources.zipf_bigram_tokens(nc * L, V, seed=0).astype(np.int32).reshape(nc, L)).to(dev)
+    state = torch.full((nc, L), V, dtype=torch.int32, device=dev)
+    committed = torch.zeros(nc, dtype=torch.int32, device=dev)
+    pol = dlmz.policy(dlmz.ENTROPY, 0, 0, C5_TAU, C5_KMIN, C5_KMAX)
+    enc = dlmz.Coder(nc, L, V, 24)
+    enc.reset_encoder()
+
+    def run(fn):
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        tot = torch.zeros(nc, dtype=torch.int64, device=dev)
+        e0, e1 = _events()
+        e0.record()
+        for _ in range(steps):
+            fn()
+            tot.add_(committed)  # tokens revealed by this step
+        e1.record()
+        e1.synchronize()
+        return e0.elapsed_time(e1), int(tot.sum().item())
+
+    enc_ms, enc_tok = run(lambda: m.encode_step(enc, pol, 0, L, sym.data_ptr(), state.data_ptr(), committed.data_ptr(),
+                                                stream))
+    enc_state = state.clone()
+    bits = torch.empty(nc, dtype=torch.int32, device=dev)
+    cap = enc.capacity_units * 2
+    raw = torch.zeros(nc * cap, dtype=torch.uint8, device=dev)
+    enc.finish(bits.data_ptr(), raw.data_ptr(), 0, stream)
+    offs = (torch.arange(nc, dtype=torch.int64, device=dev) * cap).contiguous()
+    dec = dlmz.Coder(nc, L, V, 24)
+    dec.load_decoder(raw.data_ptr(), offs.data_ptr(), bits.data_ptr(), stream)
+    state.fill_(V)
+    dec_ms, dec_tok = run(lambda: m.decode_step(dec, pol, 0, L, state.data_ptr(), committed.data_ptr(), stream))
+    dlmz.check(stream)
+    assert torch.equal(state, enc_state), "decoder state differs from the encoder's"
+    enc.close()
+    dec.close()
+    m.close()
+    del raw, state, enc_state, sym
+    torch.cuda.empty_cache()
+    return {"workload": "7B GQA-shaped masked DLM, bf16, random-init: 28 layers d=3584 28/4 heads FFN 18944 "
+                        "V=152064; 64 windows of 2048 Zipf-bigram tokens, entropy threshold 0.5 bits, at least 1 and "
+                        "at most 64 positions per step (a timed prefix of the workload)",
+            "compress_Bps": 4.0 * enc_tok / (enc_ms / 1000.0), "decompress_Bps": 4.0 * dec_tok / (dec_ms / 1000.0),
+            "ms_per_denoising_step": {"compress": enc_ms / steps, "decompress": dec_ms / steps},
+            "tokens_per_step": enc_tok / float(steps), "steps": steps, "warmup": warmup,
+            "note": "random-init weights: no position reaches 0.5 bits, so each step reveals m = 1 token per window"}
+
+
 def secondary_c2(dlmz, torch, dev, steps=2):
     """The byte workload: one 512 KiB batch compressed + decompressed per step (1 warm-up step)."""
     import numpy as np
@@ -507,6 +571,8 @@ def run(args):
     if not args.no_secondary:
         torch.cuda.empty_cache()
         secondary["byte_workload"] = secondary_c2(dlmz, torch, dev)
+        torch.cuda.empty_cache()
+        secondary["gqa_7b_prefix"] = secondary_c5(dlmz, torch, dev)
         torch.cuda.empty_cache()
         secondary["quantize_select"] = secondary_c3(dlmz, torch, dev, hbm)
     line = {

@@ -10,10 +10,11 @@
         the quantiser (CDF + scores) on spiked N(0,3) logits rows
     python -m paper_2608_11249_gb300.kernel_bench gemm --m 32768 --n 4096 --k 512
         one bf16 tensor-core GEMM with float32 output
-    python -m paper_2608_11249_gb300.kernel_bench step --layers 1 --chunks 16
+    python -m paper_2608_11249_gb300.kernel_bench step --layers 1 --chunks 16 [--decode]
         one denoising step of compression (forward, LM head and quantiser on the
         candidates, selection, range coding of 16 tokens per window) of the
-        8B-shaped model with `layers` layers over `chunks` windows of 1024 tokens
+        8B-shaped model with `layers` layers over `chunks` windows of 1024 tokens;
+        --decode: one step is compressed untimed, then its decompression is timed
 
 Prints the mean CUDA-event time per repetition.
 """
@@ -45,6 +46,7 @@ def main():
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--model", choices=["byte", "8b"], default="byte")
     ap.add_argument("--layers", type=int, default=2)
+    ap.add_argument("--decode", action="store_true")
     a = ap.parse_args()
     torch.cuda.set_device(0)
     g = torch.Generator(device="cuda").manual_seed(0)
@@ -52,6 +54,7 @@ def main():
         from paper_2608_11249_gb300 import sources
         V, L, k = 126464, 1024, 16
         m = dlmz.Model(a.layers, 4096, 32, 32, 12288, V, dlmz.BF16, seed=0)
+        m.set_logits_budget(2 << 30)  # candidate logits in slabs of 2 GiB (small device footprint)
         sym = torch.from_numpy(sources.zipf_bigram_tokens(a.chunks * L, V, seed=0).astype(np.int32)).cuda()
         state = torch.full((a.chunks, L), V, dtype=torch.int32, device="cuda")
         enc = dlmz.Coder(a.chunks, L, V, 24)
@@ -59,6 +62,18 @@ def main():
         pol = dlmz.policy(dlmz.TOPK_CONF, k, 0)
         a.reps = min(a.reps, L // k - 1)
         fn = lambda: m.encode_step(enc, pol, 0, L, sym.data_ptr(), state.data_ptr())
+        if a.decode:  # compress 1 + reps steps, then time their decompression (1 untimed + reps)
+            for _ in range(1 + a.reps):
+                fn()
+            bits = torch.empty(a.chunks, dtype=torch.int32, device="cuda")
+            cap = enc.capacity_units * 2
+            raw = torch.zeros(a.chunks * cap, dtype=torch.uint8, device="cuda")
+            enc.finish(bits.data_ptr(), raw.data_ptr())
+            offs = torch.arange(a.chunks, dtype=torch.int64, device="cuda") * cap
+            dec = dlmz.Coder(a.chunks, L, V, 24)
+            dec.load_decoder(raw.data_ptr(), offs.data_ptr(), bits.data_ptr())
+            state.fill_(V)
+            fn = lambda: m.decode_step(dec, pol, 0, L, state.data_ptr())
     elif a.what == "forward" and a.model == "8b":
         V, L, rpc = 126464, 1024, 16
         m = dlmz.Model(a.layers, 4096, 32, 32, 12288, V, dlmz.BF16, seed=0)
