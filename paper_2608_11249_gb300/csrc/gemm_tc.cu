@@ -140,6 +140,8 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
   }
   // fused RMSNorm, producer side: sums of x^2 of the rows this lane stores
   float rowsum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  // float32 epilogue: this thread's row maximum (NaN-propagating) and minimum over its 128 columns
+  float pmx = -INFINITY, pmn = INFINITY;
   EpiAux cur, nxt;
   if constexpr (EPI == EPI_RESID_F32) epi_load_aux<EPI>(cur, c0, lane, row0, M, n0, ep);
   // RoPE: a warp takes every other chunk (c = half, half + 2, ...), so with head_dim 64 all its
@@ -159,6 +161,15 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
     }
     float v[32];
     tmem_ld32(tbase + c * 32, v);
+    if constexpr (EPI == EPI_F32) {
+      if (ep.pmax) {
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          asm("max.NaN.f32 %0, %1, %2, %3;" : "=f"(pmx) : "f"(pmx), "f"(v[i]), "f"(v[i + 1]));
+          asm("min.f32 %0, %1, %2, %3;" : "=f"(pmn) : "f"(pmn), "f"(v[i]), "f"(v[i + 1]));
+        }
+      }
+    }
     if constexpr (EPI == EPI_SWIGLU_BF16) {  // columns [0,128) gate, [128,256) up of the same features
       float u[32];
       tmem_ld32(tbase + BN / 2 + c * 32, u);
@@ -254,6 +265,14 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tacc, int q, int half, in
     }
     __syncwarp();
     if constexpr (EPI == EPI_RESID_F32) cur = nxt;
+  }
+  if constexpr (EPI == EPI_F32) {
+    const int m = row0 + lane;
+    if (ep.pmax && m < M) {  // this thread's row; part = 128-column block of the output
+      const int n_part = ep.n_part, part = n0 / 128 + half;
+      ep.pmax[(size_t)m * n_part + part] = pmx;
+      ep.pmin[(size_t)m * n_part + part] = pmn;
+    }
   }
   if constexpr (EPI == EPI_RESID_F32) {
     if (ep.ssq_out && (lane & 7) == 0) {

@@ -39,6 +39,10 @@ struct GemmEpilogue {
   int n_part;
   int d_model;
   float eps;
+  // Float32 epilogue (LM head): if set, each row's maximum (NaN-propagating) and minimum over
+  // every 128 output columns, into [rows x N / 128] each -- the quantiser's first pass.
+  float* pmax;
+  float* pmin;
 };
 
 // tcgen05 path: N % 256 == 0, K % 64 == 0, 16-byte aligned operands.
@@ -91,6 +95,7 @@ int attention_bf16_mma(const bf16* qkv, int ld, int n_chunks, int L, int n_heads
 
 // ---- quantiser / selector / coder --------------------------------------------------
 int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, uint64_t* W,
-                  uint64_t* A, int32_t* Hq, int32_t* top, float* mx, cudaStream_t s);
+                  uint64_t* A, int32_t* Hq, int32_t* top, float* mx, cudaStream_t s,
+                  const float* pmax = nullptr, const float* pmin = nullptr);
 
 }  // namespace dlmz

@@ -271,7 +271,7 @@ static int layers_impl(dlmz_model* m, const int32_t* state, int nc, int L, cudaS
 // (r / rpc) * L + row0 + r % rpc) and f32 logits [R x V].
 template <typename T>
 static int head_impl(dlmz_model* m, const int32_t* idx, int R, int L, int row0, int rpc, float* logits,
-                     cudaStream_t s) {
+                     cudaStream_t s, float* pmax = nullptr, float* pmin = nullptr, bool* parts = nullptr) {
   const dlmz_model_config& c = m->cfg;
   const int d = c.d, V = c.vocab;
   if (R == 0) return DLMZ_OK;
@@ -283,6 +283,14 @@ static int head_impl(dlmz_model* m, const int32_t* idx, int R, int L, int row0, 
   GemmEpilogue ep{};
   ep.out = logits;
   ep.ldo = V;
+  // the tensor-core epilogue can also leave each row's maxima and minima per 128 columns
+  const bool tc = sizeof(T) == 2 && gemm_tc_supported(R, V, d);
+  if (parts) *parts = tc && pmax && pmin;
+  if (tc && pmax && pmin) {
+    ep.pmax = pmax;
+    ep.pmin = pmin;
+    ep.n_part = V / 128;
+  }
   return gemm<T>(hc, reinterpret_cast<const T*>(m->head), R, V, d, EPI_F32, ep, s);
 }
 
@@ -298,9 +306,11 @@ int model_layers(dlmz_model* m, const int32_t* state, int nc, int L, cudaStream_
   return layers_impl<float>(m, state, nc, L, s);
 }
 
-int model_head(dlmz_model* m, const int32_t* idx, int n, float* logits, cudaStream_t s) {
+int model_head(dlmz_model* m, const int32_t* idx, int n, float* logits, cudaStream_t s, float* pmax, float* pmin,
+               bool* parts) {
+  if (parts) *parts = false;
   if (n < 0 || (n > 0 && (!idx || !logits))) return DLMZ_EINVAL;
-  if (m->bf16) return head_impl<bf16>(m, idx, n, 0, 0, 0, logits, s);
+  if (m->bf16) return head_impl<bf16>(m, idx, n, 0, 0, 0, logits, s, pmax, pmin, parts);
   return head_impl<float>(m, idx, n, 0, 0, 0, logits, s);
 }
 

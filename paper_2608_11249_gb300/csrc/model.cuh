@@ -70,8 +70,11 @@ int model_layers(dlmz_model* m, const int32_t* state, int n_chunks, int L, cudaS
 // LM head on n rows of the last model_layers batch: final RMSNorm of the
 // residual rows idx[0..n) (token index = window * L + position) and float32
 // logits [n x V].  Each row's logits depend only on that row, so a row gives
-// bit-identical logits in any call and at any place in idx.
-int model_head(dlmz_model* m, const int32_t* idx, int n, float* logits, cudaStream_t s);
+// bit-identical logits in any call and at any place in idx.  pmax / pmin (optional,
+// [n x V / 128]): on the tensor-core path each row's maximum (NaN-propagating) and
+// minimum per 128 logits, for the quantiser; *parts tells whether they were written.
+int model_head(dlmz_model* m, const int32_t* idx, int n, float* logits, cudaStream_t s, float* pmax = nullptr,
+               float* pmin = nullptr, bool* parts = nullptr);
 // Every layer's head-averaged attention probabilities [n_layers][n_chunks][L][L]
 // for the windows' states (no LM head).
 int model_attention_maps(dlmz_model* m, const int32_t* state, int n_chunks, int L, float* maps, cudaStream_t s);

@@ -264,6 +264,7 @@ struct BatchContext {
 struct StepBufs {
   DevBuf logits, W, Hq, top, mx, sel_count, sel_pos, committed, sum, pairs;
   DevBuf rowcf, segcum, rowK, rowD;  // row-parallel coder scratch, one entry per selected row
+  DevBuf pmax, pmin;                 // LM-head rows' maxima / minima per 128 logits (the quantiser's first pass)
   // candidate rows of a model step: per-window counts, offsets [nc + 1], token index of
   // each candidate, the candidate row of each position of [row0, row0 + rpc) (-1: none),
   // token index of each selected row and the stats of the recomputed selected rows
@@ -576,11 +577,24 @@ static int model_step(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int
   DLMZ_TRY(sb.ensure(mrows, 0, nc, kcap));  // scores of every candidate, selection buffers
   DLMZ_TRY(sb.logits.ensure((slabbed ? (size_t)slab : mrows) * V * 4));
   float* logits = sb.logits.as<float>();
+  // the head's epilogue leaves each row's maxima per 128 logits, so the quantiser reads each logit
+  // once (large vocabularies: V > 512 takes the persistent kernel)
+  const bool want_parts = V > 512 && V % 128 == 0;
+  const size_t head_rows = slabbed ? (size_t)slab : mrows;
+  if (want_parts) {
+    const size_t np = head_rows < (size_t)sel_rows ? (size_t)sel_rows : head_rows;
+    DLMZ_TRY(sb.pmax.ensure(np * (V / 128) * 4));
+    DLMZ_TRY(sb.pmin.ensure(np * (V / 128) * 4));
+  }
+  float* pmx = want_parts ? sb.pmax.as<float>() : nullptr;
+  float* pmn = want_parts ? sb.pmin.as<float>() : nullptr;
   for (int64_t r0 = 0; r0 < M; r0 += slab) {
     const int n = (int)(M - r0 < slab ? M - r0 : slab);
-    DLMZ_TRY(model_head(m, cand + r0, n, logits, s));
+    bool parts = false;
+    DLMZ_TRY(model_head(m, cand + r0, n, logits, s, pmx, pmn, &parts));
     DLMZ_TRY(quantize_rows(logits, n, V, P, nullptr, sb.W.as<uint64_t>() + r0, nullptr, sb.Hq.as<int32_t>() + r0,
-                           sb.top.as<int32_t>() + r0, sb.mx.as<float>() + r0, s));
+                           sb.top.as<int32_t>() + r0, sb.mx.as<float>() + r0, s, parts ? pmx : nullptr,
+                           parts ? pmn : nullptr));
   }
   DLMZ_TRY(select_step(sb, io.state, nc, L, V, pol, row0, rpc, kcap, row_map, s));
   if (!slabbed)
@@ -592,9 +606,10 @@ static int model_step(dlmz_model* m, StepBufs& sb, const dlmz_k_policy& pol, int
   sel_tok_kernel<<<grid_for(sel_rows), 256, 0, s>>>(sb.sel_count.as<int32_t>(), sb.sel_pos.as<int32_t>(), nc, L, kcap,
                                                    stok);
   DLMZ_TRY(launch_status());
-  DLMZ_TRY(model_head(m, stok, (int)sel_rows, logits, s));
+  bool parts = false;
+  DLMZ_TRY(model_head(m, stok, (int)sel_rows, logits, s, pmx, pmn, &parts));
   DLMZ_TRY(quantize_rows(logits, (int)sel_rows, V, P, nullptr, sb.sW.as<uint64_t>(), nullptr, sb.sHq.as<int32_t>(),
-                         sb.stop.as<int32_t>(), sb.smx.as<float>(), s));
+                         sb.stop.as<int32_t>(), sb.smx.as<float>(), s, parts ? pmx : nullptr, parts ? pmn : nullptr));
   return code_rows(sb, io, logits, sb.smx.as<float>(), sb.sW.as<uint64_t>(), sb.stop.as<int32_t>(), nullptr, true, nc,
                    L, V, P, pol, row0, rpc, kcap, s);
 }

@@ -295,7 +295,8 @@ template <int NT, int CPS>
 __global__ void __launch_bounds__(NT, CPS)
     quantize_persist_kernel(const float* __restrict__ logits, int rows, int V, int P, uint32_t* __restrict__ cdf,
                             uint64_t* __restrict__ Wout, uint64_t* __restrict__ Aout, int32_t* __restrict__ Hq,
-                            int32_t* __restrict__ topout, float* __restrict__ mxout, int* err) {
+                            int32_t* __restrict__ topout, float* __restrict__ mxout, int* err,
+                            const float* __restrict__ pmax, const float* __restrict__ pmin, int npart) {
   constexpr int NW = NT / 32;
   static_assert(NT % 32 == 0 && NW <= 32 && NQ % NT == 0, "block shape");
   __shared__ uint32_t T[256];
@@ -313,9 +314,16 @@ __global__ void __launch_bounds__(NT, CPS)
   const uint32_t R = (1u << P) - (uint32_t)V;
   for (int r = blockIdx.x; r < rows; r += gridDim.x) {
     const float4* l4 = reinterpret_cast<const float4*>(logits + (size_t)r * V);
-    // pass 1 (HBM): max; x - x is NaN exactly for non-finite x
+    // pass 1 (HBM): max; x - x is NaN exactly for non-finite x.  When the LM head's epilogue left
+    // the row's maxima and minima per 128 columns (pmax: NaN-propagating), they replace the pass.
     float m = -INFINITY, nf = 0.f;
-    {
+    if (pmax) {
+      for (int i = threadIdx.x; i < npart; i += NT) {
+        const float a = pmax[(size_t)r * npart + i], b = pmin[(size_t)r * npart + i];
+        m = fmaxf(m, a);
+        nf += (a - a) + (b - b);  // NaN for a NaN or infinite maximum or an infinite minimum
+      }
+    } else {
       constexpr int U = 4;  // independent 16-byte loads in flight per thread
       int i0 = threadIdx.x;
       for (; i0 + (U - 1) * NT < n4; i0 += U * NT) {
@@ -541,7 +549,7 @@ __global__ void __launch_bounds__(NT, CPS)
 }
 
 int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, uint64_t* W, uint64_t* A, int32_t* Hq,
-                  int32_t* top, float* mx, cudaStream_t s) {
+                  int32_t* top, float* mx, cudaStream_t s, const float* pmax, const float* pmin) {
   if (rows == 0) return DLMZ_OK;
   int* err = device_error_word();
   const int grid = (rows + 7) / 8;
@@ -553,7 +561,9 @@ int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, ui
   else if (V <= 512) quantize_warp_kernel<16><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V % 4 == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0) {
     const int g = rows < QCPS * num_sms() ? rows : QCPS * num_sms();
-    quantize_persist_kernel<QNT, QCPS><<<g, QNT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
+    const bool part = pmax && pmin && V % 128 == 0;
+    quantize_persist_kernel<QNT, QCPS><<<g, QNT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err,
+                                                         part ? pmax : nullptr, part ? pmin : nullptr, V / 128);
   } else {
     quantize_cta_kernel<<<rows, QT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   }

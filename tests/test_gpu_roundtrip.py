@@ -321,3 +321,40 @@ def test_model_step_api_matches_whole_file(dev, spec, V, L, nc, pol_args):
     run(lambda r0, rpc: m.decode_step(dec, pol, r0, rpc, ptr(state), ptr(committed)))
     d.check()
     assert np.array_equal(state.cpu().numpy(), sym)
+
+
+def test_model_step_matches_logits_step_large_vocabulary(dev):
+    """V > 512: the model-driven step quantises its candidates from the LM head epilogue's row
+    maxima (one read of each logit); the logits-driven step reads the same logits twice.  Both
+    must give the same streams."""
+    import torch
+    d = dlmz()
+    V, L, nc, k, blk = 1024, 128, 3, 8, 64
+    m = d.Model(1, 256, 4, 4, 256, V, d.BF16, seed=77)
+    sym = to_dev(np.random.default_rng(5).integers(0, V, (nc, L)).astype(np.int32))
+    pol = d.policy(S.TOPK_CONF, k, blk)
+    streams = []
+    from oracle import quantizer as Q
+    for driven_by_model in (True, False):
+        coder = d.Coder(nc, L, V, Q.precision_for_vocab(V))
+        coder.reset_encoder()
+        state = to_dev(np.full((nc, L), V, dtype=np.int32))
+        logits = torch.empty(nc * blk, V, dtype=torch.float32, device="cuda")
+        for b0 in range(0, L, blk):
+            for _ in range(blk // k):
+                if driven_by_model:
+                    m.encode_step(coder, pol, b0, blk, ptr(sym), ptr(state))
+                else:
+                    m.forward_logits(ptr(state), nc, L, b0, blk, ptr(logits))
+                    coder.encode_step(pol, ptr(logits), b0, blk, ptr(sym), ptr(state))
+        d.check()
+        assert torch.equal(state, sym)
+        bits = torch.empty(nc, dtype=torch.int32, device="cuda")
+        raw = torch.zeros(nc * coder.capacity_units * 2, dtype=torch.uint8, device="cuda")
+        coder.finish(ptr(bits), ptr(raw))
+        d.check()
+        streams.append((bits.cpu().numpy().copy(), raw.cpu().numpy().copy()))
+        coder.close()
+    assert np.array_equal(streams[0][0], streams[1][0])
+    assert np.array_equal(streams[0][1], streams[1][1])
+    m.close()
