@@ -491,10 +491,24 @@ def secondary_c2(dlmz, torch, dev, steps=2):
     e1.record()
     e1.synchronize()
     ms = e0.elapsed_time(e1) / steps
+    # one more, untimed step with events around every launch: the kernel split and the rooflines
+    prof = dlmz.Profile()
+    dlmz.profile_begin()
+    step()
+    dlmz.profile_end(prof)
     m.close()
+    _, _, tf_sus, _ = peaks()
+    gi, ai = CLASSES.index("gemm_tcgen05"), CLASSES.index("attention")
+    kern_ms = sum(float(prof.ms[j]) for j in range(8))
+    split = {c: {"launches": int(prof.n[j]), "ms": round(float(prof.ms[j]), 3), "share": round(float(prof.ms[j]) / kern_ms, 4)}
+             for j, c in enumerate(CLASSES) if prof.n[j]}
+    frac = lambda j: float(prof.flops[j]) / (float(prof.ms[j]) / 1000.0) / 1e12 / tf_sus if prof.ms[j] else None
     return {"workload": C2_WORKLOAD, "value": per / (ms / 1000.0), "unit": "B/s", "ms_per_step": ms,
             "steps": steps, "warmup": 1, "bits_per_byte": 8.0 * n / per,
-            "step": "compress + decompress of one 512 KiB batch (64 + 64 denoising steps), device buffers"}
+            "step": "compress + decompress of one 512 KiB batch (64 + 64 denoising steps), device buffers",
+            "kernel_time_split": split,
+            "gemm_frac_of_sustained_bf16": frac(gi), "attention_frac_of_sustained_bf16": frac(ai),
+            "kernel_split_source": "one more untimed step, CUDA events around every launch"}
 
 
 def secondary_c3(dlmz, torch, dev, hbm, steps=5):
