@@ -561,45 +561,56 @@ __global__ void __launch_bounds__(THREADS, 1)
       constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
       constexpr uint32_t ID_O = t5::idesc_f16(BQ, HD);
       bool issued = false;
-      // S_X(J) = Q_X K_J^T; tile A waits for K_J (and, at an item's first tile, each tile for its Q)
-      auto issue_s = [&](int x, int J) -> bool {
-        const int st = J & 1, it = J / nt;
-        if (J % nt == 0 && !mbar_wait_bounded(q_full(x), it & 1, &abort_flag, err)) return false;
+      // descriptors of the operand stages (the K = 16 steps add 32 bytes to the start address)
+      const uint64_t dQ0 = t5::sw128_desc(sQ), dK0 = t5::sw128_desc(sK), dV0 = t5::sw128_desc(sVt);
+      constexpr uint64_t QT16 = S::QT >> 4, KT16 = S::KT >> 4, VT16 = S::VTT >> 4;
+      // S_X(J) = Q_X K_J^T (it = J / nt, j = J % nt); tile A waits for K_J (and, at an item's first
+      // tile, each tile for its Q)
+      auto issue_s = [&](int x, int J, int it, int j) -> bool {
+        const int st = J & 1;
+        if (j == 0 && !mbar_wait_bounded(q_full(x), it & 1, &abort_flag, err)) return false;
         if (x == 0 && !mbar_wait_bounded(k_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
         t5::fence_after();
+        const uint64_t dq = dQ0 + (uint64_t)x * QT16, dk = dK0 + (uint64_t)st * KT16;
+#pragma unroll
         for (int kb = 0; kb < HD / 64; ++kb)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            t5::mma_bf16(tS(x), t5::sw128_desc(sQ + x * S::QT + kb * BQ * 128 + 32 * k),
-                         t5::sw128_desc(sK + st * S::KT + kb * BK * 128 + 32 * k), ID_S, (kb | k) != 0);
+            t5::mma_bf16(tS(x), dq + (uint64_t)((kb * BQ * 128 + 32 * k) >> 4), dk + (uint64_t)((kb * BK * 128 + 32 * k) >> 4),
+                         ID_S, (kb | k) != 0);
         t5::commit(s_full(x));
         if (x == 1) t5::commit(k_empty(st));
-        if (J % nt == nt - 1) t5::commit(q_empty(x));
+        if (j == nt - 1) t5::commit(q_empty(x));
         issued = true;
         return true;
       };
       // O_X (+)= P_X(J) V_J, P_X in the first 64 columns of S_X (8 columns per 16 keys)
-      auto issue_pv = [&](int x, int J) -> bool {
-        const int st = J & 1, it = J / nt, j = J % nt;
+      auto issue_pv = [&](int x, int J, int it, int j) -> bool {
+        const int st = J & 1;
         if (!mbar_wait_bounded(p_ready(x), J & 1, &abort_flag, err)) return false;
         if (x == 0 && !mbar_wait_bounded(v_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
         // the first P V of an item overwrites O_X: the softmax group must have read the previous item's O_X
         if (j == 0 && it > 0 && !mbar_wait_bounded(o_free(x), (it - 1) & 1, &abort_flag, err)) return false;
         t5::fence_after();
+        const uint64_t dv = dV0 + (uint64_t)st * VT16;
 #pragma unroll
         for (int k = 0; k < BK / 16; ++k)
-          t5::mma_tmem_a(tO(x), tS(x) + 8 * k, t5::sw128_desc(sVt + st * S::VTT + (k >> 2) * HD * 128 + 32 * (k & 3)),
-                         ID_O, (j | k) != 0);
+          t5::mma_tmem_a(tO(x), tS(x) + 8 * k, dv + (uint64_t)(((k >> 2) * HD * 128 + 32 * (k & 3)) >> 4), ID_O,
+                         (j | k) != 0);
         if (x == 1) t5::commit(v_empty(st));
         if (J == total - 1) t5::commit(fin(x));
         return true;
       };
-      bool ok = total == 0 || (issue_s(0, 0) && issue_s(1, 0));
+      bool ok = total == 0 || (issue_s(0, 0, 0, 0) && issue_s(1, 0, 0, 0));
+      int it = 0, j = 0;  // J = it * nt + j
       for (int J = 0; ok && J < total; ++J) {
-        if (!issue_pv(0, J)) break;
-        if (J + 1 < total && !issue_s(0, J + 1)) break;
-        if (!issue_pv(1, J)) break;
-        if (J + 1 < total && !issue_s(1, J + 1)) break;
+        const int it1 = j + 1 == nt ? it + 1 : it, j1 = j + 1 == nt ? 0 : j + 1;  // of J + 1
+        if (!issue_pv(0, J, it, j)) break;
+        if (J + 1 < total && !issue_s(0, J + 1, it1, j1)) break;
+        if (!issue_pv(1, J, it, j)) break;
+        if (J + 1 < total && !issue_s(1, J + 1, it1, j1)) break;
+        it = it1;
+        j = j1;
       }
       if (abort_flag && issued) {
         volatile int never = 0;
