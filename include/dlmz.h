@@ -205,8 +205,8 @@ DLMZ_API int dlmz_gemm_bf16(const void* d_A, const void* d_B, float* d_D, uint32
  * d_out: bf16 [n_chunks L x n_heads hd] device.  Both 16-byte aligned; the
  *   caller owns both.
  * head_dim one of 8, 16, 32, 64, 128; n_chunks <= 65535.  Runs on the tcgen05
- * tensor cores when L % 128 == 0 and head_dim == 64 (V is converted to f16
- * there, so |v| < 65504), else on CUDA cores; P is rounded to f16 (tensor
+ * tensor cores when L % 128 == 0 and head_dim is 64 or 128 (V is converted to
+ * f16 there, so |v| < 65504), else on CUDA cores; P is rounded to f16 (tensor
  * cores) or kept in float32 (CUDA cores) before P V.  The tensor-core path
  * converts V into a library-owned V^T scratch buffer (grown with cudaMalloc
  * as needed, kept until exit): calls that overlap on the GPU race on it;

@@ -233,32 +233,39 @@ __global__ void __launch_bounds__(THREADS, Tmem<HD>::CTAS_PER_SM)  // head dim 6
       constexpr uint32_t ID_S = t5::idesc_bf16(BQ, BK);
       constexpr uint32_t ID_O = t5::idesc_f16(BQ, HD);
       bool issued = false;
-      // S_J = Q K_J^T; the first tile of an item waits for that item's Q, the
-      // last one releases Q to the next item's load
-      auto issue_s = [&](int J) -> bool {
-        const int st = J & 1, it = J / nt, qs = it & 1;
-        if (J % nt == 0 && !mbar_wait_bounded(q_full(qs), (it >> 1) & 1, &abort_flag, err)) return false;
+      // descriptors of the operand stages (the K = 16 steps add 32 bytes to the start address)
+      const uint64_t dQ0 = t5::sw128_desc(sQ), dK0 = t5::sw128_desc(sK), dV0 = t5::sw128_desc(sVt);
+      constexpr uint64_t QT16 = S::QT >> 4, KT16 = S::KT >> 4, VT16 = S::VTT >> 4;
+      // S_J = Q K_J^T (it = J / nt, j = J % nt); the first tile of an item waits for that item's Q,
+      // the last one releases Q to the next item's load
+      auto issue_s = [&](int J, int it, int j) -> bool {
+        const int st = J & 1, qs = it & 1;
+        if (j == 0 && !mbar_wait_bounded(q_full(qs), (it >> 1) & 1, &abort_flag, err)) return false;
         if (!mbar_wait_bounded(k_full(st), (J >> 1) & 1, &abort_flag, err)) return false;
         t5::fence_after();
+        const uint64_t dq = dQ0 + (uint64_t)qs * QT16, dk = dK0 + (uint64_t)st * KT16;
+#pragma unroll
         for (int kb = 0; kb < HD / 64; ++kb)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            t5::mma_bf16(tS, t5::sw128_desc(sQ + qs * S::QT + kb * BQ * 128 + 32 * k),
-                         t5::sw128_desc(sK + st * S::KT + kb * BK * 128 + 32 * k), ID_S, (kb | k) != 0);
+            t5::mma_bf16(tS, dq + (uint64_t)((kb * BQ * 128 + 32 * k) >> 4), dk + (uint64_t)((kb * BK * 128 + 32 * k) >> 4),
+                         ID_S, (kb | k) != 0);
         t5::commit(s_full);
         t5::commit(k_empty(st));
-        if (J % nt == nt - 1) t5::commit(q_empty(qs));
+        if (j == nt - 1) t5::commit(q_empty(qs));
         issued = true;
         return true;
       };
-      bool ok = total == 0 || issue_s(0);
+      bool ok = total == 0 || issue_s(0, 0, 0);
+      int it = 0, j = 0;  // J = it * nt + j
       for (int J = 0; ok && J < total; ++J) {
-        const int it = J / nt, j = J % nt, st = J & 1;
+        const int st = J & 1;
+        const int it1 = j + 1 == nt ? it + 1 : it, j1 = j + 1 == nt ? 0 : j + 1;  // of J + 1
         // S_{J+1} goes as soon as the softmax has S_J in registers, so it runs under P_J's exponentials
         // (across items too: the next item's first QK^T overlaps this item's last softmax and epilogue)
         if (J + 1 < total) {
           if (!mbar_wait_bounded(s_free, J & 1, &abort_flag, err)) break;
-          if (!issue_s(J + 1)) break;
+          if (!issue_s(J + 1, it1, j1)) break;
         }
         if (!mbar_wait_bounded(p_ready, J & 1, &abort_flag, err)) break;
         if (!mbar_wait_bounded(v_full(st), (J >> 1) & 1, &abort_flag, err)) break;
@@ -266,12 +273,15 @@ __global__ void __launch_bounds__(THREADS, Tmem<HD>::CTAS_PER_SM)  // head dim 6
         if (j == 0 && it > 0 && !mbar_wait_bounded(o_free, (it - 1) & 1, &abort_flag, err)) break;
         t5::fence_after();
         // 8 steps of 16 keys: P_j columns 8k..8k+7, V^T block k / 4 at byte offset 32 (k % 4)
+        const uint64_t dv = dV0 + (uint64_t)st * VT16;
 #pragma unroll
         for (int k = 0; k < BK / 16; ++k)
-          t5::mma_tmem_a(tO, tP + 8 * k, t5::sw128_desc(sVt + st * S::VTT + (k >> 2) * HD * 128 + 32 * (k & 3)),
-                         ID_O, (j | k) != 0);
+          t5::mma_tmem_a(tO, tP + 8 * k, dv + (uint64_t)(((k >> 2) * HD * 128 + 32 * (k & 3)) >> 4), ID_O,
+                         (j | k) != 0);
         t5::commit(v_empty(st));
         t5::commit(o_done);
+        it = it1;
+        j = j1;
       }
       if (abort_flag && issued) {
         volatile int never = 0;

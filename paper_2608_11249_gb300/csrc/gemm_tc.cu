@@ -387,6 +387,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool issued_any = false;
+      // descriptors of the ring's stages (the K = 16 steps add 32 bytes to the start address)
+      const uint64_t dA0 = t5::sw128_desc(smem_u32(sA)), dB0 = t5::sw128_desc(smem_u32(sB));
       for (int tile = cid; tile < total && !abort_flag; tile += n_ctas) {
         if (!mbar_wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1, &abort_flag, err)) break;
         fence_after();
@@ -398,11 +400,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             break;
           }
           fence_after();
-          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
-          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+          const uint64_t da = dA0 + (uint64_t)stage * (A_BYTES >> 4), db = dB0 + (uint64_t)stage * (B_BYTES >> 4);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            t5::mma_bf16(d_tmem, t5::sw128_desc(a0 + 32 * k), t5::sw128_desc(b0 + 32 * k), IDESC, (kb | k) != 0);
+            t5::mma_bf16(d_tmem, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), IDESC, (kb | k) != 0);
           issued_any = true;
           t5::commit(empty0 + 8 * stage);  // the stage is free once the products have read it
           if (++stage == STAGES) {
