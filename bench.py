@@ -59,7 +59,7 @@ C2_WORKLOAD = ("small byte-level masked DLM, bf16, 8 layers d=512 8 heads FFN 20
 C3_ROWS, C3_V, C3_GROUP, C3_TOPK = 65536, 126464, 1024, 32
 # Mean DRAM bytes per tcgen05 GEMM launch of an 8B-shaped layer at 512 windows, scaled from an ncu
 # capture of the same kernels at 16 windows (B is re-read once per row group, so traffic grows with M)
-GEMM_TRAFFIC_PER_LAUNCH = 53.1e9
+GEMM_TRAFFIC_PER_LAUNCH = 53.4e9
 CLASSES = ["gemm_tcgen05", "gemm_cuda_core", "attention", "quantize", "select", "code", "norm_rope_embed", "other"]
 
 

@@ -56,6 +56,7 @@ static int check_device(cudaStream_t s) {
   DLMZ_CUDA_TRY(cudaMemcpy(&h, e, sizeof(int), cudaMemcpyDeviceToHost));
   if (h) DLMZ_CUDA_TRY(cudaMemset(e, 0, sizeof(int)));
   if (h & ERR_TIMEOUT) return DLMZ_ETIMEOUT;
+  if (h & ERR_LAUNCH) return DLMZ_ECUDA;
   if (h & ERR_NONFINITE) return DLMZ_EBADINPUT;
   if (h & (ERR_CORRUPT | ERR_CAPACITY)) return DLMZ_ECORRUPT;
   return DLMZ_OK;

@@ -548,6 +548,496 @@ __global__ void __launch_bounds__(NT, CPS)
   }
 }
 
+// ---- large vocabularies: a cluster of two CTAs per row -------------------------------------
+// Each CTA of the pair takes one contiguous half of the row (in float4s).  With two 512-thread
+// CTAs per SM, 152 rows are in flight (77 MB at V = 126464, 92 MB at 152064), so the histogram
+// and CDF passes re-read the row from L2 rather than HBM.  Everything one half needs from the
+// other is a value or a sum over histogram bins, so the pair exchanges scalars only, through
+// distributed shared memory (thread 0 stores into both CTAs' slot and arrives on the peer's
+// mbarrier; the slots and barriers alternate between two sets):
+//   1. the halves' maxima (NaN-propagating) and minima -> m and the non-finite flag;
+//   2. W and A over each half's bins and the lowest index of m in each half;
+//   3. each half's sum of floor(w R / W) -> D and the CDF offset of the second half.
+// A half's CDF pass looks up only codes that occur in it, i.e. its own non-empty bins, so each
+// CTA fills the table value 1 + floor(w(q) R / W) for those bins alone.
+constexpr int QP_NT = 512;  // threads per CTA (two CTAs per SM)
+constexpr int QU = 8;       // float4 loads in flight per thread in the first pass
+constexpr int QH = 8;       // and in the second
+
+struct QPairSlot {  // one exchange, indexed by the sender's rank
+  uint64_t W[2], A[2];
+  float mx[2], mn[2];
+  uint32_t fs[2];
+  int top[2];
+};
+
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float d;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+  return d;
+}
+__device__ __forceinline__ float fmax3_nan(float a, float b, float c) {
+  float d;
+  asm("max.NaN.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ float fmin3(float a, float b, float c) {
+  float d;
+  asm("min.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+// table entry q of the code bits QMAGIC + q in [QMAGIC, QMAGIC + QW0] (pair_code's range): the byte
+// address base + 4 bits with base = table - 4 QMAGIC (32-bit wrap-around)
+__device__ __forceinline__ uint32_t lds_code(uint32_t base, uint32_t bits) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(base + 4u * bits));
+  return v;
+}
+__device__ __forceinline__ void red_code(uint32_t base, uint32_t bits) {
+  asm volatile("red.shared.add.u32 [%0], 1;" ::"r"(base + 4u * bits) : "memory");
+}
+// inclusive warp scan step: s += value of lane - d (lanes below d unchanged)
+template <int d>
+__device__ __forceinline__ void scan_step(uint32_t& s) {
+  asm volatile(
+      "{\n\t.reg .b32 t;\n\t.reg .pred p;\n\tshfl.sync.up.b32 t|p, %0, %1, 0, -1;\n\t@p add.u32 %0, %0, t;\n\t}"
+      : "+r"(s)
+      : "n"(d));
+}
+
+// code_bits of d = fl32(m - l) (in [QMAGIC, QMAGIC + QW0]: d >= 0 or NaN, as m is the row's maximum
+// computed here).  With PART the maximum comes from another kernel, so d is also clamped below at
+// 0 there: d < 0 (l above that maximum) never happens for consistent inputs, and the clamp keeps the
+// table index in range whatever they are (NaN stays NaN and lands on QW0).
+template <bool PART>
+__device__ __forceinline__ uint32_t pair_code(float d) {
+  if (!PART) return code_bits(d);
+  const float t = fminf(fmax_nan(__fmul_rn(d, __uint_as_float(DLMZ_QSCALE_BITS)), 0.f), (float)QW0);
+  return __float_as_uint(__fadd_rn(t, 12582912.0f));
+}
+
+template <bool PART>
+__global__ void __launch_bounds__(QP_NT, 2)
+    quantize_pair_kernel(const float* __restrict__ logits, int rows, int V, int P, uint32_t* __restrict__ cdf,
+                         uint64_t* __restrict__ Wout, uint64_t* __restrict__ Aout, int32_t* __restrict__ Hq,
+                         int32_t* __restrict__ topout, float* __restrict__ mxout, int* err,
+                         const float* __restrict__ pmax, const float* __restrict__ pmin, int npart) {
+  constexpr int NT = QP_NT, NW = NT / 32, BPT = NQ / NT;
+  __shared__ __align__(16) uint32_t tab[NQ];  // histogram of the codes, then 1 + floor(w R / W)
+  extern __shared__ uint4 stage[];             // CDF store staging, 64 16-byte chunks per warp
+  __shared__ uint32_t T[256];
+  __shared__ QPairSlot xs[2];
+  __shared__ __align__(8) uint64_t xbar[2];
+  __shared__ float rf[2][NW];
+  __shared__ uint64_t ru[2][NW];
+  __shared__ int ri[NW];
+  __shared__ uint32_t wsum[2][2][NW];
+  __shared__ float s_m;
+  __shared__ int s_bad, s_top, s_ok;
+  __shared__ uint64_t s_W, s_K;
+  __shared__ uint32_t s_D, s_carry;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (cluster_nctarank() != 2) {  // launched without its cluster shape: no cluster operation runs
+    if (tid == 0) atomicOr(err, ERR_LAUNCH);
+    return;
+  }
+  const uint32_t rank = cluster_ctarank(), peer = rank ^ 1u;
+  for (int i = tid; i < 256; i += NT) T[i] = c_exp_table[i];
+  if (tid == 0) {
+    mbar_init(smem_u32(&xbar[0]), 1);
+    mbar_init(smem_u32(&xbar[1]), 1);
+    s_ok = 1;
+    fence_mbarrier_init_cluster();
+  }
+  cluster_sync_all();  // the peer's barriers are initialised before any arrival on them
+
+  const int n4 = V >> 2, half = (n4 + 1) >> 1;
+  const int c0 = rank ? half : 0, n = rank ? n4 - half : half;  // this CTA's float4s [c0, c0 + n)
+  const uint32_t R = (1u << P) - (uint32_t)V;
+  const uint32_t tabq = smem_u32(tab) - 4u * QMAGIC;
+  const uint32_t Tt = T[tid & 255];  // bins tid + k NT share T[b & 255] (NT is a multiple of 256)
+  uint32_t xk = 0;                   // exchanges so far
+
+  // thread 0: the slot of exchange xk is written (own copy and the peer's); signal the peer and wait
+  // for its values.  Returns false (error word set) if the peer's arrival does not come.
+  auto exchange_wait = [&]() -> bool {
+    const uint32_t b = xk & 1u;
+    mbar_arrive_remote(mapa_shared(smem_u32(&xbar[b]), peer));
+    const bool ok = mbar_wait_cluster_bounded(smem_u32(&xbar[b]), (xk >> 1) & 1u, err);
+    ++xk;
+    return ok;
+  };
+  auto put_u64 = [&](uint64_t* p, uint64_t v) {
+    *p = v;
+    st_cluster_u64(mapa_shared(smem_u32(p), peer), v);
+  };
+  auto put_u32 = [&](uint32_t* p, uint32_t v) {
+    *p = v;
+    st_cluster_u32(mapa_shared(smem_u32(p), peer), v);
+  };
+
+  for (int r = blockIdx.x >> 1; r < rows; r += gridDim.x >> 1) {
+    const float4* lc = reinterpret_cast<const float4*>(logits + (size_t)r * V) + c0;
+    // ---- m and the non-finite flag
+    float mx = -INFINITY, mn = INFINITY;
+    if (PART) {  // per-128-column maxima (NaN-propagating) and minima from the LM head: the whole row
+      for (int i = tid; i < npart; i += NT) {
+        mx = fmax_nan(mx, pmax[(size_t)r * npart + i]);
+        mn = fminf(mn, pmin[(size_t)r * npart + i]);
+      }
+    } else {  // pass 1 (HBM) over this half, QU float4 loads in flight per thread
+      // past the end, a thread re-reads the half's last float4 (a repeat leaves the maximum and the
+      // minimum as they are), so every load is unconditional
+      for (int i = tid; i < n; i += QU * NT) {
+        float4 x[QU];
+#pragma unroll
+        for (int u = 0; u < QU; ++u) x[u] = lc[min(i + u * NT, n - 1)];
+#pragma unroll
+        for (int u = 0; u < QU; ++u) {
+          mx = fmax3_nan(mx, x[u].x, x[u].y);
+          mx = fmax3_nan(mx, x[u].z, x[u].w);
+          mn = fmin3(mn, x[u].x, x[u].y);
+          mn = fmin3(mn, x[u].z, x[u].w);
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      mx = fmax_nan(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    }
+    if (lane == 0) {
+      rf[0][warp] = mx;
+      rf[1][warp] = mn;
+    }
+    __syncthreads();  // also: the previous row's CDF pass is done with tab
+    for (int b = tid; b < NQ / 4; b += NT) reinterpret_cast<uint4*>(tab)[b] = make_uint4(0u, 0u, 0u, 0u);
+    if (tid == 0) {
+      float a = -INFINITY, z = INFINITY;
+      for (int w = 0; w < NW; ++w) {
+        a = fmax_nan(a, rf[0][w]);
+        z = fminf(z, rf[1][w]);
+      }
+      bool ok = true;
+      if (!PART) {
+        QPairSlot& x = xs[xk & 1u];
+        put_u32(reinterpret_cast<uint32_t*>(&x.mx[rank]), __float_as_uint(a));
+        put_u32(reinterpret_cast<uint32_t*>(&x.mn[rank]), __float_as_uint(z));
+        ok = exchange_wait();
+        a = fmax_nan(x.mx[0], x.mx[1]);
+        z = fminf(x.mn[0], x.mn[1]);
+      }
+      const int bad = !(isfinite(a) && z > -INFINITY);
+      if (bad && rank == 0) atomicOr(err, ERR_NONFINITE);
+      s_m = bad ? INFINITY : a;  // m = +inf sends every code to QW0 (no weight); W is pinned below
+      s_bad = bad;
+      s_ok = ok;
+    }
+    __syncthreads();
+    if (!s_ok) break;
+    const float m = s_m;
+    // ---- pass 2 (L2): histogram of the codes (codes >= QW0 share bin QW0, which weighs nothing) and
+    // the lowest index of m in this half (m - l == 0 exactly when l == m)
+    int topc = 0x7fffffff;
+    {
+      auto hist4 = [&](const float4 x, int i) {
+        const float d0 = __fsub_rn(m, x.x), d1 = __fsub_rn(m, x.y), d2 = __fsub_rn(m, x.z), d3 = __fsub_rn(m, x.w);
+        red_code(tabq, pair_code<PART>(d0));
+        red_code(tabq, pair_code<PART>(d1));
+        red_code(tabq, pair_code<PART>(d2));
+        red_code(tabq, pair_code<PART>(d3));
+        if (fminf(fmin3(d0, d1, d2), d3) == 0.f)
+          topc = min(topc, 4 * (c0 + i) + (d0 == 0.f ? 0 : d1 == 0.f ? 1 : d2 == 0.f ? 2 : 3));
+      };
+      for (int i = tid; i < n; i += QH * NT) {
+        float4 x[QH];
+#pragma unroll
+        for (int u = 0; u < QH; ++u) x[u] = lc[min(i + u * NT, n - 1)];
+#pragma unroll
+        for (int u = 0; u < QH; ++u)
+          if (i + u * NT < n) hist4(x[u], i + u * NT);
+      }
+    }
+    topc = __reduce_min_sync(0xffffffffu, topc);
+    if (lane == 0) ri[warp] = topc;
+    __syncthreads();  // histogram complete
+    // ---- W and A over this half's bins
+    uint64_t Ws = 0, As = 0;
+#pragma unroll 4
+    for (int k = 0; k < BPT; ++k) {
+      const int b = tid + k * NT;
+      if (b < QW0) {
+        const uint64_t hw = (uint64_t)tab[b] * (Tt >> (b >> 8));
+        Ws += hw;
+        As += hw * (uint32_t)b;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      Ws += __shfl_xor_sync(0xffffffffu, Ws, o);
+      As += __shfl_xor_sync(0xffffffffu, As, o);
+    }
+    if (lane == 0) {
+      ru[0][warp] = Ws;
+      ru[1][warp] = As;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint64_t tw = 0, ta = 0;
+      int tp = 0x7fffffff;
+      for (int w = 0; w < NW; ++w) {
+        tw += ru[0][w];
+        ta += ru[1][w];
+        tp = min(tp, ri[w]);
+      }
+      QPairSlot& x = xs[xk & 1u];
+      put_u64(&x.W[rank], tw);
+      put_u64(&x.A[rank], ta);
+      put_u32(reinterpret_cast<uint32_t*>(&x.top[rank]), (uint32_t)tp);
+      const bool ok = exchange_wait();
+      tw = x.W[0] + x.W[1];
+      ta = x.A[0] + x.A[1];
+      tp = x.top[0] != 0x7fffffff ? x.top[0] : x.top[1];
+      if (tp == 0x7fffffff) tp = 0;  // only for rows flagged non-finite
+      if (s_bad) {                   // all codes QW0 (w = 0): any W >= 2^31 keeps the tables defined
+        tw = 1ull << 31;
+        ta = 0;
+      }
+      s_top = tp;
+      s_W = tw;
+      s_K = recip_scaled(R, tw);
+      s_ok = ok;
+      if (rank == 0) {
+        Wout[r] = tw;
+        if (Aout) Aout[r] = ta;
+        Hq[r] = entropy_q(tw, ta);
+        if (topout) topout[r] = tp;
+        if (mxout) mxout[r] = m;
+      }
+    }
+    __syncthreads();
+    if (!s_ok) break;
+    if (!cdf) continue;
+    // ---- 1 + floor(w(q) R / W) for this half's non-empty bins, and the half's sum of the floors
+    {
+      const uint64_t Wr = s_W, K = s_K;
+      uint32_t fs = 0;  // <= R
+#pragma unroll 4
+      for (int k = 0; k < BPT; ++k) {
+        const int b = tid + k * NT;
+        if (b < QW0) {
+          const uint32_t h = tab[b];
+          if (h) {
+            const uint32_t f = floor_wr_over_w(Tt >> (b >> 8), R, Wr, K);
+            fs += h * f;
+            tab[b] = 1u + f;
+          }
+        }
+      }
+      fs = __reduce_add_sync(0xffffffffu, fs);
+      if (lane == 0) ri[warp] = (int)fs;
+      __syncthreads();
+      if (tid == 0) {
+        tab[QW0] = 1u;  // codes >= QW0: f = 0
+        uint32_t t = 0;
+        for (int w = 0; w < NW; ++w) t += (uint32_t)ri[w];
+        QPairSlot& x = xs[xk & 1u];
+        put_u32(&x.fs[rank], t);
+        const bool ok = exchange_wait();
+        const uint32_t D = R - x.fs[0] - x.fs[1];
+        s_D = D;
+        // the first half's entries sum to its element count + its floors (+ D if m's first index is there)
+        s_carry = rank ? (uint32_t)(4 * half) + x.fs[0] + ((uint32_t)s_top < (uint32_t)(4 * half) ? D : 0u) : 0u;
+        s_ok = ok;
+      }
+      __syncthreads();
+      if (!s_ok) break;
+    }
+    // ---- pass 3 (L2): CDF[v + 1] = sum_{u <= v} (1 + floor(w_u R / W) + (u == top ? D : 0)).  A tile is
+    // 2 NT float4s; thread t scans the 8 elements of float4s 2t, 2t + 1 in registers, then the warp
+    // and the CTA add their offsets.  Stores are aligned 16-byte quads (the row's entry 1 starts at
+    // word offset s mod 4; each lane writes the quad that starts in its own range, completed by the
+    // next lane's first elements; a warp's first and last lanes write their edges singly).
+    const uint32_t D = s_D;
+    const int top = s_top;
+    uint32_t carry = s_carry;
+    uint32_t* cr = cdf + (size_t)r * (V + 1);
+    if (rank == 0 && tid == 0) cr[0] = 0;
+    const int e0 = (int)((0u - (uint32_t)(reinterpret_cast<uintptr_t>(cr + 1) >> 2)) & 3u);
+    // local part of a tile: thread t's 8 table values (plus D at m's first index, zero past this
+    // half), their running sums in o[], and the inclusive warp scan of the threads' totals
+    auto tile_local = [&](int t0, const float4 xa, const float4 xb, uint32_t(&o)[8]) -> uint32_t {
+      const int j = t0 + 2 * tid;
+      const bool full = t0 + 2 * NT <= n;
+      const bool va = full || j < n, vb = full || j + 1 < n;
+      o[0] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.x)));
+      o[1] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.y)));
+      o[2] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.z)));
+      o[3] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.w)));
+      o[4] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.x)));
+      o[5] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.y)));
+      o[6] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.z)));
+      o[7] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.w)));
+      const uint32_t dt = (uint32_t)(top - 4 * (c0 + j));
+      if (dt < 8u) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o[e] += dt == (uint32_t)e ? D : 0u;
+      }
+      if (!full) {  // past the end of this half (the other half's elements or the row's end): nothing
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          o[e] = va ? o[e] : 0u;
+          o[e + 4] = vb ? o[e + 4] : 0u;
+        }
+      }
+#pragma unroll
+      for (int e = 1; e < 8; ++e) o[e] += o[e - 1];
+      uint32_t s = o[7];
+      scan_step<1>(s);
+      scan_step<2>(s);
+      scan_step<4>(s);
+      scan_step<8>(s);
+      scan_step<16>(s);
+      return s;
+    };
+    // the tile's CDF entries o[] + base, written out
+    auto tile_store = [&](int t0, uint32_t(&o)[8], uint32_t base) {
+      const int j = t0 + 2 * tid;
+      const bool full = t0 + 2 * NT <= n;
+      const bool va = full || j < n, vb = full || j + 1 < n;
+      const int v0 = 4 * (c0 + j);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) o[e] += base;
+      uint32_t* dst = cr + 1 + v0;
+      if (full) {
+        // this lane's aligned quads: elements e0..e0+3 and e0+4..e0+7 of its eight, the second
+        // completed by the next lane's first e0; staged per warp (chunk c of the warp block at
+        // slot c ^ ((c >> 3) & 1): no bank conflicts either way) so that each store instruction
+        // writes 512 contiguous bytes
+        uint4 q1, q2;
+        if (e0 == 0) {
+          q1 = make_uint4(o[0], o[1], o[2], o[3]);
+          q2 = make_uint4(o[4], o[5], o[6], o[7]);
+        } else {
+          const uint32_t n0 = __shfl_down_sync(0xffffffffu, o[0], 1);
+          const uint32_t n1 = __shfl_down_sync(0xffffffffu, o[1], 1);
+          const uint32_t n2 = __shfl_down_sync(0xffffffffu, o[2], 1);
+          if (e0 == 1) {
+            q1 = make_uint4(o[1], o[2], o[3], o[4]);
+            q2 = make_uint4(o[5], o[6], o[7], n0);
+          } else if (e0 == 2) {
+            q1 = make_uint4(o[2], o[3], o[4], o[5]);
+            q2 = make_uint4(o[6], o[7], n0, n1);
+          } else {
+            q1 = make_uint4(o[3], o[4], o[5], o[6]);
+            q2 = make_uint4(o[7], n0, n1, n2);
+          }
+          if (lane == 0) {  // the warp block's first e0 elements precede its first aligned quad
+#pragma unroll
+            for (int e = 0; e < 3; ++e)
+              if (e < e0) __stcs(dst + e, o[e]);
+          }
+        }
+        uint4* sb = stage + 64 * warp;
+        const int sw = (lane >> 2) & 1;
+        sb[(2 * lane) ^ sw] = q1;
+        sb[(2 * lane + 1) ^ sw] = q2;
+        __syncwarp();
+        const int rs = (lane >> 3) & 1;
+        const uint4 w0 = sb[lane ^ rs], w1 = sb[(32 + lane) ^ rs];
+        __syncwarp();
+        uint4* wq = reinterpret_cast<uint4*>(cr + 1 + 4 * (c0 + t0) + 256 * warp + e0);  // chunk 0
+        __stcs(wq + lane, w0);
+        if (lane < 31 || e0 == 0) {
+          __stcs(wq + 32 + lane, w1);
+        } else {  // chunk 63 runs e0 elements into the next warp block: its first 4 - e0 words only
+          uint32_t* t = reinterpret_cast<uint32_t*>(wq + 63);
+          __stcs(t, w1.x);
+          if (e0 < 3) __stcs(t + 1, w1.y);
+          if (e0 < 2) __stcs(t + 2, w1.z);
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          if (va) __stcs(dst + e, o[e]);
+          if (vb) __stcs(dst + 4 + e, o[e + 4]);
+        }
+      }
+    };
+    // past the end of this half: m itself (d = 0, an in-range code; the values are dropped)
+    auto ld4 = [&](int i) {
+      float4 x = make_float4(m, m, m, m);
+      if (i < n) x = __ldcs(lc + i);
+      return x;
+    };
+    // two tiles per barrier: their loads and local scans run side by side
+    int wb = 0;
+    for (int t0 = 0; t0 < n; t0 += 4 * NT) {
+      const int t1 = t0 + 2 * NT;  // the second tile (none past the end)
+      const float4 xa0 = ld4(t0 + 2 * tid), xb0 = ld4(t0 + 2 * tid + 1);
+      const float4 xa1 = ld4(t1 + 2 * tid), xb1 = ld4(t1 + 2 * tid + 1);
+      uint32_t oa[8], ob[8];
+      const uint32_t sa = tile_local(t0, xa0, xb0, oa);
+      const uint32_t sb = t1 < n ? tile_local(t1, xa1, xb1, ob) : 0u;
+      if (lane == 31) {
+        wsum[wb][0][warp] = sa;
+        wsum[wb][1][warp] = sb;
+      }
+      __syncthreads();
+      const uint32_t tva = lane < NW ? wsum[wb][0][lane] : 0u, tvb = lane < NW ? wsum[wb][1][lane] : 0u;
+      wb ^= 1;
+      tile_store(t0, oa, carry + __reduce_add_sync(0xffffffffu, lane < warp ? tva : 0u) + (sa - oa[7]));
+      carry += __reduce_add_sync(0xffffffffu, tva);
+      if (t1 < n) {
+        tile_store(t1, ob, carry + __reduce_add_sync(0xffffffffu, lane < warp ? tvb : 0u) + (sb - ob[7]));
+        carry += __reduce_add_sync(0xffffffffu, tvb);
+      }
+    }
+  }
+  cluster_sync_all();  // neither CTA leaves while the peer may still write to its shared memory
+}
+
+// clusters of quantize_pair_kernel that fit on the device at once (0: the launch shape is unavailable)
+constexpr int QP_STAGE_BYTES = QP_NT / 32 * 64 * 16;  // dynamic shared memory (static part ~34 KB)
+
+static cudaLaunchConfig_t pair_config(int grid, cudaStream_t s, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(QP_NT);
+  cfg.dynamicSmemBytes = QP_STAGE_BYTES;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+static int pair_clusters() {
+  static int n[kMaxDevices] = {};
+  const int dev = device_ordinal();
+  if (dev < 0) return 0;
+  if (!n[dev]) {
+    cudaLaunchAttribute attr[1];
+    const cudaLaunchConfig_t cfg = pair_config(2 * 2 * num_sms(), 0, attr);
+    int c = 0;
+    // static + dynamic shared memory exceeds the 48 KB default
+    if (cudaFuncSetAttribute(quantize_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             QP_STAGE_BYTES) != cudaSuccess ||
+        cudaFuncSetAttribute(quantize_pair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             QP_STAGE_BYTES) != cudaSuccess ||
+        cudaOccupancyMaxActiveClusters(&c, quantize_pair_kernel<false>, &cfg) != cudaSuccess || c < 1) {
+      cudaGetLastError();
+      c = -1;
+    }
+    n[dev] = c;
+  }
+  return n[dev] > 0 ? n[dev] : 0;
+}
+
 int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, uint64_t* W, uint64_t* A, int32_t* Hq,
                   int32_t* top, float* mx, cudaStream_t s, const float* pmax, const float* pmin) {
   if (rows == 0) return DLMZ_OK;
@@ -559,7 +1049,18 @@ int quantize_rows(const float* logits, int rows, int V, int P, uint32_t* cdf, ui
   else if (V <= 128) quantize_warp_kernel<4><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V <= 256) quantize_warp_kernel<8><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
   else if (V <= 512) quantize_warp_kernel<16><<<grid, 256, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err);
-  else if (V % 4 == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0) {
+  else if (V % 4 == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0 &&
+           (reinterpret_cast<uintptr_t>(cdf) & 15) == 0 && pair_clusters() > 0) {
+    cudaLaunchAttribute attr[1];
+    const cudaLaunchConfig_t cfg = pair_config(2 * (rows < pair_clusters() ? rows : pair_clusters()), s, attr);
+    const bool part = pmax && pmin && V % 128 == 0;
+    if (part)
+      cudaLaunchKernelEx(&cfg, quantize_pair_kernel<true>, logits, rows, V, P, cdf, W, A, Hq, top, mx, err, pmax, pmin,
+                         V / 128);
+    else
+      cudaLaunchKernelEx(&cfg, quantize_pair_kernel<false>, logits, rows, V, P, cdf, W, A, Hq, top, mx, err,
+                         (const float*)nullptr, (const float*)nullptr, 0);
+  } else if (V % 4 == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0) {
     const int g = rows < QCPS * num_sms() ? rows : QCPS * num_sms();
     const bool part = pmax && pmin && V % 128 == 0;
     quantize_persist_kernel<QNT, QCPS><<<g, QNT, 0, s>>>(logits, rows, V, P, cdf, W, A, Hq, top, mx, err,

@@ -44,6 +44,33 @@ def test_quantize_bit_exact(dev, V, n):
     assert np.array_equal(top.cpu().numpy(), ref["top"].astype(np.int32))
 
 
+@pytest.mark.parametrize("V,n", [(5000, 9), (126464, 4)])
+def test_quantize_unaligned_buffers(dev, V, n):
+    """CDF rows off a 16-byte boundary (one CTA per row in flight) and logits off a 16-byte boundary
+    (the generic kernel) give the same tables as the aligned case."""
+    import torch
+    d = dlmz()
+    l = _rows(V, n, V + 1)
+    rows = l.shape[0]
+    P = Q.precision_for_vocab(V)
+    ref = Q.quantize(l, P)
+    W = torch.empty(rows, dtype=torch.int64, device="cuda")
+    Hq = torch.empty(rows, dtype=torch.int32, device="cuda")
+    cbuf = torch.empty(rows * (V + 1) + 4, dtype=torch.int32, device="cuda")
+    cdf = cbuf[1:1 + rows * (V + 1)]  # 4 bytes past an aligned start
+    d.quantize(ptr(to_dev(l)), rows, V, P, ptr(cdf), ptr(W), 0, ptr(Hq), 0)
+    d.check()
+    assert np.array_equal(cdf.cpu().numpy().view(np.uint32).reshape(rows, V + 1), ref["cdf"])
+    assert np.array_equal(Hq.cpu().numpy(), ref["Hq"].astype(np.int32))
+    lbuf = torch.zeros(rows * V + 4, dtype=torch.float32, device="cuda")
+    lbuf[1:1 + rows * V] = torch.from_numpy(l.ravel()).cuda()
+    cdf2 = torch.empty(rows, V + 1, dtype=torch.int32, device="cuda")
+    d.quantize(ptr(lbuf[1:]), rows, V, P, ptr(cdf2), ptr(W), 0, ptr(Hq), 0)
+    d.check()
+    assert np.array_equal(cdf2.cpu().numpy().view(np.uint32), ref["cdf"])
+    assert np.array_equal(W.cpu().numpy().view(np.uint64), ref["W"])
+
+
 def test_quantize_isolated_workload_rows(dev):
     """Rows of the isolated quantise+select workload (N(0,3) + spike U(5,15), V = 126464)."""
     import torch
