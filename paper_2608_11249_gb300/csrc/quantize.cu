@@ -11,6 +11,8 @@
 //   H_q = log2q16(W) - 31*2^16 + floor(2^8 A / W)      (entropy, Sec. 3.3, 2^-16 bit)
 // Only __fsub_rn / __fmul_rn / __float2int_rn touch floating point, so the
 // result is independent of thread layout and reduction order.
+#include <type_traits>
+
 #include "kernels.cuh"
 #include "exp_table.inc"
 #include "intq.cuh"
@@ -687,19 +689,28 @@ __global__ void __launch_bounds__(QP_NT, 2)
         mn = fminf(mn, pmin[(size_t)r * npart + i]);
       }
     } else {  // pass 1 (HBM) over this half, QU float4 loads in flight per thread
-      // past the end, a thread re-reads the half's last float4 (a repeat leaves the maximum and the
-      // minimum as they are), so every load is unconditional
-      for (int i = tid; i < n; i += QU * NT) {
+      // the last round re-reads the half's last float4 past the end (a repeat leaves the maximum
+      // and the minimum as they are), so every load is unconditional
+      auto mxmn = [&](const float4 x) {
+        mx = fmax3_nan(mx, x.x, x.y);
+        mx = fmax3_nan(mx, x.z, x.w);
+        mn = fmin3(mn, x.x, x.y);
+        mn = fmin3(mn, x.z, x.w);
+      };
+      int i = tid;
+      for (; i + (QU - 1) * NT < n; i += QU * NT) {
+        float4 x[QU];
+#pragma unroll
+        for (int u = 0; u < QU; ++u) x[u] = lc[i + u * NT];
+#pragma unroll
+        for (int u = 0; u < QU; ++u) mxmn(x[u]);
+      }
+      if (i < n) {
         float4 x[QU];
 #pragma unroll
         for (int u = 0; u < QU; ++u) x[u] = lc[min(i + u * NT, n - 1)];
 #pragma unroll
-        for (int u = 0; u < QU; ++u) {
-          mx = fmax3_nan(mx, x[u].x, x[u].y);
-          mx = fmax3_nan(mx, x[u].z, x[u].w);
-          mn = fmin3(mn, x[u].x, x[u].y);
-          mn = fmin3(mn, x[u].z, x[u].w);
-        }
+        for (int u = 0; u < QU; ++u) mxmn(x[u]);
       }
     }
 #pragma unroll
@@ -750,7 +761,15 @@ __global__ void __launch_bounds__(QP_NT, 2)
         if (fminf(fmin3(d0, d1, d2), d3) == 0.f)
           topc = min(topc, 4 * (c0 + i) + (d0 == 0.f ? 0 : d1 == 0.f ? 1 : d2 == 0.f ? 2 : 3));
       };
-      for (int i = tid; i < n; i += QH * NT) {
+      int i = tid;
+      for (; i + (QH - 1) * NT < n; i += QH * NT) {
+        float4 x[QH];
+#pragma unroll
+        for (int u = 0; u < QH; ++u) x[u] = lc[i + u * NT];
+#pragma unroll
+        for (int u = 0; u < QH; ++u) hist4(x[u], i + u * NT);
+      }
+      if (i < n) {  // the last round: loads clamped into the half, only the elements inside it counted
         float4 x[QH];
 #pragma unroll
         for (int u = 0; u < QH; ++u) x[u] = lc[min(i + u * NT, n - 1)];
@@ -866,11 +885,11 @@ __global__ void __launch_bounds__(QP_NT, 2)
     if (rank == 0 && tid == 0) cr[0] = 0;
     const int e0 = (int)((0u - (uint32_t)(reinterpret_cast<uintptr_t>(cr + 1) >> 2)) & 3u);
     // local part of a tile: thread t's 8 table values (plus D at m's first index, zero past this
-    // half), their running sums in o[], and the inclusive warp scan of the threads' totals
-    auto tile_local = [&](int t0, const float4 xa, const float4 xb, uint32_t(&o)[8]) -> uint32_t {
+    // half), their running sums in o[], and the inclusive warp scan of the threads' totals.  FULL:
+    // the tile lies inside the half (known at compile time, so the common case has no predicates).
+    auto tile_local = [&](auto FULLc, int t0, const float4 xa, const float4 xb, uint32_t(&o)[8]) -> uint32_t {
+      constexpr bool FULL = decltype(FULLc)::value;
       const int j = t0 + 2 * tid;
-      const bool full = t0 + 2 * NT <= n;
-      const bool va = full || j < n, vb = full || j + 1 < n;
       o[0] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.x)));
       o[1] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.y)));
       o[2] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.z)));
@@ -884,7 +903,8 @@ __global__ void __launch_bounds__(QP_NT, 2)
 #pragma unroll
         for (int e = 0; e < 8; ++e) o[e] += dt == (uint32_t)e ? D : 0u;
       }
-      if (!full) {  // past the end of this half (the other half's elements or the row's end): nothing
+      if (!FULL) {  // past the end of this half (the other half's elements or the row's end): nothing
+        const bool va = j < n, vb = j + 1 < n;
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           o[e] = va ? o[e] : 0u;
@@ -901,68 +921,68 @@ __global__ void __launch_bounds__(QP_NT, 2)
       scan_step<16>(s);
       return s;
     };
-    // the tile's CDF entries o[] + base, written out
-    auto tile_store = [&](int t0, uint32_t(&o)[8], uint32_t base) {
+    // the tile's CDF entries o[] + base, written out.  E0 (compile time): the first of a lane's eight
+    // entries that starts a 16-byte quad.  A full tile: the lane's aligned quads (elements
+    // E0..E0+3 and E0+4..E0+7 of its eight, the second completed by the next lane's first E0) are
+    // staged per warp (chunk c of the warp block at slot c ^ ((c >> 3) & 1): no bank conflicts
+    // either way) so that each store instruction writes 512 contiguous bytes.  A partial tile:
+    // single stores.
+    auto tile_store = [&](auto FULLc, auto E0c, int t0, uint32_t(&o)[8], uint32_t base) {
+      constexpr bool FULL = decltype(FULLc)::value;
+      constexpr int E0 = decltype(E0c)::value;
       const int j = t0 + 2 * tid;
-      const bool full = t0 + 2 * NT <= n;
-      const bool va = full || j < n, vb = full || j + 1 < n;
-      const int v0 = 4 * (c0 + j);
+      uint32_t* dst = cr + 1 + 4 * (c0 + j);
 #pragma unroll
       for (int e = 0; e < 8; ++e) o[e] += base;
-      uint32_t* dst = cr + 1 + v0;
-      if (full) {
-        // this lane's aligned quads: elements e0..e0+3 and e0+4..e0+7 of its eight, the second
-        // completed by the next lane's first e0; staged per warp (chunk c of the warp block at
-        // slot c ^ ((c >> 3) & 1): no bank conflicts either way) so that each store instruction
-        // writes 512 contiguous bytes
-        uint4 q1, q2;
-        if (e0 == 0) {
-          q1 = make_uint4(o[0], o[1], o[2], o[3]);
-          q2 = make_uint4(o[4], o[5], o[6], o[7]);
-        } else {
-          const uint32_t n0 = __shfl_down_sync(0xffffffffu, o[0], 1);
-          const uint32_t n1 = __shfl_down_sync(0xffffffffu, o[1], 1);
-          const uint32_t n2 = __shfl_down_sync(0xffffffffu, o[2], 1);
-          if (e0 == 1) {
-            q1 = make_uint4(o[1], o[2], o[3], o[4]);
-            q2 = make_uint4(o[5], o[6], o[7], n0);
-          } else if (e0 == 2) {
-            q1 = make_uint4(o[2], o[3], o[4], o[5]);
-            q2 = make_uint4(o[6], o[7], n0, n1);
-          } else {
-            q1 = make_uint4(o[3], o[4], o[5], o[6]);
-            q2 = make_uint4(o[7], n0, n1, n2);
-          }
-          if (lane == 0) {  // the warp block's first e0 elements precede its first aligned quad
-#pragma unroll
-            for (int e = 0; e < 3; ++e)
-              if (e < e0) __stcs(dst + e, o[e]);
-          }
-        }
-        uint4* sb = stage + 64 * warp;
-        const int sw = (lane >> 2) & 1;
-        sb[(2 * lane) ^ sw] = q1;
-        sb[(2 * lane + 1) ^ sw] = q2;
-        __syncwarp();
-        const int rs = (lane >> 3) & 1;
-        const uint4 w0 = sb[lane ^ rs], w1 = sb[(32 + lane) ^ rs];
-        __syncwarp();
-        uint4* wq = reinterpret_cast<uint4*>(cr + 1 + 4 * (c0 + t0) + 256 * warp + e0);  // chunk 0
-        __stcs(wq + lane, w0);
-        if (lane < 31 || e0 == 0) {
-          __stcs(wq + 32 + lane, w1);
-        } else {  // chunk 63 runs e0 elements into the next warp block: its first 4 - e0 words only
-          uint32_t* t = reinterpret_cast<uint32_t*>(wq + 63);
-          __stcs(t, w1.x);
-          if (e0 < 3) __stcs(t + 1, w1.y);
-          if (e0 < 2) __stcs(t + 2, w1.z);
-        }
-      } else {
+      if (!FULL) {
+        const bool va = j < n, vb = j + 1 < n;
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           if (va) __stcs(dst + e, o[e]);
           if (vb) __stcs(dst + 4 + e, o[e + 4]);
         }
+        return;
+      }
+      uint4 q1, q2;
+      if (E0 == 0) {
+        q1 = make_uint4(o[0], o[1], o[2], o[3]);
+        q2 = make_uint4(o[4], o[5], o[6], o[7]);
+      } else {
+        const uint32_t n0 = __shfl_down_sync(0xffffffffu, o[0], 1);
+        const uint32_t n1 = E0 >= 2 ? __shfl_down_sync(0xffffffffu, o[1], 1) : 0u;
+        const uint32_t n2 = E0 >= 3 ? __shfl_down_sync(0xffffffffu, o[2], 1) : 0u;
+        if (E0 == 1) {
+          q1 = make_uint4(o[1], o[2], o[3], o[4]);
+          q2 = make_uint4(o[5], o[6], o[7], n0);
+        } else if (E0 == 2) {
+          q1 = make_uint4(o[2], o[3], o[4], o[5]);
+          q2 = make_uint4(o[6], o[7], n0, n1);
+        } else {
+          q1 = make_uint4(o[3], o[4], o[5], o[6]);
+          q2 = make_uint4(o[7], n0, n1, n2);
+        }
+        if (lane == 0) {  // the warp block's first E0 elements precede its first aligned quad
+#pragma unroll
+          for (int e = 0; e < E0; ++e) __stcs(dst + e, o[e]);
+        }
+      }
+      uint4* sb = stage + 64 * warp;
+      const int sw = (lane >> 2) & 1;
+      sb[(2 * lane) ^ sw] = q1;
+      sb[(2 * lane + 1) ^ sw] = q2;
+      __syncwarp();
+      const int rs = (lane >> 3) & 1;
+      const uint4 w0 = sb[lane ^ rs], w1 = sb[(32 + lane) ^ rs];
+      __syncwarp();
+      uint4* wq = reinterpret_cast<uint4*>(cr + 1 + 4 * (c0 + t0) + 256 * warp + E0);  // chunk 0
+      __stcs(wq + lane, w0);
+      if (E0 == 0 || lane < 31) {
+        __stcs(wq + 32 + lane, w1);
+      } else {  // chunk 63 runs E0 elements into the next warp block: its first 4 - E0 words only
+        uint32_t* t = reinterpret_cast<uint32_t*>(wq + 63);
+        __stcs(t, w1.x);
+        if (E0 < 3) __stcs(t + 1, w1.y);
+        if (E0 < 2) __stcs(t + 2, w1.z);
       }
     };
     // past the end of this half: m itself (d = 0, an in-range code; the values are dropped)
@@ -971,28 +991,57 @@ __global__ void __launch_bounds__(QP_NT, 2)
       if (i < n) x = __ldcs(lc + i);
       return x;
     };
-    // two tiles per barrier: their loads and local scans run side by side
-    int wb = 0;
-    for (int t0 = 0; t0 < n; t0 += 4 * NT) {
-      const int t1 = t0 + 2 * NT;  // the second tile (none past the end)
-      const float4 xa0 = ld4(t0 + 2 * tid), xb0 = ld4(t0 + 2 * tid + 1);
-      const float4 xa1 = ld4(t1 + 2 * tid), xb1 = ld4(t1 + 2 * tid + 1);
-      uint32_t oa[8], ob[8];
-      const uint32_t sa = tile_local(t0, xa0, xb0, oa);
-      const uint32_t sb = t1 < n ? tile_local(t1, xa1, xb1, ob) : 0u;
-      if (lane == 31) {
-        wsum[wb][0][warp] = sa;
-        wsum[wb][1][warp] = sb;
-      }
-      __syncthreads();
-      const uint32_t tva = lane < NW ? wsum[wb][0][lane] : 0u, tvb = lane < NW ? wsum[wb][1][lane] : 0u;
-      wb ^= 1;
-      tile_store(t0, oa, carry + __reduce_add_sync(0xffffffffu, lane < warp ? tva : 0u) + (sa - oa[7]));
-      carry += __reduce_add_sync(0xffffffffu, tva);
-      if (t1 < n) {
-        tile_store(t1, ob, carry + __reduce_add_sync(0xffffffffu, lane < warp ? tvb : 0u) + (sb - ob[7]));
+    // two tiles per barrier: their loads and local scans run side by side; the pairs inside the
+    // half first, then the last (partial) pair
+    auto pass3 = [&](auto E0c) {
+      const std::integral_constant<bool, true> full_c;
+      const std::integral_constant<bool, false> part_c;
+      int wb = 0;
+      auto combine = [&](uint32_t sa, uint32_t sb, uint32_t& ba, uint32_t& bb) {
+        if (lane == 31) {
+          wsum[wb][0][warp] = sa;
+          wsum[wb][1][warp] = sb;
+        }
+        __syncthreads();
+        const uint32_t tva = lane < NW ? wsum[wb][0][lane] : 0u, tvb = lane < NW ? wsum[wb][1][lane] : 0u;
+        wb ^= 1;
+        ba = carry + __reduce_add_sync(0xffffffffu, lane < warp ? tva : 0u);
+        carry += __reduce_add_sync(0xffffffffu, tva);
+        bb = carry + __reduce_add_sync(0xffffffffu, lane < warp ? tvb : 0u);
         carry += __reduce_add_sync(0xffffffffu, tvb);
+      };
+      int t0 = 0;
+      for (; t0 + 4 * NT <= n; t0 += 4 * NT) {
+        const int t1 = t0 + 2 * NT;
+        const float4 xa0 = __ldcs(lc + t0 + 2 * tid), xb0 = __ldcs(lc + t0 + 2 * tid + 1);
+        const float4 xa1 = __ldcs(lc + t1 + 2 * tid), xb1 = __ldcs(lc + t1 + 2 * tid + 1);
+        uint32_t oa[8], ob[8], ba, bb;
+        const uint32_t sa = tile_local(full_c, t0, xa0, xb0, oa);
+        const uint32_t sb = tile_local(full_c, t1, xa1, xb1, ob);
+        combine(sa, sb, ba, bb);
+        tile_store(full_c, E0c, t0, oa, ba + (sa - oa[7]));
+        tile_store(full_c, E0c, t1, ob, bb + (sb - ob[7]));
       }
+      if (t0 < n) {  // tile t0 may still be full; t1 is partial or past the end
+        const int t1 = t0 + 2 * NT;
+        const float4 xa0 = ld4(t0 + 2 * tid), xb0 = ld4(t0 + 2 * tid + 1);
+        const float4 xa1 = ld4(t1 + 2 * tid), xb1 = ld4(t1 + 2 * tid + 1);
+        uint32_t oa[8], ob[8], ba, bb;
+        const uint32_t sa = tile_local(part_c, t0, xa0, xb0, oa);
+        const uint32_t sb = tile_local(part_c, t1, xa1, xb1, ob);
+        combine(sa, sb, ba, bb);
+        if (t1 <= n)
+          tile_store(full_c, E0c, t0, oa, ba + (sa - oa[7]));
+        else
+          tile_store(part_c, E0c, t0, oa, ba + (sa - oa[7]));
+        if (t1 < n) tile_store(part_c, E0c, t1, ob, bb + (sb - ob[7]));
+      }
+    };
+    switch (e0) {
+      case 0: pass3(std::integral_constant<int, 0>()); break;
+      case 1: pass3(std::integral_constant<int, 1>()); break;
+      case 2: pass3(std::integral_constant<int, 2>()); break;
+      default: pass3(std::integral_constant<int, 3>()); break;
     }
   }
   cluster_sync_all();  // neither CTA leaves while the peer may still write to its shared memory
