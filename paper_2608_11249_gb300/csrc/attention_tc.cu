@@ -763,7 +763,7 @@ int attention_bf16_tc(const bf16* qkv, int ld, const void* vt, int n_chunks, int
   ProfScope prof(PROF_ATTN, s, 4.0 * n_chunks * nh * (double)L * L * hd, 2.0 * n_chunks * L * (double)(ld + d));
   if (hd == 128 && L % (2 * fa2::BQ) == 0) {
     // two query tiles per CTA, one CTA per SM (at head dim 64 the one-tile kernel, two CTAs per SM,
-    // measured faster: 37.6 against 40.1 ms per byte-model forward over 1024 windows of 512)
+    // measured faster: 38.9 against 39.2 ms per byte-model forward over 1024 windows of 512)
     const int64_t items2 = items / 2;
     const int grid = items2 < num_sms() ? (int)items2 : num_sms();
     constexpr int SM = fa2::Smem<128>::TOTAL;
