@@ -626,7 +626,6 @@ __global__ void __launch_bounds__(QP_NT, 2)
                          const float* __restrict__ pmax, const float* __restrict__ pmin, int npart) {
   constexpr int NT = QP_NT, NW = NT / 32, BPT = NQ / NT;
   __shared__ __align__(16) uint32_t tab[NQ];  // histogram of the codes, then 1 + floor(w R / W)
-  extern __shared__ uint4 stage[];             // CDF store staging, 64 16-byte chunks per warp
   __shared__ uint32_t T[256];
   __shared__ QPairSlot xs[2];
   __shared__ __align__(8) uint64_t xbar[2];
@@ -873,116 +872,134 @@ __global__ void __launch_bounds__(QP_NT, 2)
       __syncthreads();
       if (!s_ok) break;
     }
-    // ---- pass 3 (L2): CDF[v + 1] = sum_{u <= v} (1 + floor(w_u R / W) + (u == top ? D : 0)).  A tile is
-    // 2 NT float4s; thread t scans the 8 elements of float4s 2t, 2t + 1 in registers, then the warp
-    // and the CTA add their offsets.  Stores are aligned 16-byte quads (the row's entry 1 starts at
-    // word offset s mod 4; each lane writes the quad that starts in its own range, completed by the
-    // next lane's first elements; a warp's first and last lanes write their edges singly).
+    // ---- pass 3 (L2): CDF[v + 1] = sum_{u <= v} (1 + floor(w_u R / W) + (u == top ? D : 0)), in tiles
+    // of 2 NT float4s (layout below): running sums within each float4, warp scans of the float4
+    // totals, then the CTA's offsets (one barrier per two tiles).  The row's entry 1 starts at word
+    // offset e0 mod 4 from a 16-byte boundary; the pass is compiled once per e0.
     const uint32_t D = s_D;
     const int top = s_top;
     uint32_t carry = s_carry;
     uint32_t* cr = cdf + (size_t)r * (V + 1);
     if (rank == 0 && tid == 0) cr[0] = 0;
     const int e0 = (int)((0u - (uint32_t)(reinterpret_cast<uintptr_t>(cr + 1) >> 2)) & 3u);
-    // local part of a tile: thread t's 8 table values (plus D at m's first index, zero past this
-    // half), their running sums in o[], and the inclusive warp scan of the threads' totals.  FULL:
-    // the tile lies inside the half (known at compile time, so the common case has no predicates).
-    auto tile_local = [&](auto FULLc, int t0, const float4 xa, const float4 xb, uint32_t(&o)[8]) -> uint32_t {
+    // A tile is 2 NT float4s; warp w takes float4s [64 w, 64 w + 64) of it as two sub-blocks of 32,
+    // lane l float4s 64 w + l and 64 w + 32 + l, so loads and stores are 512 contiguous bytes per
+    // instruction.  tile_local: the lane's 8 table values (plus D at m's first index, zero past this
+    // half) as running sums within each float4, the warp's scans of the float4 totals, and the
+    // exclusive offsets ex0 / ex1 of the lane's two float4s inside the warp's 256 elements; returns
+    // the warp's total.  FULL: the tile lies inside the half (known at compile time).
+    auto tile_local = [&](auto FULLc, int t0, const float4 x0, const float4 x1, uint32_t(&o)[8], uint32_t& ex0,
+                          uint32_t& ex1) -> uint32_t {
       constexpr bool FULL = decltype(FULLc)::value;
-      const int j = t0 + 2 * tid;
-      o[0] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.x)));
-      o[1] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.y)));
-      o[2] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.z)));
-      o[3] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xa.w)));
-      o[4] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.x)));
-      o[5] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.y)));
-      o[6] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.z)));
-      o[7] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, xb.w)));
-      const uint32_t dt = (uint32_t)(top - 4 * (c0 + j));
-      if (dt < 8u) {
+      const int j0 = t0 + 64 * warp + lane, j1 = j0 + 32;
+      o[0] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x0.x)));
+      o[1] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x0.y)));
+      o[2] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x0.z)));
+      o[3] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x0.w)));
+      o[4] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x1.x)));
+      o[5] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x1.y)));
+      o[6] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x1.z)));
+      o[7] = lds_code(tabq, pair_code<PART>(__fsub_rn(m, x1.w)));
+      const uint32_t dt0 = (uint32_t)(top - 4 * (c0 + j0)), dt1 = (uint32_t)(top - 4 * (c0 + j1));
+      if (dt0 < 4u) {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) o[e] += dt == (uint32_t)e ? D : 0u;
+        for (int e = 0; e < 4; ++e) o[e] += dt0 == (uint32_t)e ? D : 0u;
+      }
+      if (dt1 < 4u) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[4 + e] += dt1 == (uint32_t)e ? D : 0u;
       }
       if (!FULL) {  // past the end of this half (the other half's elements or the row's end): nothing
-        const bool va = j < n, vb = j + 1 < n;
+        const bool v0 = j0 < n, v1 = j1 < n;
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          o[e] = va ? o[e] : 0u;
-          o[e + 4] = vb ? o[e + 4] : 0u;
+          o[e] = v0 ? o[e] : 0u;
+          o[e + 4] = v1 ? o[e + 4] : 0u;
         }
       }
 #pragma unroll
-      for (int e = 1; e < 8; ++e) o[e] += o[e - 1];
-      uint32_t s = o[7];
-      scan_step<1>(s);
-      scan_step<2>(s);
-      scan_step<4>(s);
-      scan_step<8>(s);
-      scan_step<16>(s);
-      return s;
+      for (int e = 1; e < 4; ++e) {
+        o[e] += o[e - 1];
+        o[4 + e] += o[3 + e];
+      }
+      uint32_t s0 = o[3], s1 = o[7];
+      scan_step<1>(s0);
+      scan_step<1>(s1);
+      scan_step<2>(s0);
+      scan_step<2>(s1);
+      scan_step<4>(s0);
+      scan_step<4>(s1);
+      scan_step<8>(s0);
+      scan_step<8>(s1);
+      scan_step<16>(s0);
+      scan_step<16>(s1);
+      const uint32_t t0tot = __shfl_sync(0xffffffffu, s0, 31), t1tot = __shfl_sync(0xffffffffu, s1, 31);
+      ex0 = s0 - o[3];
+      ex1 = t0tot + s1 - o[7];
+      return t0tot + t1tot;
     };
-    // the tile's CDF entries o[] + base, written out.  E0 (compile time): the first of a lane's eight
-    // entries that starts a 16-byte quad.  A full tile: the lane's aligned quads (elements
-    // E0..E0+3 and E0+4..E0+7 of its eight, the second completed by the next lane's first E0) are
-    // staged per warp (chunk c of the warp block at slot c ^ ((c >> 3) & 1): no bank conflicts
-    // either way) so that each store instruction writes 512 contiguous bytes.  A partial tile:
-    // single stores.
-    auto tile_store = [&](auto FULLc, auto E0c, int t0, uint32_t(&o)[8], uint32_t base) {
+    // the tile's CDF entries o[] + offsets, written out.  E0 (compile time): the first entry of a
+    // float4 that starts a 16-byte quad.  Full tiles: each lane stores the quads that start at its
+    // float4s' entry E0, completed by the next lane's first E0 entries (lane 31 of the first
+    // sub-block by lane 0 of the second); a warp's first E0 entries and the tail of its last quad,
+    // which the next warp completes, go singly.  Partial tiles: single stores.
+    auto tile_store = [&](auto FULLc, auto E0c, int t0, uint32_t(&o)[8], uint32_t b0, uint32_t b1) {
       constexpr bool FULL = decltype(FULLc)::value;
       constexpr int E0 = decltype(E0c)::value;
-      const int j = t0 + 2 * tid;
-      uint32_t* dst = cr + 1 + 4 * (c0 + j);
+      const int j0 = t0 + 64 * warp + lane, j1 = j0 + 32;
+      uint32_t* d0 = cr + 1 + 4 * (c0 + j0);
+      uint32_t* d1 = d0 + 128;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) o[e] += base;
+      for (int e = 0; e < 4; ++e) {
+        o[e] += b0;
+        o[4 + e] += b1;
+      }
       if (!FULL) {
-        const bool va = j < n, vb = j + 1 < n;
+        const bool v0 = j0 < n, v1 = j1 < n;
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          if (va) __stcs(dst + e, o[e]);
-          if (vb) __stcs(dst + 4 + e, o[e + 4]);
+          if (v0) __stcs(d0 + e, o[e]);
+          if (v1) __stcs(d1 + e, o[4 + e]);
         }
         return;
       }
-      uint4 q1, q2;
       if (E0 == 0) {
-        q1 = make_uint4(o[0], o[1], o[2], o[3]);
-        q2 = make_uint4(o[4], o[5], o[6], o[7]);
-      } else {
-        const uint32_t n0 = __shfl_down_sync(0xffffffffu, o[0], 1);
-        const uint32_t n1 = E0 >= 2 ? __shfl_down_sync(0xffffffffu, o[1], 1) : 0u;
-        const uint32_t n2 = E0 >= 3 ? __shfl_down_sync(0xffffffffu, o[2], 1) : 0u;
-        if (E0 == 1) {
-          q1 = make_uint4(o[1], o[2], o[3], o[4]);
-          q2 = make_uint4(o[5], o[6], o[7], n0);
-        } else if (E0 == 2) {
-          q1 = make_uint4(o[2], o[3], o[4], o[5]);
-          q2 = make_uint4(o[6], o[7], n0, n1);
-        } else {
-          q1 = make_uint4(o[3], o[4], o[5], o[6]);
-          q2 = make_uint4(o[7], n0, n1, n2);
-        }
-        if (lane == 0) {  // the warp block's first E0 elements precede its first aligned quad
+        __stcs(reinterpret_cast<uint4*>(d0), make_uint4(o[0], o[1], o[2], o[3]));
+        __stcs(reinterpret_cast<uint4*>(d1), make_uint4(o[4], o[5], o[6], o[7]));
+        return;
+      }
+      const int nl = (lane + 1) & 31;
+      uint32_t y[3], z[3];
 #pragma unroll
-          for (int e = 0; e < E0; ++e) __stcs(dst + e, o[e]);
+      for (int e = 0; e < 3; ++e) {
+        if (e < E0) {
+          y[e] = __shfl_sync(0xffffffffu, o[e], nl);
+          z[e] = __shfl_sync(0xffffffffu, o[4 + e], nl);
+          if (lane == 31) y[e] = z[e];  // the first sub-block's last float4 continues into the second's first
         }
       }
-      uint4* sb = stage + 64 * warp;
-      const int sw = (lane >> 2) & 1;
-      sb[(2 * lane) ^ sw] = q1;
-      sb[(2 * lane + 1) ^ sw] = q2;
-      __syncwarp();
-      const int rs = (lane >> 3) & 1;
-      const uint4 w0 = sb[lane ^ rs], w1 = sb[(32 + lane) ^ rs];
-      __syncwarp();
-      uint4* wq = reinterpret_cast<uint4*>(cr + 1 + 4 * (c0 + t0) + 256 * warp + E0);  // chunk 0
-      __stcs(wq + lane, w0);
-      if (E0 == 0 || lane < 31) {
-        __stcs(wq + 32 + lane, w1);
-      } else {  // chunk 63 runs E0 elements into the next warp block: its first 4 - E0 words only
-        uint32_t* t = reinterpret_cast<uint32_t*>(wq + 63);
-        __stcs(t, w1.x);
-        if (E0 < 3) __stcs(t + 1, w1.y);
-        if (E0 < 2) __stcs(t + 2, w1.z);
+      if (E0 == 1) {
+        __stcs(reinterpret_cast<uint4*>(d0 + 1), make_uint4(o[1], o[2], o[3], y[0]));
+      } else if (E0 == 2) {
+        __stcs(reinterpret_cast<uint4*>(d0 + 2), make_uint4(o[2], o[3], y[0], y[1]));
+      } else {
+        __stcs(reinterpret_cast<uint4*>(d0 + 3), make_uint4(o[3], y[0], y[1], y[2]));
+      }
+      if (lane < 31) {
+        if (E0 == 1) {
+          __stcs(reinterpret_cast<uint4*>(d1 + 1), make_uint4(o[5], o[6], o[7], z[0]));
+        } else if (E0 == 2) {
+          __stcs(reinterpret_cast<uint4*>(d1 + 2), make_uint4(o[6], o[7], z[0], z[1]));
+        } else {
+          __stcs(reinterpret_cast<uint4*>(d1 + 3), make_uint4(o[7], z[0], z[1], z[2]));
+        }
+      } else {  // the warp block's last quad runs into the next warp's block: this lane's part only
+#pragma unroll
+        for (int e = E0; e < 4; ++e) __stcs(d1 + e, o[4 + e]);
+      }
+      if (lane == 0) {  // the warp block's first E0 entries precede its first aligned quad
+#pragma unroll
+        for (int e = 0; e < E0; ++e) __stcs(d0 + e, o[e]);
       }
     };
     // past the end of this half: m itself (d = 0, an in-range code; the values are dropped)
@@ -998,7 +1015,7 @@ __global__ void __launch_bounds__(QP_NT, 2)
       const std::integral_constant<bool, false> part_c;
       int wb = 0;
       auto combine = [&](uint32_t sa, uint32_t sb, uint32_t& ba, uint32_t& bb) {
-        if (lane == 31) {
+        if (lane == 0) {
           wsum[wb][0][warp] = sa;
           wsum[wb][1][warp] = sb;
         }
@@ -1013,28 +1030,30 @@ __global__ void __launch_bounds__(QP_NT, 2)
       int t0 = 0;
       for (; t0 + 4 * NT <= n; t0 += 4 * NT) {
         const int t1 = t0 + 2 * NT;
-        const float4 xa0 = __ldcs(lc + t0 + 2 * tid), xb0 = __ldcs(lc + t0 + 2 * tid + 1);
-        const float4 xa1 = __ldcs(lc + t1 + 2 * tid), xb1 = __ldcs(lc + t1 + 2 * tid + 1);
-        uint32_t oa[8], ob[8], ba, bb;
-        const uint32_t sa = tile_local(full_c, t0, xa0, xb0, oa);
-        const uint32_t sb = tile_local(full_c, t1, xa1, xb1, ob);
+        const int jw = 64 * warp + lane;
+        const float4 xa0 = __ldcs(lc + t0 + jw), xb0 = __ldcs(lc + t0 + jw + 32);
+        const float4 xa1 = __ldcs(lc + t1 + jw), xb1 = __ldcs(lc + t1 + jw + 32);
+        uint32_t oa[8], ob[8], ea0, ea1, eb0, eb1, ba, bb;
+        const uint32_t sa = tile_local(full_c, t0, xa0, xb0, oa, ea0, ea1);
+        const uint32_t sb = tile_local(full_c, t1, xa1, xb1, ob, eb0, eb1);
         combine(sa, sb, ba, bb);
-        tile_store(full_c, E0c, t0, oa, ba + (sa - oa[7]));
-        tile_store(full_c, E0c, t1, ob, bb + (sb - ob[7]));
+        tile_store(full_c, E0c, t0, oa, ba + ea0, ba + ea1);
+        tile_store(full_c, E0c, t1, ob, bb + eb0, bb + eb1);
       }
       if (t0 < n) {  // tile t0 may still be full; t1 is partial or past the end
         const int t1 = t0 + 2 * NT;
-        const float4 xa0 = ld4(t0 + 2 * tid), xb0 = ld4(t0 + 2 * tid + 1);
-        const float4 xa1 = ld4(t1 + 2 * tid), xb1 = ld4(t1 + 2 * tid + 1);
-        uint32_t oa[8], ob[8], ba, bb;
-        const uint32_t sa = tile_local(part_c, t0, xa0, xb0, oa);
-        const uint32_t sb = tile_local(part_c, t1, xa1, xb1, ob);
+        const int jw = 64 * warp + lane;
+        const float4 xa0 = ld4(t0 + jw), xb0 = ld4(t0 + jw + 32);
+        const float4 xa1 = ld4(t1 + jw), xb1 = ld4(t1 + jw + 32);
+        uint32_t oa[8], ob[8], ea0, ea1, eb0, eb1, ba, bb;
+        const uint32_t sa = tile_local(part_c, t0, xa0, xb0, oa, ea0, ea1);
+        const uint32_t sb = tile_local(part_c, t1, xa1, xb1, ob, eb0, eb1);
         combine(sa, sb, ba, bb);
         if (t1 <= n)
-          tile_store(full_c, E0c, t0, oa, ba + (sa - oa[7]));
+          tile_store(full_c, E0c, t0, oa, ba + ea0, ba + ea1);
         else
-          tile_store(part_c, E0c, t0, oa, ba + (sa - oa[7]));
-        if (t1 < n) tile_store(part_c, E0c, t1, ob, bb + (sb - ob[7]));
+          tile_store(part_c, E0c, t0, oa, ba + ea0, ba + ea1);
+        if (t1 < n) tile_store(part_c, E0c, t1, ob, bb + eb0, bb + eb1);
       }
     };
     switch (e0) {
@@ -1048,13 +1067,10 @@ __global__ void __launch_bounds__(QP_NT, 2)
 }
 
 // clusters of quantize_pair_kernel that fit on the device at once (0: the launch shape is unavailable)
-constexpr int QP_STAGE_BYTES = QP_NT / 32 * 64 * 16;  // dynamic shared memory (static part ~34 KB)
-
 static cudaLaunchConfig_t pair_config(int grid, cudaStream_t s, cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(QP_NT);
-  cfg.dynamicSmemBytes = QP_STAGE_BYTES;
   cfg.stream = s;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
@@ -1073,12 +1089,7 @@ static int pair_clusters() {
     cudaLaunchAttribute attr[1];
     const cudaLaunchConfig_t cfg = pair_config(2 * 2 * num_sms(), 0, attr);
     int c = 0;
-    // static + dynamic shared memory exceeds the 48 KB default
-    if (cudaFuncSetAttribute(quantize_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             QP_STAGE_BYTES) != cudaSuccess ||
-        cudaFuncSetAttribute(quantize_pair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             QP_STAGE_BYTES) != cudaSuccess ||
-        cudaOccupancyMaxActiveClusters(&c, quantize_pair_kernel<false>, &cfg) != cudaSuccess || c < 1) {
+    if (cudaOccupancyMaxActiveClusters(&c, quantize_pair_kernel<false>, &cfg) != cudaSuccess || c < 1) {
       cudaGetLastError();
       c = -1;
     }
