@@ -320,6 +320,14 @@ DLMZ_API int dlmz_check(void* stream);
  * pipeline wait is; the device error word is cleared and the context stays
  * usable.  Errors: EINVAL (limit), ECUDA. */
 DLMZ_API int dlmz_selftest_wait_timeout(uint32_t limit_us, void* stream);
+/* The same for the cluster-scope wait of the quantiser's CTA pairs: a cluster
+ * of two CTAs, CTA 0 waits (limit_us, 1 .. 1e6) on its mbarrier for one
+ * arrival that CTA 1 makes through distributed shared memory only when
+ * peer_arrives is 1.  Returns DLMZ_OK when the wait completed (peer_arrives
+ * 1), DLMZ_ETIMEOUT when it gave up (peer_arrives 0); the device error word
+ * is cleared and the context stays usable.  Errors: EINVAL (limit,
+ * peer_arrives > 1), ECUDA. */
+DLMZ_API int dlmz_selftest_cluster_wait(uint32_t limit_us, uint32_t peer_arrives, void* stream);
 
 /* ---- live profiling (not part of the method) ------------------------------
  * Between dlmz_profile_begin and dlmz_profile_end the library records CUDA

@@ -91,6 +91,7 @@ _sig("dlmz_model_decode_step", c_int, _P, _P, POINTER(KPolicy), c_uint32, c_uint
 _sig("dlmz_coder_capacity_units", c_uint32, _P)
 _sig("dlmz_check", c_int, _P)
 _sig("dlmz_selftest_wait_timeout", c_int, c_uint32, _P)
+_sig("dlmz_selftest_cluster_wait", c_int, c_uint32, c_uint32, _P)
 _sig("dlmz_profile_begin", c_int)
 _sig("dlmz_profile_end", c_int, POINTER(Profile))
 _sig("dlmz_launch_count", c_uint64)
@@ -235,6 +236,11 @@ def check(stream=0):
 def selftest_wait_timeout(limit_us, stream=0):
     """Return code of dlmz_selftest_wait_timeout (DLMZ_ETIMEOUT when the bounded wait gave up)."""
     return lib.dlmz_selftest_wait_timeout(limit_us, stream)
+
+
+def selftest_cluster_wait(limit_us, peer_arrives, stream=0):
+    """Return code of dlmz_selftest_cluster_wait (OK when the peer CTA arrived, ETIMEOUT when not)."""
+    return lib.dlmz_selftest_cluster_wait(limit_us, peer_arrives, stream)
 
 
 class Coder:

@@ -30,6 +30,20 @@ def test_bounded_wait_times_out_and_context_stays_usable(dev):
     assert float((D.double() - ref).abs().max()) < 1e-3
 
 
+def test_cluster_wait_times_out_only_without_the_peer(dev):
+    """The cluster-scope bounded wait of the quantiser's CTA pairs: it completes when the other CTA
+    of the cluster arrives through distributed shared memory and gives up (ETIMEOUT, context
+    usable) when it does not."""
+    d = dlmz()
+    assert d.selftest_cluster_wait(1000, 1) == 0
+    assert d.selftest_cluster_wait(1000, 0) == d.ETIMEOUT
+    assert d.selftest_cluster_wait(200, 0) == d.ETIMEOUT
+    assert d.selftest_cluster_wait(1000, 1) == 0
+    d.check()
+    assert d.selftest_cluster_wait(0, 0) == d.EINVAL
+    assert d.selftest_cluster_wait(1000, 2) == d.EINVAL
+
+
 def test_selftest_rejects_bad_limits(dev):
     d = dlmz()
     assert d.selftest_wait_timeout(0) == d.EINVAL
