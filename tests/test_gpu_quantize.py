@@ -21,7 +21,10 @@ def _rows(V, n, seed):
 @pytest.mark.parametrize("V,n", [(2, 9), (4, 33), (37, 70), (256, 300), (300, 50), (512, 40), (1000, 20), (1001, 7),
                                  (5000, 17), (126464, 5), (152064, 3),
                                  # more rows than SMs: each CTA of the large-vocabulary kernel walks several rows
-                                 (1000, 1300), (4100, 700)])
+                                 (1000, 1300), (4100, 700),
+                                 # the smallest halves of the two-CTA kernel (V = 516: 65 and 64 float4s)
+                                 # and a vocabulary whose rows start at every word offset modulo 4
+                                 (516, 11), (1028, 9)])
 def test_quantize_bit_exact(dev, V, n):
     import torch
     d = dlmz()
